@@ -1,0 +1,143 @@
+"""Pins of the oracle's worker gradient and end-to-end simulation.
+
+The gradient (the worker's dtheta = -eta grad L(s), notation table) is pinned by central
+finite differences in double, by the closed form at zero weights, and the TF32 operand
+rounding by hand-worked bit patterns.  The simulation's wiring is pinned by its
+reduction to plain SGD for one worker without momentum.
+"""
+import math
+
+import numpy as np
+import pytest
+
+import oracle
+from paper_1805_08469_gb300 import synth
+
+
+def _loss(dims, theta, X, y):
+    return oracle.mlp_loss_grad(dims, theta, X, y)[0]
+
+
+def _fd_check(dims, theta, X, y, coords, h=1e-6, rtol=1e-6):
+    _, g = oracle.mlp_loss_grad(dims, theta, X, y)
+    for j in coords:
+        tp = theta.copy()
+        tm = theta.copy()
+        tp[j] += h
+        tm[j] -= h
+        fd = (_loss(dims, tp, X, y) - _loss(dims, tm, X, y)) / (2 * h)
+        assert abs(fd - g[j]) <= rtol * max(1.0, abs(g[j])) + 1e-9, (j, fd, g[j])
+    return g
+
+
+def test_finite_differences_tiny_mlp():
+    rng = np.random.default_rng(21)
+    dims = [5, 4, 3]
+    P = synth.mlp_param_count(dims)
+    theta = rng.standard_normal(P)
+    X = rng.standard_normal((6, 5))
+    y = rng.integers(0, 3, 6)
+    g = _fd_check(dims, theta, X, y, range(P))
+    assert np.abs(g).max() > 1e-3
+
+
+def test_finite_differences_deeper_mlp():
+    rng = np.random.default_rng(22)
+    dims = [7, 6, 5, 4]
+    P = synth.mlp_param_count(dims)
+    theta = 0.7 * rng.standard_normal(P)
+    X = rng.standard_normal((9, 7))
+    y = rng.integers(0, 4, 9)
+    _fd_check(dims, theta, X, y, range(P))
+
+
+def test_finite_differences_mnist_shaped_subset():
+    dims = [784, 64, 10]
+    theta = synth.xavier_theta0(5, dims).astype(np.float64)
+    lay = synth.mlp_layout(dims)
+    rng = np.random.default_rng(23)
+    # non-zero biases so that every parameter block is exercised
+    for (_wo, bo, fo, _fi) in lay:
+        theta[bo:bo + fo] = 0.1 * rng.standard_normal(fo)
+    rows = np.arange(8)
+    X = synth.data_rows(1, rows, 784).astype(np.float64)
+    y = synth.teacher_labels(1, rows, 784, 10)
+    coords = []
+    for (wo, bo, fo, fi) in lay:
+        coords += list(rng.choice(np.arange(wo, wo + fo * fi), 25, replace=False))
+        coords += list(rng.choice(np.arange(bo, bo + fo), 5, replace=False))
+    _fd_check(dims, theta, X, y, coords, h=1e-5, rtol=1e-5)
+
+
+def test_zero_weights_closed_form():
+    # All parameters zero: the logits are 0, the softmax is uniform, the loss is ln C, the
+    # last bias gradient is mean(1/C - onehot(y)) and every other gradient vanishes
+    # (hidden activations are ReLU(0) = 0).
+    dims = [6, 5, 4]
+    P = synth.mlp_param_count(dims)
+    rng = np.random.default_rng(24)
+    X = rng.standard_normal((10, 6))
+    y = rng.integers(0, 4, 10)
+    loss, g = oracle.mlp_loss_grad(dims, np.zeros(P), X, y)
+    assert math.isclose(loss, math.log(4), rel_tol=1e-15)
+    lay = synth.mlp_layout(dims)
+    _wo, bo, fo, _fi = lay[-1]
+    expect = np.full(4, 0.25) - np.bincount(y, minlength=4) / 10
+    np.testing.assert_allclose(g[bo:bo + fo], expect, atol=1e-15)
+    mask = np.ones(P, bool)
+    mask[bo:bo + fo] = False
+    assert np.all(g[mask] == 0)
+
+
+def test_tf32_round_to_nearest_ties_away():
+    one = 1.0
+    assert oracle.tf32_rna(one + 2.0 ** -10) == one + 2.0 ** -10          # representable
+    assert oracle.tf32_rna(one + 2.0 ** -11) == one + 2.0 ** -10          # tie -> away
+    assert oracle.tf32_rna(-(one + 2.0 ** -11)) == -(one + 2.0 ** -10)    # sign-symmetric
+    assert oracle.tf32_rna(one + 2.0 ** -11 - 2.0 ** -23) == one          # below the tie
+    assert oracle.tf32_rna(one + 3 * 2.0 ** -11) == one + 2.0 ** -9       # tie -> away (up)
+    assert oracle.tf32_rna(2.0 - 2.0 ** -11) == 2.0                       # carry into exponent
+    assert oracle.tf32_rna(0.0) == 0.0
+
+
+def test_tf32_mode_leaves_exact_single_layer_forward_unchanged():
+    # With TF32-representable inputs and weights, a single layer's forward product is
+    # unchanged by operand rounding, so the loss is the same in both modes.
+    rng = np.random.default_rng(25)
+    dims = [12, 5]
+    P = synth.mlp_param_count(dims)
+    theta = np.round(rng.standard_normal(P) * 64) / 64
+    X = np.round(rng.standard_normal((7, 12)) * 64) / 64
+    y = rng.integers(0, 5, 7)
+    l0, g0 = oracle.mlp_loss_grad(dims, theta, X, y)
+    l1, g1 = oracle.mlp_loss_grad(dims, theta, X, y, tf32=True)
+    assert l0 == l1
+    # backward operands carry TF32's relative rounding of 2**-11 each
+    np.testing.assert_allclose(g1, g0, rtol=0, atol=2e-3 * np.abs(g0).max())
+    assert not np.array_equal(g0, g1)  # the backward operands are rounded
+
+
+def test_simulation_single_worker_without_momentum_is_minibatch_sgd():
+    dims = [784, 16, 10]
+    P = synth.mlp_param_count(dims)
+    T, b, eta = 12, 8, 0.05
+    theta0 = synth.xavier_theta0(7, dims)
+    order = np.zeros(T, dtype=np.int32)
+    batches = synth.schedule_batches(7, order, b)
+    rows, inv = np.unique(batches, return_inverse=True)
+    X = synth.data_rows(7, rows, 784)
+    labels = synth.teacher_labels(7, rows, 784, 10)
+    local = inv.reshape(batches.shape).astype(np.int32)
+    theta = theta0.copy()
+    m = np.zeros((1, P), np.float32)
+    s = theta0.copy()[None, :]
+    rec, losses = oracle.mlp_sim_run(dims, theta, m, s, order, X, labels, local, eta=eta,
+                                     mu=0.0, eps=1e-30, record_at=range(T), want_losses=True)
+    ref = theta0.copy()
+    for t in range(T):
+        loss, g = oracle.mlp_loss_grad(dims, ref.astype(np.float64), X[local[t]], labels[local[t]])
+        assert loss == losses[t]
+        g32 = g.astype(np.float32)
+        # plain SGD step in fp32; coordinates with a zero gradient are untouched
+        ref = ref - np.float32(eta) * g32
+        assert np.array_equal(rec[t], ref)
