@@ -1,0 +1,375 @@
+"""Benchmark of the GEM commit path on GB300.
+
+Workload (one step = one pass of the commit path over one batch): P = 25,000,000 fp32
+parameters (ResNet-50-sized), n = 100 workers, a batch of 100 commits in seeded
+uniform-tick order, each with a gradient from a pool of 100 synthetic heavy-tailed
+gradients (N(0, 1e-4) on 90% of coordinates, 0.01 Student-t(3) on a fixed 10%) held in
+HBM.  The working set (theta, m and s of 100 workers, the pool: about 30 GB) is far larger
+than L2, so no flush is needed between steps.
+
+Metric: algorithmic HBM GB/s of the commit path, 20 bytes per parameter and commit
+(g, m_w, s_w read; m_w, s_w written) plus 8 bytes per parameter and batch (theta read and
+written once), and the matching commits/s.
+
+Usage: python bench.py [--gpus N] [--steps K] [--warmup W] [--impl gem|reference]
+For N > 1 run under torch.distributed.run: every rank runs an independent replica on its
+own GPU (no collective on the data path); the timing takes the max over ranks.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+from pathlib import Path
+
+ROOT = Path(__file__).resolve().parent
+sys.path.insert(0, str(ROOT))
+
+METRIC = "GEM commit GB/s (% of HBM peak) at P=25M,n=100; async MLP commits/sec"
+P_FULL = 25_000_000
+N_WORKERS = 100
+K_BATCH = 100
+POOL_ROWS = 100
+SEED = 5
+ETA, MU, EPS = 0.01, 0.9, 1e-8
+BYTES_PER_BATCH = P_FULL * (20 * K_BATCH + 8)
+FALLBACK_HBM_GBS = 6800.0
+
+# DRAM traffic of one launch of the batched commit kernel, from an ncu capture of the
+# same workload (see profiles/commit_batch_p25m_n100.md).  Valid only for the kernel
+# source it was taken on; reported as null once that source changes.
+NCU_TRAFFIC_BYTES_PER_LAUNCH = None
+NCU_TRAFFIC_SOURCE_SHA = None
+
+
+def kernel_source_sha() -> str:
+    src = ROOT / "paper_1805_08469_gb300" / "csrc" / "gem_commit.cu"
+    return hashlib.sha256(src.read_bytes()).hexdigest()[:16]
+
+
+def measured_peaks() -> tuple[float, str]:
+    f = ROOT / "MEASURED_PEAKS.json"
+    try:
+        d = json.loads(f.read_text())
+        return float(d["hbm_gbs"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi clock and throttle-reason samples taken during the timed region."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_index: int):
+        self.dev = device_index
+        self.proc = None
+        self.lines: list[str] = []
+        self.thread = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.dev), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except Exception:
+            self.proc = None
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+            if self.thread:
+                self.thread.join(timeout=2)
+
+    def summary(self) -> dict:
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in self.lines:
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                mx.append(float(parts[2]))
+            except ValueError:
+                continue
+            for name, val in zip(names, parts[5:9]):
+                if val.lower() == "active":
+                    reasons.add(name)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def dist_setup():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    pg = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("gloo")
+        pg = dist
+    return world, rank, local, pg
+
+
+def max_over_ranks(pg, value: float) -> float:
+    if pg is None:
+        return value
+    import torch
+    t = torch.tensor([value], dtype=torch.float64)
+    pg.all_reduce(t, op=pg.ReduceOp.MAX)
+    return float(t.item())
+
+
+def barrier(pg):
+    if pg is not None:
+        pg.barrier()
+
+
+# ------------------------------------------------------------------------- CPU oracle
+
+ORACLE_SAMPLE = 250_000
+
+
+class OracleSample:
+    """The oracle's commit loop on coordinates [0, S) of the workload: inputs drawn once by
+    the host generators, state carried from one timed run to the next."""
+
+    def __init__(self, S: int, seed: int, max_batches: int = 200):
+        import numpy as np
+
+        import oracle
+        from paper_1805_08469_gb300 import synth
+
+        self.S = S
+        self.order, _ = oracle.schedule_uniform(seed, N_WORKERS, max_batches * K_BATCH)
+        cols = np.arange(S)
+        self.theta = synth.theta0_flat(seed, cols)
+        self.pool = np.stack([synth.grad_heavytail(seed, r, cols) for r in range(POOL_ROWS)])
+        self.m = np.zeros((N_WORKERS, S), np.float32)
+        self.s = np.tile(self.theta, (N_WORKERS, 1))
+        self.next = 0
+        oracle.lib()
+
+    def run(self, batches: int) -> float:
+        """Time `batches` batches of K_BATCH commits; returns seconds."""
+        import numpy as np
+
+        import oracle
+
+        t0, t1 = self.next * K_BATCH, (self.next + batches) * K_BATCH
+        if t1 > len(self.order):
+            self.next, t0, t1 = 0, 0, batches * K_BATCH
+        order = self.order[t0:t1]
+        gidx = np.arange(t0, t1) % POOL_ROWS
+        start = time.perf_counter()
+        oracle.gem_run(self.theta, self.m, self.s, self.pool, order, grad_index=gidx,
+                       eta=ETA, mu=MU, eps=EPS)
+        dt = time.perf_counter() - start
+        self.next += batches
+        return dt
+
+
+def cpu_baseline(seconds_target: float = 15.0) -> dict:
+    import oracle
+    sample = OracleSample(ORACLE_SAMPLE, SEED)
+    dt1 = sample.run(1)
+    batches = max(1, min(150, int(seconds_target / max(dt1, 1e-3))))
+    dt = sample.run(batches)
+    S, T = ORACLE_SAMPLE, batches * K_BATCH
+    gbs = S * (20 * T + 8 * batches) / dt / 1e9
+    return {"value": round(gbs, 3), "unit": "GB/s", "cores": 1, "kind": "oracle",
+            "sample": f"coordinates [0, {S}) of P={P_FULL}, n={N_WORKERS}: {batches} batches of "
+                      f"{K_BATCH} commits in {dt:.1f} s; same algorithmic bytes per coordinate",
+            "commits_per_s_scaled_to_P": round(T / dt * S / P_FULL, 3),
+            "oracle_threads_available": oracle.threads()}
+
+
+def run_reference(args, world, rank, pg):
+    """Reference arm: the oracle as it stands, on the host cores, one bounded sample per step."""
+    if rank != 0:
+        return
+    S = ORACLE_SAMPLE
+    sample = OracleSample(S, SEED, max_batches=args.warmup + args.steps + 1)
+    for _ in range(args.warmup):
+        sample.run(1)
+    total = sum(sample.run(1) for _ in range(args.steps))
+    gbs = S * (20 * K_BATCH + 8) * args.steps / total / 1e9
+    line = {
+        "impl": "reference", "metric": METRIC, "value": round(gbs, 3), "unit": "GB/s",
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": round(1e3 * total / args.steps, 3), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "config": {"workload": "gem_commit_batch P=25M n=100, batches of 100 commits, heavy-tailed gradient pool",
+                   "P": P_FULL, "n": N_WORKERS, "commits_per_step": K_BATCH,
+                   "sample": f"coordinates [0, {S}) per step"},
+        "cpu_baseline": {"value": round(gbs, 3), "unit": "GB/s", "cores": 1, "kind": "oracle",
+                         "sample": f"coordinates [0, {S}) of P={P_FULL}, one batch of {K_BATCH} commits per step"},
+        "e2e": {"value": round(gbs, 3), "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+# ------------------------------------------------------------------------- GPU arm
+
+def run_gem(args, world, rank, local, pg):
+    import torch
+
+    from paper_1805_08469_gb300 import gem, sim, synth_gpu
+
+    global P_FULL, N_WORKERS, K_BATCH, POOL_ROWS, BYTES_PER_BATCH
+    P_FULL, N_WORKERS, K_BATCH, POOL_ROWS = args.P, args.workers, args.batch, args.pool
+    BYTES_PER_BATCH = P_FULL * (20 * K_BATCH + 8)
+    torch.cuda.set_device(local)
+    seed = SEED + rank
+    stream = torch.cuda.Stream()
+    steps_total = args.warmup + args.steps
+    order, _ = sim.gem_schedule_uniform(seed, N_WORKERS, steps_total * K_BATCH)
+
+    with torch.cuda.stream(stream):
+        G = gem.Gem(P_FULL, N_WORKERS, ETA, MU, EPS, stream=stream)
+        theta0 = synth_gpu.theta0_flat(seed, torch.empty(P_FULL, device="cuda"), stream=stream)
+        G.set_theta(theta0)
+        pool = torch.empty((POOL_ROWS, P_FULL), device="cuda")
+        synth_gpu.grad_heavytail(seed, 0, pool, P_FULL, stream=stream)
+        stream.synchronize()
+
+        def batch(b):
+            ks = range(b * K_BATCH, (b + 1) * K_BATCH)
+            return [int(order[k]) for k in ks], [pool[k % POOL_ROWS] for k in ks]
+
+        for b in range(args.warmup):
+            G.commit_batch(*batch(b))
+        stream.synchronize()
+        barrier(pg)
+        starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+        ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+        launches0 = G.launches()
+        batches = [batch(args.warmup + i) for i in range(args.steps)]
+        with ClockSampler(local) as clocks:
+            torch.cuda.synchronize()
+            for i in range(args.steps):
+                starts[i].record(stream)
+                G.commit_batch(*batches[i])
+                ends[i].record(stream)
+            torch.cuda.synchronize()
+        launches = G.launches() - launches0
+        per_step_ms = [s.elapsed_time(e) for s, e in zip(starts, ends)]
+        total_ms = starts[0].elapsed_time(ends[-1])
+        total_ms = max_over_ranks(pg, total_ms)
+        barrier(pg)
+
+        # end to end through the public API: gradients in pinned host memory, copied in
+        # each step, and theta read back to the host after each step
+        e2e = None
+        if not args.no_e2e:
+            host_rows = 16
+            host_pool = [pool[r].cpu().pin_memory() for r in range(host_rows)]
+            theta_host = torch.empty(P_FULL, dtype=torch.float32).pin_memory()
+            e2e_steps = max(2, min(args.steps, 5))
+
+            def host_batch(b):
+                ks = range(b * K_BATCH, (b + 1) * K_BATCH)
+                return [int(order[k]) for k in ks], [host_pool[k % host_rows] for k in ks]
+
+            G.commit_batch_host(*host_batch(0))
+            gem.gem_read_theta(G.h, theta_host)
+            G.sync()
+            barrier(pg)
+            t0 = time.perf_counter()
+            for i in range(e2e_steps):
+                G.commit_batch_host(*host_batch(i))
+                gem.gem_read_theta(G.h, theta_host)
+                G.sync()
+            e2e_s = max_over_ranks(pg, time.perf_counter() - t0)
+            e2e = {"value": round(world * BYTES_PER_BATCH * e2e_steps / e2e_s / 1e9, 1), "unit": "GB/s",
+                   "h2d_bytes_per_step": K_BATCH * P_FULL * 4, "d2h_bytes_per_step": P_FULL * 4,
+                   "steps": e2e_steps, "commits_per_s": round(world * K_BATCH * e2e_steps / e2e_s, 1),
+                   "host_gradients": f"{host_rows} distinct pinned host buffers reused cyclically"}
+        G.close()
+
+    if rank != 0:
+        return
+    peak, peak_src = measured_peaks()
+    avg_launch_ms = sum(per_step_ms) / len(per_step_ms)
+    achieved = BYTES_PER_BATCH / (avg_launch_ms * 1e-3) / 1e9
+    value = world * BYTES_PER_BATCH * args.steps / (total_ms * 1e-3) / 1e9
+    traffic = NCU_TRAFFIC_BYTES_PER_LAUNCH if NCU_TRAFFIC_SOURCE_SHA == kernel_source_sha() else None
+    line = {
+        "metric": METRIC, "value": round(value, 1), "unit": "GB/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(total_ms / args.steps, 4),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+        "data": "synthetic",
+        "config": {"workload": "gem_commit_batch P=25M n=100, batches of 100 commits, heavy-tailed gradient pool",
+                   "P": P_FULL, "n": N_WORKERS, "commits_per_step": K_BATCH, "pool_gradients": POOL_ROWS,
+                   "eta": ETA, "mu": MU, "eps": EPS, "schedule": "uniform tick, seed 5 + rank",
+                   "l2": "inputs larger than L2 (about 30 GB working set), no flush",
+                   "parallelism": f"{world} independent replica(s)"},
+        "commits_per_s": round(world * K_BATCH * args.steps / (total_ms * 1e-3), 1),
+        "frac_of_hbm_peak": round(value / world / peak, 4),
+        "frac_of_8tbs_nominal": round(value / world / 8000.0, 4),
+        "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
+                     "frac": round(achieved / peak, 4), "traffic": traffic,
+                     "peak_source": f"{peak_src} copy bandwidth (burst)",
+                     "kernel": "commit_batch_kernel", "algorithmic_bytes_per_launch": BYTES_PER_BATCH,
+                     "launch_ms_min": round(min(per_step_ms), 4), "launch_ms_max": round(max(per_step_ms), 4)},
+        "gpu_launches": int(launches),
+        "clocks": clocks.summary(),
+        "e2e": e2e,
+    }
+    if not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline()
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["gem", "reference"], default="gem")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    # smaller cases for profiling; the defaults are the benchmark workload
+    ap.add_argument("--P", type=int, default=P_FULL)
+    ap.add_argument("--workers", type=int, default=N_WORKERS)
+    ap.add_argument("--batch", type=int, default=K_BATCH)
+    ap.add_argument("--pool", type=int, default=POOL_ROWS)
+    args = ap.parse_args()
+    if args.warmup < 3 and args.impl == "gem":
+        print("note: fewer than 3 warm-up steps", file=sys.stderr)
+    world, rank, local, pg = dist_setup()
+    if args.impl == "reference":
+        run_reference(args, world, rank, pg)
+    else:
+        from paper_1805_08469_gb300._build import build_library
+        build_library()
+        run_gem(args, world, rank, local, pg)
+    if pg is not None:
+        pg.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,131 @@
+/* gem.h -- C ABI of the Gradient Energy Matching commit path for GB300 (sm_103a).
+ *
+ * Gradient Energy Matching (GEM; Hermans & Louppe, "Gradient Energy Matching for
+ * Distributed Asynchronous Gradient Descent", arXiv 1805.08469) lets n asynchronous
+ * workers update a central variable theta.  Each commit is rescaled elementwise so the
+ * kinetic energy the workers put into theta together stays at or below the energy of
+ * momentum SGD.  This library keeps theta, every worker's first moment m_w and its
+ * snapshot s_w in the memory of one GPU.  A commit by worker w with gradient g
+ * (computed by the caller at s_w) does, for every coordinate j:
+ *
+ *   dtheta = -(eta * g)                    worker update (notation table; Algorithm 1, Worker)
+ *   m_w    = mu * m_w + dtheta             Psi_GEM, first step (Eq. moment_estimate)
+ *   pi     = (|m_w| - |theta - s_w|) / (|dtheta| + eps),  clamped to pi >= 0
+ *                                          Psi_GEM, second step (Eq. new_pi; |m_w| is
+ *                                          sqrt(2) sqrt(E_k) by Eq. proxy_estimate)
+ *   theta  = theta + pi * dtheta           Commit (Eqs. traditional_async_update, update_psi)
+ *   s_w    = theta                         the worker's pull for its next gradient
+ *
+ * Every step is one IEEE-754 fp32 operation rounded to nearest: no fused multiply-add
+ * and an IEEE division.  This order is part of the contract; it makes each commit
+ * reproducible bit for bit.
+ *
+ * Conventions shared by every call:
+ *   - Return value: GEM_OK (0) or a negative gem_status.  Arguments are checked on the
+ *     host; a call that fails a check changes nothing and launches nothing.
+ *   - Device work is asynchronous and ordered on the handle's stream (gem_set_stream;
+ *     the legacy default stream until set).  A CUDA error raised by device work is
+ *     reported by a later call, at the latest by gem_sync, as GEM_ECUDA.
+ *   - Caller buffers are fp32, 16-byte aligned, and must stay valid and unmodified until
+ *     the work that reads them has completed on the stream.  The library never keeps a
+ *     caller pointer beyond that work.
+ *   - State is library-owned device memory: theta [P] and m, s [n][stride] fp32, row w of
+ *     m and s belonging to worker w.  stride is P rounded up to a multiple of 32 floats
+ *     (128 bytes).  Elements past P hold 0 and stay 0.
+ *   - A handle is not thread-safe; separate handles are independent.
+ */
+#ifndef GEM_H
+#define GEM_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct gem_ctx gem_t;
+
+enum gem_status {
+  GEM_OK = 0,
+  GEM_EINVAL = -1, /* an argument failed a host-side check */
+  GEM_ENOMEM = -2, /* device or pinned-host allocation failed */
+  GEM_ECUDA = -3,  /* a CUDA call failed, or device work raised an error */
+  GEM_ESTATE = -4  /* the handle is unusable after an earlier CUDA error */
+};
+
+/* Create a handle for P parameters and n workers on the current CUDA device.
+ * Hyper-parameters follow Algorithm 1: learning rate eta > 0, momentum 0 <= mu < 1,
+ * eps > 0 (the term that keeps pi finite when dtheta = 0; the paper's default is 1e-16).
+ * Allocates theta [P] and m, s [n][stride] on the device; theta = 0, m = 0, s = 0.
+ * Requires P >= 1 and n >= 1.  On success *out receives the handle. */
+int gem_create(size_t P, int n, float eta, float mu, float eps, gem_t** out);
+
+/* Free every resource of the handle after finishing its pending work.  NULL is a no-op. */
+void gem_destroy(gem_t* h);
+
+/* Order all later device work of the handle on `stream` (a cudaStream_t of the handle's
+ * device; NULL selects the legacy default stream).  Work already issued is not moved. */
+int gem_set_stream(gem_t* h, void* stream);
+
+/* Initial pull (Algorithm 1, Worker: m <- 0, s <- Pull()): theta = theta0, s_w = theta0
+ * and m_w = 0 for every worker.  theta0 holds P fp32 values in device memory or in host
+ * memory (any pointer the CUDA runtime can copy from). */
+int gem_set_theta(gem_t* h, const float* theta0);
+
+/* Pull (Algorithm 1, Worker): *snapshot receives the device address of s_w, the central
+ * variable as it was right after worker w's last commit (theta0 before its first).  The
+ * memory is borrowed: read-only for the caller, and valid, with that content, until the
+ * next commit of worker w is issued.  Requires 0 <= worker < n. */
+int gem_pull(gem_t* h, int worker, const float** snapshot);
+
+/* One commit by worker w (Algorithm 1, Psi_GEM then Commit, then s <- theta): the five
+ * steps listed at the top of this file, over all P coordinates, in one kernel that
+ * reads grad, m_w, s_w, theta and writes m_w, s_w, theta once each.  grad is P fp32
+ * values in device memory (the gradient of the loss at s_w; the call forms
+ * dtheta = -eta grad itself).  Requires 0 <= worker < n and grad 16-byte aligned. */
+int gem_commit(gem_t* h, int worker, const float* grad);
+
+/* K commits in order: commit k is made by worker order[k] with gradient grads[k].  The
+ * result equals K calls of gem_commit in that order, bit for bit, including repeated
+ * workers.  order and grads are host arrays of length K, read before the call returns;
+ * each grads[k] is P fp32 values in device memory, 16-byte aligned.  theta is read and
+ * written once per batch instead of once per commit.  Requires K >= 0 (K = 0 is a
+ * no-op) and 0 <= order[k] < n. */
+int gem_commit_batch(gem_t* h, const int* order, const float* const* grads, int K);
+
+/* As gem_commit_batch, with each grads[k] in host memory instead (page-locked memory
+ * gives full copy bandwidth).  The gradients are copied to library-owned device staging
+ * buffers on a second stream, in chunks that overlap with the commits of earlier chunks.
+ * The host buffers must stay valid and unmodified until the handle's stream has
+ * finished the batch.  The staging buffers are allocated by the first call (at most 16
+ * gradients of `stride` floats). */
+int gem_commit_batch_host(gem_t* h, const int* order, const float* const* grads, int K);
+
+/* *theta receives the device address of theta [P] (borrowed, read-only, valid until
+ * gem_destroy; its content changes with every commit). */
+int gem_theta(gem_t* h, const float** theta);
+
+/* *moment receives the device address of m_w [P] (borrowed, read-only). */
+int gem_moment(gem_t* h, int worker, const float** moment);
+
+/* Stream-ordered copy of theta [P] into `out` (host or device memory). */
+int gem_read_theta(gem_t* h, float* out);
+
+/* Block until the handle's stream has finished; GEM_ECUDA if device work failed. */
+int gem_sync(gem_t* h);
+
+/* Layout query: P, n and the row stride (in floats) of m and s.  Any output may be NULL. */
+int gem_shape(const gem_t* h, size_t* P, int* n, size_t* stride);
+
+/* Number of kernels this handle has launched since it was created. */
+uint64_t gem_launch_count(const gem_t* h);
+
+/* Human-readable name of a gem_status value (static storage). */
+const char* gem_status_string(int status);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* GEM_H */

@@ -1,0 +1,317 @@
+// Host side of the GEM commit ABI (include/gem.h): handle life cycle, argument checks,
+// stream plumbing and the staging of host-resident gradients.
+#include <cstdint>
+#include <cstdlib>
+#include <new>
+
+#include "gem_internal.h"
+
+namespace {
+
+// Makes the handle's device current for the duration of a call, then restores the
+// caller's device.
+class DeviceScope {
+ public:
+  explicit DeviceScope(int device) {
+    if (cudaGetDevice(&prev_) != cudaSuccess) prev_ = -1;
+    if (prev_ != device) ok_ = cudaSetDevice(device) == cudaSuccess;
+    target_ = device;
+  }
+  ~DeviceScope() {
+    if (prev_ >= 0 && prev_ != target_) cudaSetDevice(prev_);
+  }
+  bool ok() const { return ok_; }
+
+ private:
+  int prev_ = -1;
+  int target_ = 0;
+  bool ok_ = true;
+};
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+int cuda_status(gem_t* h, cudaError_t e) {
+  if (e == cudaSuccess) return GEM_OK;
+  if (h) h->broken = true;
+  return GEM_ECUDA;
+}
+
+int check_handle(const gem_t* h) {
+  if (!h) return GEM_EINVAL;
+  if (h->broken) return GEM_ESTATE;
+  return GEM_OK;
+}
+
+gem::BatchArgs base_args(const gem_t* h) {
+  gem::BatchArgs a;
+  a.theta = h->theta;
+  a.m = h->m;
+  a.s = h->s;
+  a.P = h->P;
+  a.stride = h->stride;
+  a.eta = h->eta;
+  a.mu = h->mu;
+  a.eps = h->eps;
+  a.K = 0;
+  return a;
+}
+
+// Launch the commits [0, K) in chunks of at most kMaxBatchPerLaunch, in order.
+int launch_commits(gem_t* h, const int* order, const float* const* grads, int K) {
+  gem::BatchArgs a = base_args(h);
+  for (int k0 = 0; k0 < K; k0 += gem::kMaxBatchPerLaunch) {
+    const int kc = (K - k0) < gem::kMaxBatchPerLaunch ? (K - k0) : gem::kMaxBatchPerLaunch;
+    a.K = kc;
+    for (int k = 0; k < kc; ++k) {
+      a.worker[k] = order[k0 + k];
+      a.grad[k] = grads[k0 + k];
+    }
+    const int rc = cuda_status(h, gem::launch_commit_batch(a, h->sm_count, h->stream));
+    if (rc) return rc;
+    h->launches += 1;
+  }
+  return GEM_OK;
+}
+
+int check_batch(const gem_t* h, const int* order, const float* const* grads, int K) {
+  if (K < 0) return GEM_EINVAL;
+  if (K > 0 && (!order || !grads)) return GEM_EINVAL;
+  for (int k = 0; k < K; ++k) {
+    if (order[k] < 0 || order[k] >= h->n) return GEM_EINVAL;
+    if (!grads[k] || !aligned16(grads[k])) return GEM_EINVAL;
+  }
+  return GEM_OK;
+}
+
+int ensure_staging(gem_t* h) {
+  if (h->stage) return GEM_OK;
+  const size_t bytes = size_t(2 * gem::kStageChunk) * h->stride * sizeof(float);
+  if (cudaMalloc(&h->stage, bytes) != cudaSuccess) {
+    cudaGetLastError();
+    h->stage = nullptr;
+    return GEM_ENOMEM;
+  }
+  cudaError_t e = cudaStreamCreateWithFlags(&h->copy_stream, cudaStreamNonBlocking);
+  for (int i = 0; i < 2 && e == cudaSuccess; ++i) {
+    e = cudaEventCreateWithFlags(&h->stage_filled[i], cudaEventDisableTiming);
+    if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->stage_free[i], cudaEventDisableTiming);
+  }
+  return cuda_status(h, e);
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* gem_status_string(int status) {
+  switch (status) {
+    case GEM_OK: return "GEM_OK";
+    case GEM_EINVAL: return "GEM_EINVAL: invalid argument";
+    case GEM_ENOMEM: return "GEM_ENOMEM: allocation failed";
+    case GEM_ECUDA: return "GEM_ECUDA: CUDA error";
+    case GEM_ESTATE: return "GEM_ESTATE: handle unusable after an earlier CUDA error";
+    default: return "unknown gem_status";
+  }
+}
+
+int gem_create(size_t P, int n, float eta, float mu, float eps, gem_t** out) {
+  if (!out) return GEM_EINVAL;
+  *out = nullptr;
+  if (P == 0 || n < 1) return GEM_EINVAL;
+  if (!(eta > 0.0f) || !(mu >= 0.0f) || !(mu < 1.0f) || !(eps > 0.0f)) return GEM_EINVAL;
+  const size_t stride = (P + gem::kStrideAlign - 1) / gem::kStrideAlign * gem::kStrideAlign;
+  if (stride > (SIZE_MAX / sizeof(float)) / (size_t(n) + 1)) return GEM_EINVAL;
+  gem_t* h = new (std::nothrow) gem_t();
+  if (!h) return GEM_ENOMEM;
+  h->P = P;
+  h->stride = stride;
+  h->n = n;
+  h->eta = eta;
+  h->mu = mu;
+  h->eps = eps;
+  if (cudaGetDevice(&h->device) != cudaSuccess ||
+      cudaDeviceGetAttribute(&h->sm_count, cudaDevAttrMultiProcessorCount, h->device) !=
+          cudaSuccess) {
+    cudaGetLastError();
+    delete h;
+    return GEM_ECUDA;
+  }
+  const size_t row = stride * sizeof(float);
+  const size_t rows = size_t(n) * row;
+  if (cudaMalloc(&h->theta, row) != cudaSuccess || cudaMalloc(&h->m, rows) != cudaSuccess ||
+      cudaMalloc(&h->s, rows) != cudaSuccess) {
+    cudaGetLastError();
+    cudaFree(h->theta);
+    cudaFree(h->m);
+    cudaFree(h->s);
+    delete h;
+    return GEM_ENOMEM;
+  }
+  cudaError_t e = cudaMemset(h->theta, 0, row);
+  if (e == cudaSuccess) e = cudaMemset(h->m, 0, rows);
+  if (e == cudaSuccess) e = cudaMemset(h->s, 0, rows);
+  if (e == cudaSuccess) e = cudaDeviceSynchronize();
+  if (e != cudaSuccess) {
+    cudaFree(h->theta);
+    cudaFree(h->m);
+    cudaFree(h->s);
+    delete h;
+    return GEM_ECUDA;
+  }
+  *out = h;
+  return GEM_OK;
+}
+
+void gem_destroy(gem_t* h) {
+  if (!h) return;
+  DeviceScope scope(h->device);
+  cudaStreamSynchronize(h->stream);
+  if (h->copy_stream) cudaStreamSynchronize(h->copy_stream);
+  for (int i = 0; i < 2; ++i) {
+    if (h->stage_filled[i]) cudaEventDestroy(h->stage_filled[i]);
+    if (h->stage_free[i]) cudaEventDestroy(h->stage_free[i]);
+  }
+  if (h->copy_stream) cudaStreamDestroy(h->copy_stream);
+  cudaFree(h->stage);
+  cudaFree(h->theta);
+  cudaFree(h->m);
+  cudaFree(h->s);
+  cudaGetLastError();
+  delete h;
+}
+
+int gem_set_stream(gem_t* h, void* stream) {
+  if (!h) return GEM_EINVAL;
+  h->stream = static_cast<cudaStream_t>(stream);
+  return GEM_OK;
+}
+
+int gem_set_theta(gem_t* h, const float* theta0) {
+  int rc = check_handle(h);
+  if (rc) return rc;
+  if (!theta0) return GEM_EINVAL;
+  DeviceScope scope(h->device);
+  if (!scope.ok()) return GEM_ECUDA;
+  const size_t row = h->stride * sizeof(float);
+  cudaError_t e = cudaMemcpyAsync(h->theta, theta0, h->P * sizeof(float), cudaMemcpyDefault,
+                                  h->stream);
+  for (int w = 0; w < h->n && e == cudaSuccess; ++w)
+    e = cudaMemcpyAsync(h->s + size_t(w) * h->stride, h->theta, row, cudaMemcpyDeviceToDevice,
+                        h->stream);
+  if (e == cudaSuccess) e = cudaMemsetAsync(h->m, 0, size_t(h->n) * row, h->stream);
+  return cuda_status(h, e);
+}
+
+int gem_pull(gem_t* h, int worker, const float** snapshot) {
+  int rc = check_handle(h);
+  if (rc) return rc;
+  if (!snapshot || worker < 0 || worker >= h->n) return GEM_EINVAL;
+  *snapshot = h->s + size_t(worker) * h->stride;
+  return GEM_OK;
+}
+
+int gem_moment(gem_t* h, int worker, const float** moment) {
+  int rc = check_handle(h);
+  if (rc) return rc;
+  if (!moment || worker < 0 || worker >= h->n) return GEM_EINVAL;
+  *moment = h->m + size_t(worker) * h->stride;
+  return GEM_OK;
+}
+
+int gem_theta(gem_t* h, const float** theta) {
+  int rc = check_handle(h);
+  if (rc) return rc;
+  if (!theta) return GEM_EINVAL;
+  *theta = h->theta;
+  return GEM_OK;
+}
+
+int gem_shape(const gem_t* h, size_t* P, int* n, size_t* stride) {
+  if (!h) return GEM_EINVAL;
+  if (P) *P = h->P;
+  if (n) *n = h->n;
+  if (stride) *stride = h->stride;
+  return GEM_OK;
+}
+
+uint64_t gem_launch_count(const gem_t* h) { return h ? h->launches : 0; }
+
+int gem_commit(gem_t* h, int worker, const float* grad) {
+  int rc = check_handle(h);
+  if (rc) return rc;
+  rc = check_batch(h, &worker, &grad, 1);
+  if (rc) return rc;
+  DeviceScope scope(h->device);
+  if (!scope.ok()) return GEM_ECUDA;
+  return launch_commits(h, &worker, &grad, 1);
+}
+
+int gem_commit_batch(gem_t* h, const int* order, const float* const* grads, int K) {
+  int rc = check_handle(h);
+  if (rc) return rc;
+  rc = check_batch(h, order, grads, K);
+  if (rc || K == 0) return rc;
+  DeviceScope scope(h->device);
+  if (!scope.ok()) return GEM_ECUDA;
+  return launch_commits(h, order, grads, K);
+}
+
+int gem_commit_batch_host(gem_t* h, const int* order, const float* const* grads, int K) {
+  int rc = check_handle(h);
+  if (rc) return rc;
+  if (K < 0 || (K > 0 && (!order || !grads))) return GEM_EINVAL;
+  for (int k = 0; k < K; ++k)
+    if (order[k] < 0 || order[k] >= h->n || !grads[k]) return GEM_EINVAL;
+  if (K == 0) return GEM_OK;
+  DeviceScope scope(h->device);
+  if (!scope.ok()) return GEM_ECUDA;
+  rc = ensure_staging(h);
+  if (rc) return rc;
+  // Chunk j uses staging half j % 2: the copy stream fills it once the commits that last
+  // read it have finished, and the commit stream starts on it once it is filled, so the
+  // copy of chunk j + 1 overlaps the commits of chunk j.
+  const float* slot[gem::kStageChunk];
+  for (int k0 = 0, j = 0; k0 < K; k0 += gem::kStageChunk, ++j) {
+    const int half = j & 1;
+    const int kc = (K - k0) < gem::kStageChunk ? (K - k0) : gem::kStageChunk;
+    cudaError_t e = cudaStreamWaitEvent(h->copy_stream, h->stage_free[half], 0);
+    for (int i = 0; i < kc && e == cudaSuccess; ++i) {
+      float* dst = h->stage + size_t(half * gem::kStageChunk + i) * h->stride;
+      e = cudaMemcpyAsync(dst, grads[k0 + i], h->P * sizeof(float), cudaMemcpyDefault,
+                          h->copy_stream);
+      slot[i] = dst;
+    }
+    if (e == cudaSuccess) e = cudaEventRecord(h->stage_filled[half], h->copy_stream);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(h->stream, h->stage_filled[half], 0);
+    rc = cuda_status(h, e);
+    if (rc) return rc;
+    rc = launch_commits(h, order + k0, slot, kc);
+    if (rc) return rc;
+    rc = cuda_status(h, cudaEventRecord(h->stage_free[half], h->stream));
+    if (rc) return rc;
+  }
+  return GEM_OK;
+}
+
+int gem_read_theta(gem_t* h, float* out) {
+  int rc = check_handle(h);
+  if (rc) return rc;
+  if (!out) return GEM_EINVAL;
+  DeviceScope scope(h->device);
+  if (!scope.ok()) return GEM_ECUDA;
+  return cuda_status(h, cudaMemcpyAsync(out, h->theta, h->P * sizeof(float), cudaMemcpyDefault,
+                                        h->stream));
+}
+
+int gem_sync(gem_t* h) {
+  if (!h) return GEM_EINVAL;
+  if (h->broken) return GEM_ESTATE;
+  DeviceScope scope(h->device);
+  if (!scope.ok()) return GEM_ECUDA;
+  cudaError_t e = cudaStreamSynchronize(h->stream);
+  if (e == cudaSuccess && h->copy_stream) e = cudaStreamSynchronize(h->copy_stream);
+  if (e == cudaSuccess) e = cudaGetLastError();
+  return cuda_status(h, e);
+}
+
+}  // extern "C"

@@ -1,0 +1,140 @@
+// Fused GEM commit kernel (Algorithm 1: Psi_GEM, Commit, and the worker's next pull).
+//
+// Every step of a commit is elementwise over the P coordinates (the scaling factor pi is
+// a per-parameter vector, applied with a Hadamard product), so coordinate j of theta,
+// m_w and s_w depends only on coordinate j of the gradients.  The kernel therefore
+// gives each thread a few 16-byte lanes of coordinates and walks *all* commits of the
+// launch, in order, on those lanes: commit order is preserved without any lock or
+// inter-block communication, repeated workers inside a batch see their own earlier
+// results by program order, and theta stays in registers across the batch (read and
+// written once per launch instead of once per commit).
+//
+// Per coordinate and commit the kernel streams 12 bytes in (g, m_w, s_w) and 8 bytes
+// out (m_w, s_w); theta adds 8 bytes per launch.  The path is HBM-bound (about 0.5 flop
+// per byte), so the design goals are coalesced 128-bit accesses, enough independent
+// loads in flight per SM, and evict-first cache hints on the streamed vectors so that
+// theta and the next batch's lines are not pushed out of L2.
+#include "gem_internal.h"
+
+namespace gem {
+namespace {
+
+constexpr int kThreads = 256;
+
+// One coordinate of one commit.  One IEEE fp32 operation per step, rounded to nearest,
+// no contraction into FMA (the __f*_rn intrinsics are never fused), IEEE division.
+__device__ __forceinline__ void commit_coord(float& theta, float& m, float& s, float g,
+                                             float eta, float mu, float eps) {
+  const float dtheta = -__fmul_rn(eta, g);                       // -eta grad L(s)
+  const float m_new = __fadd_rn(__fmul_rn(mu, m), dtheta);       // m <- mu m + dtheta
+  const float drift = fabsf(__fsub_rn(theta, s));                // |theta - s|
+  float pi = __fdiv_rn(__fsub_rn(fabsf(m_new), drift),           // (|m| - |theta - s|)
+                       __fadd_rn(fabsf(dtheta), eps));           //   / (|dtheta| + eps)
+  pi = pi > 0.0f ? pi : 0.0f;                                    // pi >= 0
+  theta = __fadd_rn(theta, __fmul_rn(pi, dtheta));               // theta + pi dtheta
+  m = m_new;
+  s = theta;                                                     // s <- theta
+}
+
+__device__ __forceinline__ void commit_vec(float4& th, float4& m, float4& s, const float4 g,
+                                           float eta, float mu, float eps) {
+  commit_coord(th.x, m.x, s.x, g.x, eta, mu, eps);
+  commit_coord(th.y, m.y, s.y, g.y, eta, mu, eps);
+  commit_coord(th.z, m.z, s.z, g.z, eta, mu, eps);
+  commit_coord(th.w, m.w, s.w, g.w, eta, mu, eps);
+}
+
+// L independent 16-byte lanes per thread, strided by the grid so that each warp
+// touches 512 contiguous bytes per lane and array.
+template <int L>
+__global__ void __launch_bounds__(kThreads)
+commit_batch_kernel(const __grid_constant__ BatchArgs a) {
+  const size_t nvec = a.P >> 2;
+  const size_t nthreads = size_t(gridDim.x) * kThreads;
+  const size_t tid = size_t(blockIdx.x) * kThreads + threadIdx.x;
+  float4* theta4 = reinterpret_cast<float4*>(a.theta);
+
+  for (size_t base = tid; base < nvec; base += nthreads * L) {
+    float4 th[L];
+#pragma unroll
+    for (int l = 0; l < L; ++l) {
+      const size_t i = base + size_t(l) * nthreads;
+      if (i < nvec) th[l] = theta4[i];
+    }
+    for (int k = 0; k < a.K; ++k) {
+      const float4* g4 = reinterpret_cast<const float4*>(a.grad[k]);
+      const size_t row = size_t(a.worker[k]) * a.stride;
+      float4* m4 = reinterpret_cast<float4*>(a.m + row);
+      float4* s4 = reinterpret_cast<float4*>(a.s + row);
+      float4 g[L], m[L], s[L];
+#pragma unroll
+      for (int l = 0; l < L; ++l) {
+        const size_t i = base + size_t(l) * nthreads;
+        if (i < nvec) {
+          g[l] = __ldcs(g4 + i);
+          m[l] = __ldcs(m4 + i);
+          s[l] = __ldcs(s4 + i);
+        }
+      }
+#pragma unroll
+      for (int l = 0; l < L; ++l) {
+        const size_t i = base + size_t(l) * nthreads;
+        if (i < nvec) {
+          commit_vec(th[l], m[l], s[l], g[l], a.eta, a.mu, a.eps);
+          __stcs(m4 + i, m[l]);
+          __stcs(s4 + i, s[l]);
+        }
+      }
+    }
+#pragma unroll
+    for (int l = 0; l < L; ++l) {
+      const size_t i = base + size_t(l) * nthreads;
+      if (i < nvec) theta4[i] = th[l];
+    }
+  }
+
+  // Ragged tail: the last P mod 4 coordinates, one thread each, scalar accesses (the
+  // caller's gradient holds exactly P floats).
+  const size_t tail0 = nvec << 2;
+  if (tid < a.P - tail0) {
+    const size_t j = tail0 + tid;
+    float th = a.theta[j];
+    for (int k = 0; k < a.K; ++k) {
+      const size_t row = size_t(a.worker[k]) * a.stride;
+      float m = a.m[row + j], s = a.s[row + j];
+      commit_coord(th, m, s, a.grad[k][j], a.eta, a.mu, a.eps);
+      a.m[row + j] = m;
+      a.s[row + j] = s;
+    }
+    a.theta[j] = th;
+  }
+}
+
+constexpr int kLanes = 2;
+
+}  // namespace
+
+cudaError_t launch_commit_batch(const BatchArgs& a, int sm_count, cudaStream_t stream) {
+  static int blocks_per_sm = 0;
+  if (blocks_per_sm == 0) {
+    cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(
+        &blocks_per_sm, commit_batch_kernel<kLanes>, kThreads, 0);
+    if (e != cudaSuccess) return e;
+    if (blocks_per_sm < 1) blocks_per_sm = 1;
+  }
+  const size_t nvec = a.P >> 2;
+  const size_t per_block = size_t(kThreads) * kLanes;
+  const size_t max_grid = size_t(sm_count) * size_t(blocks_per_sm);
+  size_t grid = (nvec + per_block - 1) / per_block;
+  if (grid > max_grid) {
+    // Same number of rounds per thread as the full resident grid, with the grid trimmed
+    // so that the last round is as full as possible.
+    const size_t rounds = (nvec + max_grid * per_block - 1) / (max_grid * per_block);
+    grid = (nvec + rounds * per_block - 1) / (rounds * per_block);
+  }
+  if (grid < 1) grid = 1;
+  commit_batch_kernel<kLanes><<<unsigned(grid), kThreads, 0, stream>>>(a);
+  return cudaGetLastError();
+}
+
+}  // namespace gem

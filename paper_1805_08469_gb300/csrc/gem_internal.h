@@ -1,0 +1,59 @@
+// Internal declarations of the GEM commit library (not installed, not part of the ABI).
+#pragma once
+
+#include <cuda_runtime.h>
+
+#include <cstddef>
+#include <cstdint>
+
+#include "../../include/gem.h"
+
+namespace gem {
+
+// Commits carried by one launch of the batched commit kernel.  They travel in the
+// kernel's parameter block (2.4 KB + header), so a launch needs no device-side
+// descriptor; longer batches are split into several launches, in order.
+constexpr int kMaxBatchPerLaunch = 200;
+
+// Row stride of m and s (and length of theta): P rounded up to 32 floats = 128 bytes.
+constexpr size_t kStrideAlign = 32;
+
+// Host-gradient staging for gem_commit_batch_host: two halves of kStageChunk slots.
+constexpr int kStageChunk = 8;
+
+struct BatchArgs {
+  float* theta;                            // [stride]
+  float* m;                                // [n][stride]
+  float* s;                                // [n][stride]
+  size_t P;
+  size_t stride;
+  float eta, mu, eps;
+  int K;                                   // commits in this launch, 1..kMaxBatchPerLaunch
+  const float* grad[kMaxBatchPerLaunch];   // gradient of commit k, P floats
+  int worker[kMaxBatchPerLaunch];          // worker of commit k
+};
+
+// Launch the fused commit kernel for a.K commits on `stream`.
+cudaError_t launch_commit_batch(const BatchArgs& a, int sm_count, cudaStream_t stream);
+
+}  // namespace gem
+
+struct gem_ctx {
+  int device = 0;
+  int sm_count = 0;
+  size_t P = 0;
+  size_t stride = 0;
+  int n = 0;
+  float eta = 0.f, mu = 0.f, eps = 0.f;
+  float* theta = nullptr;
+  float* m = nullptr;
+  float* s = nullptr;
+  cudaStream_t stream = nullptr;
+  uint64_t launches = 0;
+  bool broken = false;
+  // staging of host gradients (gem_commit_batch_host), allocated on first use
+  float* stage = nullptr;
+  cudaStream_t copy_stream = nullptr;
+  cudaEvent_t stage_filled[2] = {nullptr, nullptr};
+  cudaEvent_t stage_free[2] = {nullptr, nullptr};
+};

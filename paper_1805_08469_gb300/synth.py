@@ -161,9 +161,10 @@ def grad_heavytail(seed: int, i: int, j) -> np.ndarray:
     """Pool gradient i at coordinates j: 0.01 * (normal, or Student-t(3) on the mask)."""
     j = _cols(j)
     c = (_U64(i) << _U64(32)) | j
-    z = normal(key(seed, STREAM_GRAD_Z), c)
-    t = student_t3(key(seed, STREAM_GRAD_T), c)
-    v = np.where(heavy_mask(seed, j), t, z)
+    mask = heavy_mask(seed, j)
+    v = np.empty(j.shape, dtype=np.float32)
+    v[~mask] = normal(key(seed, STREAM_GRAD_Z), c[~mask])
+    v[mask] = student_t3(key(seed, STREAM_GRAD_T), c[mask])
     return (FLAT_GRAD_SCALE * v).astype(np.float32)
 
 
