@@ -63,63 +63,104 @@ def measured_peaks() -> tuple[float, str]:
 
 
 class ClockSampler:
-    """nvidia-smi clock and throttle-reason samples taken during the timed region."""
+    """SM clock and throttle reasons sampled every 10 ms during the timed region.
 
-    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
-              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
-              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+    Reads NVML through ctypes (libnvidia-ml); nvidia-smi at 100 ms is the fallback.
+    Only reads: no clock, power or mode setting is touched.
+    """
 
-    def __init__(self, device_index: int):
-        self.dev = device_index
-        self.proc = None
-        self.lines: list[str] = []
-        self.thread = None
+    REASONS = {0x4: "sw_power_cap", 0x8: "hw_slowdown", 0x20: "sw_thermal_slowdown",
+               0x40: "hw_thermal_slowdown", 0x80: "hw_power_brake_slowdown"}
+
+    def __init__(self, cuda_index: int, period_s: float = 0.01):
+        self.cuda_index = cuda_index
+        self.period = period_s
+        self.samples: list[tuple[float, float, int]] = []
+        self._stop = threading.Event()
+        self._thread = None
+        self._proc = None
+        self.source = None
+
+    def _nvml_handle(self):
+        import ctypes
+        nv = ctypes.CDLL("libnvidia-ml.so.1")
+        if nv.nvmlInit_v2() != 0:
+            raise RuntimeError("nvmlInit failed")
+        h = ctypes.c_void_p()
+        bus = None
+        try:
+            import torch
+            pr = torch.cuda.get_device_properties(self.cuda_index)
+            bus = f"{pr.pci_domain_id:08x}:{pr.pci_bus_id:02x}:{pr.pci_device_id:02x}.0"
+        except Exception:
+            bus = None
+        if bus is None or nv.nvmlDeviceGetHandleByPciBusId_v2(bus.encode(), ctypes.byref(h)) != 0:
+            if nv.nvmlDeviceGetHandleByIndex_v2(self.cuda_index, ctypes.byref(h)) != 0:
+                raise RuntimeError("no NVML handle")
+        return nv, h
+
+    def _run_nvml(self, nv, h):
+        import ctypes
+        clk = ctypes.c_uint()
+        mx = ctypes.c_uint()
+        rs = ctypes.c_ulonglong()
+        get_reasons = getattr(nv, "nvmlDeviceGetCurrentClocksEventReasons", None) or \
+            nv.nvmlDeviceGetCurrentClocksThrottleReasons
+        while not self._stop.is_set():
+            ok = nv.nvmlDeviceGetClockInfo(h, 1, ctypes.byref(clk)) == 0
+            ok = ok and nv.nvmlDeviceGetMaxClockInfo(h, 1, ctypes.byref(mx)) == 0
+            ok = ok and get_reasons(h, ctypes.byref(rs)) == 0
+            if ok:
+                self.samples.append((float(clk.value), float(mx.value), int(rs.value)))
+            time.sleep(self.period)
+
+    def _run_smi(self):
+        fields = ("clocks.sm,clocks.max.sm,clocks_event_reasons.hw_slowdown,"
+                  "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+                  "clocks_event_reasons.sw_power_cap")
+        self._proc = subprocess.Popen(["nvidia-smi", "-i", str(self.cuda_index), f"--query-gpu={fields}",
+                                       "--format=csv,noheader,nounits", "-lms", "100"],
+                                      stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        bits = [0x8, 0x40, 0x20, 0x4]
+        for line in self._proc.stdout:
+            parts = [p.strip() for p in line.split(",")]
+            try:
+                r = sum(b for b, v in zip(bits, parts[2:6]) if v.lower() == "active")
+                self.samples.append((float(parts[0]), float(parts[1]), r))
+            except (ValueError, IndexError):
+                continue
 
     def __enter__(self):
         try:
-            self.proc = subprocess.Popen(
-                ["nvidia-smi", "-i", str(self.dev), f"--query-gpu={self.FIELDS}",
-                 "--format=csv,noheader,nounits", "-lms", "200"],
-                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
-            self.thread = threading.Thread(target=self._read, daemon=True)
-            self.thread.start()
+            nv, h = self._nvml_handle()
+            self.source = "nvml"
+            self._thread = threading.Thread(target=self._run_nvml, args=(nv, h), daemon=True)
         except Exception:
-            self.proc = None
+            self.source = "nvidia-smi"
+            self._thread = threading.Thread(target=self._run_smi, daemon=True)
+        self._thread.start()
         return self
 
-    def _read(self):
-        for line in self.proc.stdout:
-            self.lines.append(line.strip())
-
     def __exit__(self, *exc):
-        if self.proc is not None:
-            self.proc.terminate()
+        self._stop.set()
+        if self._proc is not None:
+            self._proc.terminate()
             try:
-                self.proc.wait(timeout=5)
+                self._proc.wait(timeout=5)
             except Exception:
-                self.proc.kill()
-            if self.thread:
-                self.thread.join(timeout=2)
+                self._proc.kill()
+        if self._thread is not None:
+            self._thread.join(timeout=5)
 
     def summary(self) -> dict:
-        sm, mx, reasons = [], [], set()
-        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        for line in self.lines:
-            parts = [p.strip() for p in line.split(",")]
-            if len(parts) < 9:
-                continue
-            try:
-                sm.append(float(parts[1]))
-                mx.append(float(parts[2]))
-            except ValueError:
-                continue
-            for name, val in zip(names, parts[5:9]):
-                if val.lower() == "active":
-                    reasons.add(name)
-        if not sm:
-            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
-        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
-                "samples": len(sm)}
+        if not self.samples:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0, "source": self.source}
+        reasons = set()
+        for _, _, r in self.samples:
+            reasons.update(name for bit, name in self.REASONS.items() if r & bit)
+        return {"sm_mhz": statistics.median(s[0] for s in self.samples),
+                "sm_max_mhz": max(s[1] for s in self.samples), "reasons": sorted(reasons),
+                "samples": len(self.samples), "source": self.source}
 
 
 def dist_setup():
@@ -322,7 +363,8 @@ def run_gem(args, world, rank, local, pg):
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(total_ms / args.steps, 4),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
         "data": "synthetic",
-        "config": {"workload": "gem_commit_batch P=25M n=100, batches of 100 commits, heavy-tailed gradient pool",
+        "config": {"workload": f"gem_commit_batch P={P_FULL} n={N_WORKERS}, batches of {K_BATCH} commits, "
+                               f"heavy-tailed gradient pool of {POOL_ROWS}",
                    "P": P_FULL, "n": N_WORKERS, "commits_per_step": K_BATCH, "pool_gradients": POOL_ROWS,
                    "eta": ETA, "mu": MU, "eps": EPS, "schedule": "uniform tick, seed 5 + rank",
                    "l2": "inputs larger than L2 (about 30 GB working set), no flush",
@@ -347,7 +389,7 @@ def run_gem(args, world, rank, local, pg):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--steps", type=int, default=30)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["gem", "reference"], default="gem")
     ap.add_argument("--no-cpu-baseline", action="store_true")

@@ -10,14 +10,16 @@
  *
  * Random numbers: SplitMix64 (Steele, Lea & Flood, OOPSLA 2014).  The stream for
  * (seed, id) starts at mix64(seed * 0x9E3779B97F4A7C15 + id) and its c-th output is
- * mix64(start + 0x9E3779B97F4A7C15 (c + 1)).  Host-only functions; they return 0, or -1
- * on an invalid argument.
+ * mix64(start + 0x9E3779B97F4A7C15 (c + 1)).  The schedule functions are host-only and
+ * return 0, or -1 on an invalid argument; the MLP calls return a gem_status.
  */
 #ifndef GEM_SIM_H
 #define GEM_SIM_H
 
 #include <stddef.h>
 #include <stdint.h>
+
+#include "gem.h"
 
 #ifdef __cplusplus
 extern "C" {
@@ -40,6 +42,54 @@ int gem_schedule_queue(uint64_t seed, int n, int T, double rate, int32_t* order,
  * workers.  seg_start [T + 1] receives the first commit of each segment followed by T;
  * returns the number of segments S (seg_start[0..S]), or -1 on an invalid argument. */
 int gem_plan_segments(const int32_t* order, int T, int n, int32_t* seg_start);
+
+/* ---------------------------------------------------------------------------------
+ * Worker gradients of a fully connected ReLU network, batched over stale snapshots.
+ *
+ * A worker computes dtheta = -eta grad L(s) at its snapshot s (notation table; Algorithm 1,
+ * Worker).  The model here is an MLP dims[0] -> dims[1] -> ... -> dims[L] with ReLU on the
+ * hidden layers and the mean softmax cross-entropy over the worker's minibatch as L.  Its
+ * parameters are GEM's flat vector [W_1, b_1, W_2, b_2, ...], W_l stored dims[l] x
+ * dims[l-1] row-major (out x in).  The gradients of a segment's workers (distinct workers,
+ * so every snapshot is fixed for the whole segment) are computed together: each GEMM of
+ * the forward and backward pass is one grouped launch over the segment.
+ */
+typedef struct gem_mlp gem_mlp_t;
+
+enum gem_mlp_precision {
+  GEM_MLP_FP32 = 0, /* fp32 products and sums (CUDA cores) */
+  GEM_MLP_TF32 = 1  /* operands rounded to TF32 (nearest, ties away), fp32 accumulation,
+                       tensor cores (tcgen05) for the large products */
+};
+
+/* Bind an MLP to a GEM handle (its P must equal the MLP's parameter count).  batch is the
+ * per-worker minibatch b (1..1024); dims[L] <= 32 classes.  Allocates per-worker scratch
+ * (activations and deltas) and one gradient buffer per worker on the handle's device. */
+int gem_mlp_create(gem_t* gem, int n_layers, const int32_t* dims, int batch, int precision,
+                   gem_mlp_t** out);
+
+/* Training set: X [rows][dims[0]] fp32 and labels [rows] int32 in device memory, borrowed
+ * (they must stay valid while the MLP is used). */
+int gem_mlp_set_data(gem_mlp_t* mlp, const float* X, const int32_t* labels, int64_t rows);
+
+/* Gradients of the mean loss at the snapshots of workers[0..L) (any workers, repeats
+ * allowed) on minibatches batch_rows [L][batch] (device, row indices into X), written to
+ * grads[i] (device, P floats, 16-byte aligned, caller-owned).  losses (device [L], may be
+ * NULL) receives each minibatch's mean loss.  Asynchronous on the GEM handle's stream. */
+int gem_mlp_grad(gem_mlp_t* mlp, const int32_t* workers, int L, const int32_t* batch_rows,
+                 float* const* grads, float* losses);
+
+/* End-to-end asynchronous GEM: commits t = 0..T-1 by workers order[t] (host array), commit
+ * t using the minibatch batch_rows[t][0..batch) (device).  The schedule is cut into
+ * segments of distinct workers (gem_plan_segments); per segment the workers' gradients
+ * are computed at their snapshots in one batched forward/backward, then committed in
+ * order with the fused commit kernel (so each snapshot is refreshed to the post-commit
+ * theta).  losses (device [T], may be NULL) receives each commit's minibatch loss. */
+int gem_mlp_run(gem_mlp_t* mlp, const int32_t* order, int T, const int32_t* batch_rows,
+                float* losses);
+
+/* Free the MLP's scratch (after its pending work).  NULL is a no-op. */
+void gem_mlp_destroy(gem_mlp_t* mlp);
 
 #ifdef __cplusplus
 }
