@@ -73,14 +73,17 @@ int gem_mlp_create(gem_t* gem, int n_layers, const int32_t* dims, int batch, int
 int gem_mlp_set_data(gem_mlp_t* mlp, const float* X, const int32_t* labels, int64_t rows);
 
 /* Gradients of the mean loss at the snapshots of workers[0..L) (any workers, repeats
- * allowed) on minibatches batch_rows [L][batch] (device, row indices into X), written to
+ * allowed) on minibatches batch_rows [L][batch] (host array of row indices into X, checked
+ * against the data set and copied to the device before the call returns), written to
  * grads[i] (device, P floats, 16-byte aligned, caller-owned).  losses (device [L], may be
  * NULL) receives each minibatch's mean loss.  Asynchronous on the GEM handle's stream. */
 int gem_mlp_grad(gem_mlp_t* mlp, const int32_t* workers, int L, const int32_t* batch_rows,
                  float* const* grads, float* losses);
 
 /* End-to-end asynchronous GEM: commits t = 0..T-1 by workers order[t] (host array), commit
- * t using the minibatch batch_rows[t][0..batch) (device).  The schedule is cut into
+ * t using the minibatch batch_rows[t][0..batch) (host array, checked and copied to the
+ * device before the call returns; an index outside the data set is GEM_EINVAL).  A label
+ * outside [0, dims[L]) yields a NaN loss and gradient.  The schedule is cut into
  * segments of distinct workers (gem_plan_segments); per segment the workers' gradients
  * are computed at their snapshots in one batched forward/backward, then committed in
  * order with the fused commit kernel (so each snapshot is refreshed to the post-commit

@@ -39,6 +39,11 @@ def _declare(L):
         "gem_schedule_uniform": ([C.c_uint64, i, i, p, p], i),
         "gem_schedule_queue": ([C.c_uint64, i, i, C.c_double, p, p], i),
         "gem_plan_segments": ([p, i, i, p], i),
+        "gem_mlp_create": ([p, i, p, i, i, p], i),
+        "gem_mlp_set_data": ([p, p, p, C.c_int64], i),
+        "gem_mlp_grad": ([p, p, i, p, p, p], i),
+        "gem_mlp_run": ([p, p, i, p, p], i),
+        "gem_mlp_destroy": ([p], None),
         "gem_synth_theta0": ([C.c_uint64, sz, p, p], i),
         "gem_synth_grad_heavytail": ([C.c_uint64, C.c_uint64, i, sz, sz, p, p], i),
         "gem_synth_grad_loguniform": ([C.c_uint64, C.c_uint64, sz, p, p, p], i),

@@ -1,0 +1,547 @@
+// Batched worker gradients of a ReLU MLP over stale snapshots, and the end-to-end
+// asynchronous GEM loop built on them (include/gem_sim.h).
+//
+// A worker computes dtheta = -eta grad L(s) at its snapshot s (notation table; Algorithm
+// 1, Worker).  Workers of one segment (distinct workers, see gem_plan_segments) have
+// fixed snapshots, so each product of their forward and backward passes is one grouped
+// launch over the segment: group g works on worker order[a + g]'s snapshot (weights read
+// straight from s_w inside GEM's state) and on slot g of the scratch (activations,
+// deltas, gradient).  The gradients are then committed in schedule order by the fused
+// commit kernel.
+//
+// Products per layer l (dims d_l -> d_{l+1}, batch b), all written for row-major storage:
+//   forward   Z_l  = A_l W_l^T + b_l     A_l [b x d_l],   W_l [d_{l+1} x d_l]
+//   weights   dW_l = D_{l+1}^T A_l       D_{l+1} [b x d_{l+1}]
+//   inputs    D_l  = (D_{l+1} W_l) * [A_l > 0]
+//   biases    db_l = column sums of D_{l+1} (fixed order, no atomics)
+// Every sum runs in a fixed order, so the gradients are deterministic.
+#include <cstdint>
+#include <cstring>
+#include <new>
+#include <vector>
+
+#include "../../include/gem_sim.h"
+#include "gem_internal.h"
+
+namespace gem {
+namespace mlp {
+
+constexpr int kMaxLayers = 8;
+constexpr int kMaxGroups = 128;
+constexpr int kMaxClasses = 32;
+constexpr int kMaxBatch = 1024;
+
+// SIMT tile: 128 x 64 outputs per block of 256 threads, 8 x 4 per thread, k-steps of 16.
+constexpr int BM = 128, BN = 64, BK = 16, kThreads = 256;
+
+enum Epilogue : int { kStore = 0, kBias = 1, kBiasRelu = 2, kMask = 3 };
+
+struct Operand {
+  const float* base;
+  long long group_stride;  // elements between the operands of consecutive groups
+  long long ld;            // leading dimension of its row-major storage
+  int by_worker;           // group g uses index workers[g] (GEM state) instead of g (scratch)
+};
+
+struct GemmArgs {
+  int M, N, K;
+  Operand A;  // element (m, k)
+  Operand B;  // element (k, n)
+  float* C;
+  long long c_group_stride, ldc;
+  const float* bias;  // by worker, bias[n]
+  long long bias_group_stride;
+  const float* mask;  // by group, keep C(m, n) where mask(m, n) > 0
+  long long mask_group_stride, ldmask;
+  int workers[kMaxGroups];
+};
+
+__device__ __forceinline__ float to_tf32(float x) {
+  uint32_t r;
+  asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(r) : "f"(x));
+  return __uint_as_float(r);
+}
+
+// C[g] (M x N) = epilogue( op(A[g]) op(B[g]) ).  A_KMAJOR: A(m, k) at A[m*lda + k], else at
+// A[k*lda + m].  B_KMAJOR: B(k, n) at B[n*ldb + k], else at B[k*ldb + n].
+template <bool A_KMAJOR, bool B_KMAJOR, int EPI, bool TF32>
+__global__ void __launch_bounds__(kThreads)
+gemm_grouped_kernel(const __grid_constant__ GemmArgs p) {
+  __shared__ float As[BM][BK + 1];
+  __shared__ float Bs[BN][BK + 1];
+  const int g = blockIdx.z;
+  const int m0 = blockIdx.y * BM, n0 = blockIdx.x * BN;
+  const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
+  const float* A = p.A.base + (p.A.by_worker ? (long long)p.workers[g] : (long long)g) * p.A.group_stride;
+  const float* B = p.B.base + (p.B.by_worker ? (long long)p.workers[g] : (long long)g) * p.B.group_stride;
+  const long long lda = p.A.ld, ldb = p.B.ld;
+  const int M = p.M, N = p.N, K = p.K;
+
+  float ra[8], rb[4];
+  auto load = [&](int k0) {
+#pragma unroll
+    for (int it = 0; it < 8; ++it) {
+      int m, k;
+      if (A_KMAJOR) { m = (tid >> 4) + 16 * it; k = tid & 15; }
+      else          { m = tid & 127;            k = (tid >> 7) + 2 * it; }
+      const int gm = m0 + m, gk = k0 + k;
+      float v = 0.f;
+      if (gm < M && gk < K) v = A_KMAJOR ? A[gm * lda + gk] : A[gk * lda + gm];
+      ra[it] = TF32 ? to_tf32(v) : v;
+    }
+#pragma unroll
+    for (int it = 0; it < 4; ++it) {
+      int n, k;
+      if (B_KMAJOR) { n = (tid >> 4) + 16 * it; k = tid & 15; }
+      else          { n = tid & 63;             k = (tid >> 6) + 4 * it; }
+      const int gn = n0 + n, gk = k0 + k;
+      float v = 0.f;
+      if (gn < N && gk < K) v = B_KMAJOR ? B[gn * ldb + gk] : B[gk * ldb + gn];
+      rb[it] = TF32 ? to_tf32(v) : v;
+    }
+  };
+  auto store = [&]() {
+#pragma unroll
+    for (int it = 0; it < 8; ++it) {
+      if (A_KMAJOR) As[(tid >> 4) + 16 * it][tid & 15] = ra[it];
+      else          As[tid & 127][(tid >> 7) + 2 * it] = ra[it];
+    }
+#pragma unroll
+    for (int it = 0; it < 4; ++it) {
+      if (B_KMAJOR) Bs[(tid >> 4) + 16 * it][tid & 15] = rb[it];
+      else          Bs[tid & 63][(tid >> 6) + 4 * it] = rb[it];
+    }
+  };
+
+  float acc[8][4];
+#pragma unroll
+  for (int i = 0; i < 8; ++i)
+#pragma unroll
+    for (int j = 0; j < 4; ++j) acc[i][j] = 0.f;
+
+  load(0);
+  store();
+  __syncthreads();
+  for (int k0 = 0; k0 < K; k0 += BK) {
+    const bool more = k0 + BK < K;
+    if (more) load(k0 + BK);
+#pragma unroll
+    for (int k = 0; k < BK; ++k) {
+      float a[8], b[4];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) a[i] = As[ty + 16 * i][k];
+#pragma unroll
+      for (int j = 0; j < 4; ++j) b[j] = Bs[tx + 16 * j][k];
+#pragma unroll
+      for (int i = 0; i < 8; ++i)
+#pragma unroll
+        for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(a[i], b[j], acc[i][j]);
+    }
+    __syncthreads();
+    if (more) {
+      store();
+      __syncthreads();
+    }
+  }
+
+  float* C = p.C + (long long)g * p.c_group_stride;
+  const float* bias = (EPI == kBias || EPI == kBiasRelu)
+                          ? p.bias + (long long)p.workers[g] * p.bias_group_stride : nullptr;
+  const float* mask = EPI == kMask ? p.mask + (long long)g * p.mask_group_stride : nullptr;
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    const int m = m0 + ty + 16 * i;
+    if (m >= M) continue;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const int n = n0 + tx + 16 * j;
+      if (n >= N) continue;
+      float v = acc[i][j];
+      if (EPI == kBias) v = v + bias[n];
+      if (EPI == kBiasRelu) v = fmaxf(v + bias[n], 0.f);
+      if (EPI == kMask) v = mask[m * p.ldmask + n] > 0.f ? v : 0.f;
+      C[m * p.ldc + n] = v;
+    }
+  }
+}
+
+// Minibatch gather: slot g's rows X[batch_rows[g][r]] -> Xs[g][r][:].
+__global__ void gather_rows_kernel(const float* X, int d0, const int32_t* batch_rows, int b,
+                                   float* Xs, long long slot_stride) {
+  const int g = blockIdx.y, r = blockIdx.x;
+  const long long row = batch_rows[(long long)g * b + r];
+  const float* src = X + row * d0;
+  float* dst = Xs + g * slot_stride + (long long)r * d0;
+  for (int k = threadIdx.x; k < d0; k += blockDim.x) dst[k] = src[k];
+}
+
+// Softmax cross-entropy over C classes for the b rows of each slot: the mean loss, and the
+// gradient of the mean with respect to the logits, (softmax - onehot) / b.
+__global__ void softmax_xent_kernel(const float* logits, float* delta, long long slot_stride,
+                                   int b, int C, const int32_t* labels,
+                                   const int32_t* batch_rows, float* losses) {
+  __shared__ float row_loss[kMaxBatch];
+  const int g = blockIdx.x;
+  const float* z = logits + g * slot_stride;
+  float* d = delta + g * slot_stride;
+  for (int r = threadIdx.x; r < b; r += blockDim.x) {
+    const float* zr = z + (long long)r * C;
+    int y = labels[batch_rows[(long long)g * b + r]];
+    const bool bad_label = y < 0 || y >= C;  // reported as a NaN loss and gradient
+    if (bad_label) y = 0;
+    float zmax = zr[0];
+    for (int c = 1; c < C; ++c) zmax = fmaxf(zmax, zr[c]);
+    float e[kMaxClasses];
+    float sum = 0.f;
+    for (int c = 0; c < C; ++c) {
+      e[c] = expf(zr[c] - zmax);
+      sum += e[c];
+    }
+    const float inv_b = 1.0f / float(b);
+    const float poison = bad_label ? __int_as_float(0x7fc00000) : 0.f;
+    for (int c = 0; c < C; ++c)
+      d[(long long)r * C + c] = (e[c] / sum - (c == y ? 1.f : 0.f)) * inv_b + poison;
+    row_loss[r] = (logf(sum) + zmax) - zr[y] + poison;
+  }
+  __syncthreads();
+  if (losses && threadIdx.x == 0) {
+    float s = 0.f;
+    for (int r = 0; r < b; ++r) s += row_loss[r];
+    losses[g] = s / float(b);
+  }
+}
+
+struct BiasGradArgs {
+  int n_layers, b;
+  long long grad_off[kMaxLayers];   // offset of db_l in the flat gradient
+  long long delta_off[kMaxLayers];  // offset of D_{l+1} in the slot scratch
+  int width[kMaxLayers];            // d_{l+1}
+  int first[kMaxLayers + 1];        // prefix sums of width
+};
+
+// db_l[o] = sum over the batch of D_{l+1}[r][o], every layer in one launch.
+__global__ void bias_grad_kernel(const __grid_constant__ BiasGradArgs a, const float* delta,
+                                 long long slot_stride, float* grad, long long grad_stride) {
+  const int g = blockIdx.y;
+  const int q = blockIdx.x * blockDim.x + threadIdx.x;
+  if (q >= a.first[a.n_layers]) return;
+  int l = 0;
+  while (q >= a.first[l + 1]) ++l;
+  const int o = q - a.first[l];
+  const float* D = delta + g * slot_stride + a.delta_off[l];
+  float s = 0.f;
+  for (int r = 0; r < a.b; ++r) s += D[(long long)r * a.width[l] + o];
+  grad[g * grad_stride + a.grad_off[l] + o] = s;
+}
+
+template <bool AK, bool BK_, int EPI>
+cudaError_t launch_gemm(const GemmArgs& a, int groups, bool tf32, cudaStream_t st) {
+  dim3 grid((a.N + BN - 1) / BN, (a.M + BM - 1) / BM, groups);
+  if (tf32)
+    gemm_grouped_kernel<AK, BK_, EPI, true><<<grid, kThreads, 0, st>>>(a);
+  else
+    gemm_grouped_kernel<AK, BK_, EPI, false><<<grid, kThreads, 0, st>>>(a);
+  return cudaGetLastError();
+}
+
+}  // namespace mlp
+}  // namespace gem
+
+using namespace gem::mlp;
+
+struct gem_mlp {
+  gem_t* gem = nullptr;
+  int L = 0;
+  int dims[kMaxLayers + 1] = {};
+  long long w_off[kMaxLayers] = {}, b_off[kMaxLayers] = {};
+  int batch = 0;
+  int precision = 0;
+  const float* X = nullptr;
+  const int32_t* labels = nullptr;
+  int64_t rows = 0;
+  // per-slot scratch: X_s [b x d0], A_l [b x d_l] (l = 1..L-1), logits [b x C],
+  // D_l [b x d_l] (l = 1..L)
+  long long off_x = 0, off_act[kMaxLayers + 1] = {}, off_logits = 0, off_delta[kMaxLayers + 1] = {};
+  long long slot_stride = 0;
+  int slots = 0;
+  float* scratch = nullptr;
+  float* grads = nullptr;  // [n][gem stride]
+  int32_t* rows_dev = nullptr;  // minibatch rows uploaded from the host
+  size_t rows_cap = 0;
+  uint64_t launches = 0;
+};
+
+namespace {
+
+long long round32(long long x) { return (x + 31) / 32 * 32; }
+
+int cuda_rc(cudaError_t e) { return e == cudaSuccess ? GEM_OK : GEM_ECUDA; }
+
+// Forward and backward for groups [0, G) of one chunk: workers[g], minibatch rows
+// batch_rows[g][0..b), gradient of group g written at grads + g * grad_stride.
+int mlp_chunk(gem_mlp* M, const int32_t* workers, int G, const int32_t* batch_rows,
+              float* grads, long long grad_stride, float* losses) {
+  gem_t* h = M->gem;
+  cudaStream_t st = h->stream;
+  const bool tf32 = M->precision == GEM_MLP_TF32;
+  const int L = M->L, b = M->batch;
+  const long long S = M->slot_stride;
+  float* scr = M->scratch;
+  auto act = [&](int l) -> float* { return l == 0 ? scr + M->off_x : scr + M->off_act[l]; };
+
+  gather_rows_kernel<<<dim3(b, G), 256, 0, st>>>(M->X, M->dims[0], batch_rows, b,
+                                                 scr + M->off_x, S);
+  int rc = cuda_rc(cudaGetLastError());
+  if (rc) return rc;
+  M->launches++;
+
+  GemmArgs a;
+  std::memset(&a, 0, sizeof(a));
+  for (int g = 0; g < G; ++g) a.workers[g] = workers[g];
+  const long long wstride = (long long)h->stride;
+
+  // forward
+  for (int l = 0; l < L; ++l) {
+    const int din = M->dims[l], dout = M->dims[l + 1];
+    a.M = b; a.N = dout; a.K = din;
+    a.A = Operand{act(l), S, din, 0};
+    a.B = Operand{h->s + M->w_off[l], wstride, din, 1};
+    a.bias = h->s + M->b_off[l];
+    a.bias_group_stride = wstride;
+    const bool last = l == L - 1;
+    a.C = last ? scr + M->off_logits : act(l + 1);
+    a.c_group_stride = S;
+    a.ldc = dout;
+    cudaError_t e = last ? launch_gemm<true, true, kBias>(a, G, tf32, st)
+                         : launch_gemm<true, true, kBiasRelu>(a, G, tf32, st);
+    if ((rc = cuda_rc(e))) return rc;
+    M->launches++;
+  }
+  softmax_xent_kernel<<<G, 128, 0, st>>>(scr + M->off_logits, scr + M->off_delta[L], S, b,
+                                         M->dims[L], M->labels, batch_rows, losses);
+  if ((rc = cuda_rc(cudaGetLastError()))) return rc;
+  M->launches++;
+
+  // backward
+  for (int l = L - 1; l >= 0; --l) {
+    const int din = M->dims[l], dout = M->dims[l + 1];
+    // dW_l = D_{l+1}^T A_l: (m = o, k = r) from D [b x dout], (k = r, n = j) from A [b x din]
+    a.M = dout; a.N = din; a.K = b;
+    a.A = Operand{scr + M->off_delta[l + 1], S, dout, 0};
+    a.B = Operand{act(l), S, din, 0};
+    a.C = grads + M->w_off[l];
+    a.c_group_stride = grad_stride;
+    a.ldc = din;
+    if ((rc = cuda_rc(launch_gemm<false, false, kStore>(a, G, tf32, st)))) return rc;
+    M->launches++;
+    if (l == 0) break;
+    // D_l = (D_{l+1} W_l) * [A_l > 0]: (m = r, k = o) from D, (k = o, n = j) from W_l [dout x din]
+    a.M = b; a.N = din; a.K = dout;
+    a.A = Operand{scr + M->off_delta[l + 1], S, dout, 0};
+    a.B = Operand{h->s + M->w_off[l], wstride, din, 1};
+    a.C = scr + M->off_delta[l];
+    a.c_group_stride = S;
+    a.ldc = din;
+    a.mask = act(l);
+    a.mask_group_stride = S;
+    a.ldmask = din;
+    if ((rc = cuda_rc(launch_gemm<true, false, kMask>(a, G, tf32, st)))) return rc;
+    M->launches++;
+  }
+  BiasGradArgs ba;
+  std::memset(&ba, 0, sizeof(ba));
+  ba.n_layers = L;
+  ba.b = b;
+  ba.first[0] = 0;
+  for (int l = 0; l < L; ++l) {
+    ba.grad_off[l] = M->b_off[l];
+    ba.delta_off[l] = M->off_delta[l + 1];
+    ba.width[l] = M->dims[l + 1];
+    ba.first[l + 1] = ba.first[l] + M->dims[l + 1];
+  }
+  bias_grad_kernel<<<dim3((ba.first[L] + 255) / 256, G), 256, 0, st>>>(ba, scr, S, grads,
+                                                                        grad_stride);
+  if ((rc = cuda_rc(cudaGetLastError()))) return rc;
+  M->launches++;
+  return GEM_OK;
+}
+
+// Check minibatch rows on the host and copy them to the device (stream-ordered).
+int upload_rows(gem_mlp* M, const int32_t* rows_host, long long count) {
+  for (long long i = 0; i < count; ++i)
+    if (rows_host[i] < 0 || rows_host[i] >= M->rows) return GEM_EINVAL;
+  if ((size_t)count > M->rows_cap) {
+    cudaFree(M->rows_dev);  // synchronises with work still reading the old buffer
+    M->rows_dev = nullptr;
+    M->rows_cap = 0;
+    if (cudaMalloc(&M->rows_dev, sizeof(int32_t) * size_t(count)) != cudaSuccess) {
+      cudaGetLastError();
+      return GEM_ENOMEM;
+    }
+    M->rows_cap = size_t(count);
+  }
+  return cuda_rc(cudaMemcpyAsync(M->rows_dev, rows_host, sizeof(int32_t) * size_t(count),
+                                 cudaMemcpyHostToDevice, M->gem->stream));
+}
+
+}  // namespace
+
+extern "C" {
+
+int gem_mlp_create(gem_t* g, int n_layers, const int32_t* dims, int batch, int precision,
+                   gem_mlp_t** out) {
+  if (!out) return GEM_EINVAL;
+  *out = nullptr;
+  if (!g || !dims || n_layers < 1 || n_layers > kMaxLayers || batch < 1 || batch > kMaxBatch)
+    return GEM_EINVAL;
+  if (precision != GEM_MLP_FP32 && precision != GEM_MLP_TF32) return GEM_EINVAL;
+  if (g->broken) return GEM_ESTATE;
+  long long P = 0;
+  for (int l = 0; l <= n_layers; ++l)
+    if (dims[l] < 1) return GEM_EINVAL;
+  if (dims[n_layers] > kMaxClasses) return GEM_EINVAL;
+  gem_mlp* M = new (std::nothrow) gem_mlp();
+  if (!M) return GEM_ENOMEM;
+  M->gem = g;
+  M->L = n_layers;
+  M->batch = batch;
+  M->precision = precision;
+  for (int l = 0; l <= n_layers; ++l) M->dims[l] = dims[l];
+  for (int l = 0; l < n_layers; ++l) {
+    M->w_off[l] = P;
+    M->b_off[l] = P + (long long)dims[l + 1] * dims[l];
+    P = M->b_off[l] + dims[l + 1];
+  }
+  if ((size_t)P != g->P) {
+    delete M;
+    return GEM_EINVAL;
+  }
+  long long off = 0;
+  M->off_x = off;
+  off += round32((long long)batch * dims[0]);
+  for (int l = 1; l < n_layers; ++l) {
+    M->off_act[l] = off;
+    off += round32((long long)batch * dims[l]);
+  }
+  M->off_logits = off;
+  off += round32((long long)batch * dims[n_layers]);
+  for (int l = 1; l <= n_layers; ++l) {
+    M->off_delta[l] = off;
+    off += round32((long long)batch * dims[l]);
+  }
+  M->slot_stride = off;
+  M->slots = g->n < kMaxGroups ? g->n : kMaxGroups;
+  int dev_prev = 0;
+  cudaGetDevice(&dev_prev);
+  cudaSetDevice(g->device);
+  cudaError_t e = cudaMalloc(&M->scratch, sizeof(float) * size_t(M->slot_stride) * M->slots);
+  if (e == cudaSuccess) e = cudaMalloc(&M->grads, sizeof(float) * g->stride * size_t(g->n));
+  cudaSetDevice(dev_prev);
+  if (e != cudaSuccess) {
+    cudaGetLastError();
+    cudaFree(M->scratch);
+    cudaFree(M->grads);
+    delete M;
+    return GEM_ENOMEM;
+  }
+  *out = M;
+  return GEM_OK;
+}
+
+void gem_mlp_destroy(gem_mlp_t* M) {
+  if (!M) return;
+  int dev_prev = 0;
+  cudaGetDevice(&dev_prev);
+  cudaSetDevice(M->gem->device);
+  cudaStreamSynchronize(M->gem->stream);
+  cudaFree(M->scratch);
+  cudaFree(M->grads);
+  cudaFree(M->rows_dev);
+  cudaGetLastError();
+  cudaSetDevice(dev_prev);
+  delete M;
+}
+
+int gem_mlp_set_data(gem_mlp_t* M, const float* X, const int32_t* labels, int64_t rows) {
+  if (!M || !X || !labels || rows < 1) return GEM_EINVAL;
+  M->X = X;
+  M->labels = labels;
+  M->rows = rows;
+  return GEM_OK;
+}
+
+int gem_mlp_grad(gem_mlp_t* M, const int32_t* workers, int L, const int32_t* batch_rows,
+                 float* const* grads, float* losses) {
+  if (!M || L < 0 || (L > 0 && (!workers || !batch_rows || !grads))) return GEM_EINVAL;
+  if (!M->X) return GEM_EINVAL;
+  gem_t* h = M->gem;
+  if (h->broken) return GEM_ESTATE;
+  for (int i = 0; i < L; ++i) {
+    if (workers[i] < 0 || workers[i] >= h->n || !grads[i]) return GEM_EINVAL;
+    if ((reinterpret_cast<uintptr_t>(grads[i]) & 15u) != 0) return GEM_EINVAL;
+  }
+  int dev_prev = 0;
+  cudaGetDevice(&dev_prev);
+  cudaSetDevice(h->device);
+  int rc = upload_rows(M, batch_rows, (long long)L * M->batch);
+  for (int c0 = 0; c0 < L && rc == GEM_OK; c0 += M->slots) {
+    const int G = (L - c0) < M->slots ? (L - c0) : M->slots;
+    rc = mlp_chunk(M, workers + c0, G, M->rows_dev + (long long)c0 * M->batch, M->grads,
+                   (long long)h->stride, losses ? losses + c0 : nullptr);
+    for (int g = 0; g < G && rc == GEM_OK; ++g)
+      rc = cuda_rc(cudaMemcpyAsync(grads[c0 + g], M->grads + (long long)g * h->stride,
+                                   h->P * sizeof(float), cudaMemcpyDeviceToDevice, h->stream));
+  }
+  if (rc == GEM_ECUDA) h->broken = true;
+  cudaSetDevice(dev_prev);
+  return rc;
+}
+
+int gem_mlp_run(gem_mlp_t* M, const int32_t* order, int T, const int32_t* batch_rows,
+                float* losses) {
+  if (!M || T < 0 || (T > 0 && (!order || !batch_rows))) return GEM_EINVAL;
+  if (!M->X) return GEM_EINVAL;
+  gem_t* h = M->gem;
+  if (h->broken) return GEM_ESTATE;
+  if (T == 0) return GEM_OK;
+  std::vector<int32_t> seg(size_t(T) + 1);
+  const int S = gem_plan_segments(order, T, h->n, seg.data());
+  if (S < 0) return GEM_EINVAL;
+  int dev_prev = 0;
+  cudaGetDevice(&dev_prev);
+  cudaSetDevice(h->device);
+  int rc = upload_rows(M, batch_rows, (long long)T * M->batch);
+  gem::BatchArgs ca;
+  ca.theta = h->theta;
+  ca.m = h->m;
+  ca.s = h->s;
+  ca.P = h->P;
+  ca.stride = h->stride;
+  ca.eta = h->eta;
+  ca.mu = h->mu;
+  ca.eps = h->eps;
+  for (int i = 0; i < S && rc == GEM_OK; ++i) {
+    const int a = seg[i], e = seg[i + 1];
+    for (int c0 = a; c0 < e && rc == GEM_OK; c0 += M->slots) {
+      const int G = (e - c0) < M->slots ? (e - c0) : M->slots;
+      rc = mlp_chunk(M, order + c0, G, M->rows_dev + (long long)c0 * M->batch,
+                     M->grads + (long long)(c0 - a) * h->stride, (long long)h->stride,
+                     losses ? losses + c0 : nullptr);
+    }
+    for (int k0 = a; k0 < e && rc == GEM_OK; k0 += gem::kMaxBatchPerLaunch) {
+      const int kc = (e - k0) < gem::kMaxBatchPerLaunch ? (e - k0) : gem::kMaxBatchPerLaunch;
+      ca.K = kc;
+      for (int k = 0; k < kc; ++k) {
+        ca.worker[k] = order[k0 + k];
+        ca.grad[k] = M->grads + (long long)(k0 + k - a) * h->stride;
+      }
+      rc = cuda_rc(gem::launch_commit_batch(ca, h->sm_count, h->stream));
+      h->launches++;
+    }
+  }
+  if (rc == GEM_ECUDA) h->broken = true;
+  cudaSetDevice(dev_prev);
+  return rc;
+}
+
+}  // extern "C"

@@ -37,3 +37,50 @@ def gem_plan_segments(order, n: int) -> np.ndarray:
     if S < 0:
         raise ValueError("gem_plan_segments: invalid argument")
     return seg[:S + 1].copy()
+
+
+GEM_MLP_FP32 = 0
+GEM_MLP_TF32 = 1
+
+
+def gem_mlp_create(gem_handle: int, dims, batch: int, precision: int = GEM_MLP_FP32) -> int:
+    from ._lib import check
+    d = (C.c_int32 * len(dims))(*[int(x) for x in dims])
+    h = C.c_void_p()
+    check(lib().gem_mlp_create(C.c_void_p(gem_handle), len(dims) - 1, d, batch, precision,
+                               C.byref(h)), "gem_mlp_create")
+    return int(h.value)
+
+
+def gem_mlp_destroy(h: int) -> None:
+    lib().gem_mlp_destroy(C.c_void_p(h))
+
+
+def gem_mlp_set_data(h: int, X, labels) -> None:
+    """X: float32 CUDA tensor [rows, d0]; labels: int32 CUDA tensor [rows] (borrowed)."""
+    from ._lib import check
+    check(lib().gem_mlp_set_data(C.c_void_p(h), C.c_void_p(X.data_ptr()),
+                                 C.c_void_p(labels.data_ptr()), X.shape[0]), "gem_mlp_set_data")
+
+
+def _opt_ptr(t):
+    return C.c_void_p(0 if t is None else t.data_ptr())
+
+
+def gem_mlp_grad(h: int, workers, batch_rows, grads, losses=None) -> None:
+    """workers [L] ints; batch_rows host int array [L, b]; grads: L float32 CUDA tensors."""
+    from ._lib import check
+    w = np.ascontiguousarray(workers, dtype=np.int32)
+    r = np.ascontiguousarray(batch_rows, dtype=np.int32)
+    g = (C.c_void_p * len(grads))(*[x.data_ptr() for x in grads])
+    check(lib().gem_mlp_grad(C.c_void_p(h), _p(w), len(w), _p(r), g, _opt_ptr(losses)), "gem_mlp_grad")
+
+
+def gem_mlp_run(h: int, order, batch_rows, losses=None) -> None:
+    """order [T] ints; batch_rows host int array [T, b]; losses: float32 CUDA tensor [T] or None."""
+    from ._lib import check
+    o = np.ascontiguousarray(order, dtype=np.int32)
+    r = np.ascontiguousarray(batch_rows, dtype=np.int32)
+    if r.shape[0] != o.shape[0]:
+        raise ValueError("batch_rows must have one row per commit")
+    check(lib().gem_mlp_run(C.c_void_p(h), _p(o), len(o), _p(r), _opt_ptr(losses)), "gem_mlp_run")
