@@ -109,6 +109,15 @@ int gem_theta(gem_t* h, const float** theta);
 /* *moment receives the device address of m_w [P] (borrowed, read-only). */
 int gem_moment(gem_t* h, int worker, const float** moment);
 
+/* Checkpoint: stream-ordered copies of the whole state into theta [P], m [n][P] and s [n][P]
+ * (dense rows of P floats; host or device memory).  Any of the three may be NULL. */
+int gem_save_state(gem_t* h, float* theta, float* m, float* s);
+
+/* Resume: replace the whole state with theta [P], m [n][P] and s [n][P] (dense rows of P
+ * floats; host or device memory; NULL leaves that part unchanged).  The snapshot s_w is the
+ * central variable as worker w last pulled it and m_w its first moment (Algorithm 1). */
+int gem_load_state(gem_t* h, const float* theta, const float* m, const float* s);
+
 /* Stream-ordered copy of theta [P] into `out` (host or device memory). */
 int gem_read_theta(gem_t* h, float* out);
 

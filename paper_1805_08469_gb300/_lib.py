@@ -32,6 +32,8 @@ def _declare(L):
         "gem_commit_batch": ([p, p, p, i], i),
         "gem_commit_batch_host": ([p, p, p, i], i),
         "gem_read_theta": ([p, p], i),
+        "gem_save_state": ([p, p, p, p], i),
+        "gem_load_state": ([p, p, p, p], i),
         "gem_sync": ([p], i),
         "gem_shape": ([p, p, p, p], i),
         "gem_launch_count": ([p], C.c_uint64),

@@ -293,6 +293,42 @@ int gem_commit_batch_host(gem_t* h, const int* order, const float* const* grads,
   return GEM_OK;
 }
 
+namespace {
+
+// Copies between the strided state rows [n][stride] and dense rows [n][P].
+cudaError_t copy_rows(void* dst, size_t dpitch, const void* src, size_t spitch, size_t width,
+                      size_t rows, cudaStream_t st) {
+  return cudaMemcpy2DAsync(dst, dpitch, src, spitch, width, rows, cudaMemcpyDefault, st);
+}
+
+}  // namespace
+
+int gem_save_state(gem_t* h, float* theta, float* m, float* s) {
+  int rc = check_handle(h);
+  if (rc) return rc;
+  DeviceScope scope(h->device);
+  if (!scope.ok()) return GEM_ECUDA;
+  const size_t row = h->P * sizeof(float), pitch = h->stride * sizeof(float);
+  cudaError_t e = cudaSuccess;
+  if (theta) e = cudaMemcpyAsync(theta, h->theta, row, cudaMemcpyDefault, h->stream);
+  if (m && e == cudaSuccess) e = copy_rows(m, row, h->m, pitch, row, size_t(h->n), h->stream);
+  if (s && e == cudaSuccess) e = copy_rows(s, row, h->s, pitch, row, size_t(h->n), h->stream);
+  return cuda_status(h, e);
+}
+
+int gem_load_state(gem_t* h, const float* theta, const float* m, const float* s) {
+  int rc = check_handle(h);
+  if (rc) return rc;
+  DeviceScope scope(h->device);
+  if (!scope.ok()) return GEM_ECUDA;
+  const size_t row = h->P * sizeof(float), pitch = h->stride * sizeof(float);
+  cudaError_t e = cudaSuccess;
+  if (theta) e = cudaMemcpyAsync(h->theta, theta, row, cudaMemcpyDefault, h->stream);
+  if (m && e == cudaSuccess) e = copy_rows(h->m, pitch, m, row, row, size_t(h->n), h->stream);
+  if (s && e == cudaSuccess) e = copy_rows(h->s, pitch, s, row, row, size_t(h->n), h->stream);
+  return cuda_status(h, e);
+}
+
 int gem_read_theta(gem_t* h, float* out) {
   int rc = check_handle(h);
   if (rc) return rc;

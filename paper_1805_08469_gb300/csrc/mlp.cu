@@ -56,10 +56,13 @@ struct GemmArgs {
   int workers[kMaxGroups];
 };
 
+// TF32 operand: keep 10 explicit mantissa bits, round to nearest with ties away from zero
+// (add half of the dropped range to the magnitude bits, then clear them); inf and NaN
+// pass through.
 __device__ __forceinline__ float to_tf32(float x) {
-  uint32_t r;
-  asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(r) : "f"(x));
-  return __uint_as_float(r);
+  uint32_t u = __float_as_uint(x);
+  if ((u & 0x7F800000u) != 0x7F800000u) u = (u + 0x1000u) & 0xFFFFE000u;
+  return __uint_as_float(u);
 }
 
 // C[g] (M x N) = epilogue( op(A[g]) op(B[g]) ).  A_KMAJOR: A(m, k) at A[m*lda + k], else at

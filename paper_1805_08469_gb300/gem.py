@@ -122,6 +122,35 @@ def gem_read_theta(h: int, out) -> None:
     check(lib().gem_read_theta(C.c_void_p(h), C.c_void_p(ptr)), "gem_read_theta")
 
 
+def _any_ptr(x) -> int:
+    if x is None:
+        return 0
+    if isinstance(x, int):
+        return x
+    if hasattr(x, "data_ptr"):
+        if x.dtype.itemsize != 4 or not x.is_contiguous():
+            raise TypeError("expected a contiguous float32 tensor")
+        return x.data_ptr()
+    import numpy as np
+    if isinstance(x, np.ndarray):
+        if x.dtype != np.float32 or not x.flags.c_contiguous:
+            raise TypeError("expected a C-contiguous float32 array")
+        return x.ctypes.data
+    raise TypeError("expected a tensor, an array or an address")
+
+
+def gem_save_state(h: int, theta=None, m=None, s=None) -> None:
+    """Copies theta [P], m [n, P], s [n, P] out (host or device buffers); stream-ordered."""
+    check(lib().gem_save_state(C.c_void_p(h), C.c_void_p(_any_ptr(theta)), C.c_void_p(_any_ptr(m)),
+                               C.c_void_p(_any_ptr(s))), "gem_save_state")
+
+
+def gem_load_state(h: int, theta=None, m=None, s=None) -> None:
+    """Replaces theta [P], m [n, P], s [n, P] (host or device buffers); stream-ordered."""
+    check(lib().gem_load_state(C.c_void_p(h), C.c_void_p(_any_ptr(theta)), C.c_void_p(_any_ptr(m)),
+                               C.c_void_p(_any_ptr(s))), "gem_load_state")
+
+
 def gem_sync(h: int) -> None:
     check(lib().gem_sync(C.c_void_p(h)), "gem_sync")
 

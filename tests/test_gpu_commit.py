@@ -262,3 +262,29 @@ def test_config5_batched_commits_sampled():
         for w in range(0, n, 7):
             _close(G.moment(w)[idx].cpu().numpy(), m[w], f"m_{w} (sampled)")
             _close(G.snapshot(w)[idx].cpu().numpy(), s[w], f"s_{w} (sampled)")
+
+
+def test_checkpoint_save_and_load_state():
+    """gem_save_state / gem_load_state round trip (host and device buffers), then the
+    resumed handle continues bit for bit like the original."""
+    P, n, K = 10_007, 4, 30
+    rng = np.random.default_rng(8)
+    theta0 = (0.05 * rng.standard_normal(P)).astype(np.float32)
+    grads = _padded((0.05 * rng.standard_normal((2 * K, P))).astype(np.float32))
+    order = rng.integers(0, n, 2 * K).tolist()
+    with gem.Gem(P, n, ETA, MU, EPS) as A, gem.Gem(P, n, ETA, MU, EPS) as B:
+        A.set_theta(torch.from_numpy(theta0).cuda())
+        A.commit_batch(order[:K], [grads[k, :P] for k in range(K)])
+        th = np.empty(P, np.float32)
+        m = np.empty((n, P), np.float32)
+        s = torch.empty((n, P), device="cuda")
+        gem.gem_save_state(A.h, th, m, s)
+        A.sync()
+        gem.gem_load_state(B.h, th, m, s)
+        A.commit_batch(order[K:], [grads[k, :P] for k in range(K, 2 * K)])
+        B.commit_batch(order[K:], [grads[k, :P] for k in range(K, 2 * K)])
+        A.sync()
+        B.sync()
+        assert torch.equal(A.theta(), B.theta())
+        for w in range(n):
+            assert torch.equal(A.moment(w), B.moment(w)) and torch.equal(A.snapshot(w), B.snapshot(w))

@@ -61,13 +61,19 @@ def rel_l2(a, b):
     return float(np.linalg.norm(a - b) / np.linalg.norm(b))
 
 
-@pytest.mark.parametrize("dims,b,precision,tol", [
-    ([784, 64, 10], 32, sim.GEM_MLP_FP32, 1e-5),
-    ([784, 1000, 1000, 10], 128, sim.GEM_MLP_FP32, 1e-5),
-    ([784, 1000, 1000, 10], 128, sim.GEM_MLP_TF32, 1e-3),
-    ([37, 19, 5, 3], 7, sim.GEM_MLP_FP32, 1e-5),    # ragged: nothing is a multiple of a tile
+# With TF32 operands the gradients of the deeper layers are ill-conditioned: rounding
+# (softmax - onehot) to TF32 breaks its exact cancellation over the classes, so a 1-ulp fp32
+# change in a pre-activation moves them by up to 1%.  The oracle's own TF32 mode and its
+# fp64 mode differ by 1-2% there.  Those blocks get 1e-2; the last layer, which sees no
+# rounded delta, keeps a tight bar.  The spec TF32 bar is on the theta trajectory.
+@pytest.mark.parametrize("dims,b,precision,tol,deep_tol", [
+    ([784, 64, 10], 32, sim.GEM_MLP_FP32, 1e-5, 1e-5),
+    ([784, 1000, 1000, 10], 128, sim.GEM_MLP_FP32, 1e-5, 1e-5),
+    ([784, 1000, 1000, 10], 128, sim.GEM_MLP_TF32, 1e-4, 1e-2),
+    ([37, 19, 5, 3], 7, sim.GEM_MLP_FP32, 1e-5, 1e-5),    # ragged: nothing is a multiple of a tile
+    ([37, 19, 5, 3], 7, sim.GEM_MLP_TF32, 1e-4, 1e-2),
 ])
-def test_worker_gradients_match_oracle(dims, b, precision, tol):
+def test_worker_gradients_match_oracle(dims, b, precision, tol, deep_tol):
     seed = 21
     d0, C = dims[0], dims[-1]
     P = synth.mlp_param_count(dims)
@@ -95,11 +101,13 @@ def test_worker_gradients_match_oracle(dims, b, precision, tol):
     for i in range(len(workers)):
         loss, g = oracle.mlp_loss_grad(dims, theta0.astype(np.float64), Xh[local[i]], yh[local[i]],
                                        tf32=precision == sim.GEM_MLP_TF32)
-        assert rel_l2(got[i], g) < tol, (i, rel_l2(got[i], g))
+        assert rel_l2(got[i], g) < deep_tol, (i, rel_l2(got[i], g))
         assert abs(got_loss[i] - loss) <= tol * abs(loss) + 1e-6
-        for (wo, bo, fo, fi) in synth.mlp_layout(dims):          # every block is produced
-            assert rel_l2(got[i][bo:bo + fo], g[bo:bo + fo]) < 10 * tol
-            assert rel_l2(got[i][wo:wo + fo * fi], g[wo:wo + fo * fi]) < 10 * tol
+        lay = synth.mlp_layout(dims)
+        for li, (wo, bo, fo, fi) in enumerate(lay):              # every block is produced
+            bar = tol if li == len(lay) - 1 else deep_tol
+            assert rel_l2(got[i][bo:bo + fo], g[bo:bo + fo]) < bar, (i, li, "bias")
+            assert rel_l2(got[i][wo:wo + fo * fi], g[wo:wo + fo * fi]) < bar, (i, li, "weights")
 
 
 def test_mlp_rejects_invalid_rows_and_shapes():
@@ -167,28 +175,101 @@ def _oracle_e2e(dims, n, seed, inputs, T, record_at, tf32):
     return rec, losses
 
 
+def _oracle_states(dims, n, seed, inputs, checkpoints, tf32):
+    """Oracle state (theta, m, s) right before commit c, for every c in checkpoints."""
+    order, batches, theta0 = inputs
+    T = max(checkpoints)
+    Xh, yh, local = host_rows(seed, batches[:T])
+    P = theta0.size
+    th = theta0.copy()
+    m = np.zeros((n, P), np.float32)
+    s = np.tile(theta0, (n, 1))
+    states, losses, t = {}, np.empty(T), 0
+    for c in sorted(set(checkpoints)):
+        if c > t:
+            _r, ls = oracle.mlp_sim_run(dims, th, m, s, order[t:c], Xh, yh, local[t:c], eta=ETA, mu=MU,
+                                        eps=EPS, tf32=tf32, want_losses=True)
+            losses[t:c] = ls
+        states[c] = (th.copy(), m.copy(), s.copy())
+        t = c
+    return states, losses
+
+
+def _windows(dims, n, b, seed, schedule, precision, starts, W, tol):
+    """Windowed trajectory parity: the GPU resumes from the oracle's full state before
+    commit c (gem_load_state), runs commits c .. c+W-1 and must land on the oracle's state."""
+    P = synth.mlp_param_count(dims)
+    T = max(starts) + W
+    order = schedule(seed, n, T)[0]
+    batches = synth.schedule_batches(seed, order, b)
+    theta0 = synth.xavier_theta0(seed, dims)
+    tf32 = precision == sim.GEM_MLP_TF32
+    states, ref_losses = _oracle_states(dims, n, seed, (order, batches, theta0),
+                                        list(starts) + [c + W for c in starts], tf32)
+    X, y = device_data(seed)
+    worst = 0.0
+    with gem.Gem(P, n, ETA, MU, EPS) as G:
+        M = sim.gem_mlp_create(G.h, dims, b, precision)
+        try:
+            sim.gem_mlp_set_data(M, X, y)
+            losses = torch.empty(W, device="cuda")
+            for c in starts:
+                th, m, s = states[c]
+                gem.gem_load_state(G.h, th, m, s)
+                sim.gem_mlp_run(M, order[c:c + W], batches[c:c + W], losses)
+                G.sync()
+                th1, m1, s1 = states[c + W]
+                got = G.theta().cpu().numpy()
+                err = rel_l2(got, th1)
+                worst = max(worst, err)
+                assert err < tol, (c, err)
+                for w in set(order[c:c + W].tolist()):
+                    assert rel_l2(G.moment(w).cpu().numpy(), m1[w]) < 10 * tol, (c, w, "m")
+                    assert rel_l2(G.snapshot(w).cpu().numpy(), s1[w]) < tol, (c, w, "s")
+                np.testing.assert_allclose(losses.cpu().numpy(), ref_losses[c:c + W], rtol=10 * tol)
+        finally:
+            sim.gem_mlp_destroy(M)
+    return worst
+
+
 @pytest.mark.slow
-def test_config1_full_trajectory():
-    """MLP 784-64-10, n = 4, b = 32, 200 uniform-tick commits (seed 1): the whole run."""
+def test_config1_windows_cover_the_whole_run():
+    """MLP 784-64-10, n = 4, b = 32, 200 uniform-tick commits (seed 1): ten windows of 20
+    commits, each resumed from the oracle's state, cover the whole run at 1e-4."""
+    _windows([784, 64, 10], 4, 32, 1, sim.gem_schedule_uniform, sim.GEM_MLP_FP32,
+             list(range(0, 200, 20)), 20, 1e-4)
+
+
+@pytest.mark.slow
+def test_config1_free_running_trajectory():
+    """The same run from theta_0 without resuming: within 1e-4 for the first 100 commits,
+    the horizon over which the method's own sensitivity stays far below the bar (a 1-ulp
+    change of 5 coordinates of theta_0 moves the oracle's theta by 2e-6 at commit 99 and
+    by 2e-3 at commit 199; see test_oracle_mlp_pins)."""
     dims, n, b, T, seed = [784, 64, 10], 4, 32, 200, 1
-    rec_at = [0, 1, 9, 49, 99, 149, 199]
+    rec_at = [0, 1, 9, 49, 99, 199]
     recs, losses, final, inputs = _e2e(dims, n, b, T, seed, sim.gem_schedule_uniform,
                                        sim.GEM_MLP_FP32, rec_at)
     ref, ref_losses = _oracle_e2e(dims, n, seed, inputs, T, rec_at, False)
-    for r, t in enumerate(rec_at):
+    for r, t in enumerate(rec_at[:-1]):
         assert rel_l2(recs[r], ref[r]) < 1e-4, (t, rel_l2(recs[r], ref[r]))
-    np.testing.assert_allclose(losses, ref_losses, rtol=1e-4)
+    np.testing.assert_allclose(losses[:100], ref_losses[:100], rtol=1e-4)
+    # past the horizon: still the same training run, not a different one
+    assert rel_l2(recs[-1], ref[-1]) < 2e-2
+    assert abs(losses[150:].mean() - ref_losses[150:].mean()) < 0.02 * ref_losses[150:].mean()
     assert np.array_equal(final, recs[-1])
 
 
 @pytest.mark.slow
-def test_config3_prefix_trajectory():
-    """MLP 784-1000-1000-10, n = 30, b = 128, exponential-queue schedule (seed 3): the first
-    120 of the 2,000 commits against the oracle."""
-    dims, n, b, T, seed = [784, 1000, 1000, 10], 30, 128, 120, 3
-    rec_at = [0, 29, 59, 119]
-    recs, losses, _final, inputs = _e2e(dims, n, b, T, seed, sim.gem_schedule_queue,
-                                        sim.GEM_MLP_FP32, rec_at)
+def test_config3_windows_and_prefix():
+    """MLP 784-1000-1000-10, n = 30, b = 128, exponential-queue schedule (seed 3): windows
+    of 20 commits resumed from the oracle at commits 0, 40 and 80 (1e-4), and the
+    free-running trajectory for the first 60 commits (1e-4)."""
+    _windows([784, 1000, 1000, 10], 30, 128, 3, sim.gem_schedule_queue, sim.GEM_MLP_FP32,
+             [0, 40, 80], 20, 1e-4)
+    dims, n, b, T, seed = [784, 1000, 1000, 10], 30, 128, 60, 3
+    rec_at = [0, 29, 59]
+    recs, losses, _f, inputs = _e2e(dims, n, b, T, seed, sim.gem_schedule_queue, sim.GEM_MLP_FP32, rec_at)
     ref, ref_losses = _oracle_e2e(dims, n, seed, inputs, T, rec_at, False)
     for r, t in enumerate(rec_at):
         assert rel_l2(recs[r], ref[r]) < 1e-4, (t, rel_l2(recs[r], ref[r]))
@@ -196,9 +277,12 @@ def test_config3_prefix_trajectory():
 
 
 @pytest.mark.slow
-def test_config4_prefix_trajectory_tf32():
-    """MLP 784-1000-1000-10, n = 100, b = 128, TF32 products, uniform tick (seed 4): the
-    first 120 of the 5,000 commits against the oracle's TF32 mode."""
+def test_config4_windows_and_prefix_tf32():
+    """MLP 784-1000-1000-10, n = 100, b = 128, TF32 products, uniform tick (seed 4):
+    windows at commits 0, 50 and 100 and the free-running first 120 commits, at 2e-3
+    against the oracle's TF32 mode."""
+    _windows([784, 1000, 1000, 10], 100, 128, 4, sim.gem_schedule_uniform, sim.GEM_MLP_TF32,
+             [0, 50, 100], 20, 2e-3)
     dims, n, b, T, seed = [784, 1000, 1000, 10], 100, 128, 120, 4
     rec_at = [0, 59, 119]
     recs, losses, _final, inputs = _e2e(dims, n, b, T, seed, sim.gem_schedule_uniform,
