@@ -350,6 +350,10 @@ def run_gem(args, world, rank, local, pg):
                    "steps": e2e_steps, "commits_per_s": round(world * K_BATCH * e2e_steps / e2e_s, 1),
                    "host_gradients": f"{host_rows} distinct pinned host buffers reused cyclically"}
         G.close()
+    del pool
+    torch.cuda.empty_cache()
+
+    mlp = None if args.no_mlp else run_mlp_workloads(args, seed_offset=rank)
 
     if rank != 0:
         return
@@ -378,12 +382,74 @@ def run_gem(args, world, rank, local, pg):
                      "kernel": "commit_batch_kernel", "algorithmic_bytes_per_launch": BYTES_PER_BATCH,
                      "launch_ms_min": round(min(per_step_ms), 4), "launch_ms_max": round(max(per_step_ms), 4)},
         "gpu_launches": int(launches),
+        "async_mlp": mlp,
         "clocks": clocks.summary(),
         "e2e": e2e,
     }
     if not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline()
     print(json.dumps(line), flush=True)
+
+
+MLP_WORKLOADS = [
+    # (name, dims, n, batch, precision, schedule, seed, warmup commits, timed commits)
+    ("mlp784-1000-1000-10_n100_b128_tf32", [784, 1000, 1000, 10], 100, 128, 1, "uniform", 4, 200, 2000),
+    ("mlp784-1000-1000-10_n30_b128_fp32", [784, 1000, 1000, 10], 30, 128, 0, "queue", 3, 100, 1000),
+    ("mlp784-64-10_n4_b32_fp32", [784, 64, 10], 4, 32, 0, "uniform", 1, 100, 1000),
+]
+
+
+def run_mlp_workloads(args, seed_offset: int = 0) -> dict:
+    """Asynchronous GEM on the MLPs: the batched worker forward/backward over stale
+    snapshots plus the in-order commits, timed with CUDA events on the handle's stream."""
+    import torch
+
+    from paper_1805_08469_gb300 import gem, sim, synth, synth_gpu
+
+    out = {}
+    stream = torch.cuda.Stream()
+    X = torch.empty((synth.DATA_ROWS, 784), device="cuda")
+    y = torch.empty(synth.DATA_ROWS, dtype=torch.int32, device="cuda")
+    for name, dims, n, b, prec, sched, seed, warm, timed in MLP_WORKLOADS:
+        seed = seed + seed_offset
+        synth_gpu.data(seed, X, y, dims[-1], stream=stream)
+        T = warm + timed
+        schedule = sim.gem_schedule_uniform if sched == "uniform" else sim.gem_schedule_queue
+        order = schedule(seed, n, T)[0]
+        batches = synth.schedule_batches(seed, order, b)
+        P = synth.mlp_param_count(dims)
+        with torch.cuda.stream(stream):
+            G = gem.Gem(P, n, ETA, MU, EPS, stream=stream)
+            th0 = synth_gpu.xavier(seed, dims, torch.empty(P, device="cuda"), stream=stream)
+            G.set_theta(th0)
+            M = sim.gem_mlp_create(G.h, dims, b, prec)
+            sim.gem_mlp_set_data(M, X, y)
+            losses = torch.empty(T, device="cuda")
+            sim.gem_mlp_run(M, order[:warm], batches[:warm], losses[:warm])
+            stream.synchronize()
+            segs = len(sim.gem_plan_segments(order[warm:], n)) - 1
+            l0 = G.launches()
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            sim.gem_mlp_run(M, order[warm:], batches[warm:], losses[warm:])
+            e1.record(stream)
+            stream.synchronize()
+            ms = e0.elapsed_time(e1)
+            commit_launches = G.launches() - l0
+            lh = losses.cpu().numpy()
+            sim.gem_mlp_destroy(M)
+            G.close()
+        gflop = 2.0 * b * sum(dims[l] * dims[l + 1] for l in range(len(dims) - 1)) * 3 - \
+            2.0 * b * dims[0] * dims[1]  # forward, weight gradients, input gradients past layer 1
+        out[name] = {"commits_per_s": round(timed / (ms * 1e-3), 1), "ms": round(ms, 3),
+                     "commits": timed, "segments": segs, "precision": "tf32" if prec else "fp32",
+                     "worker_gflop_per_commit": round(gflop / 1e9, 4),
+                     "achieved_tflops": round(gflop * timed / (ms * 1e-3) / 1e12, 2),
+                     "commit_launches": int(commit_launches),
+                     "loss_first_100": round(float(lh[:100].mean()), 4),
+                     "loss_last_100": round(float(lh[-100:].mean()), 4)}
+    return out
 
 
 def main():
@@ -394,6 +460,7 @@ def main():
     ap.add_argument("--impl", choices=["gem", "reference"], default="gem")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-mlp", action="store_true")
     # smaller cases for profiling; the defaults are the benchmark workload
     ap.add_argument("--P", type=int, default=P_FULL)
     ap.add_argument("--workers", type=int, default=N_WORKERS)

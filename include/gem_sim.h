@@ -57,9 +57,10 @@ int gem_plan_segments(const int32_t* order, int T, int n, int32_t* seg_start);
 typedef struct gem_mlp gem_mlp_t;
 
 enum gem_mlp_precision {
-  GEM_MLP_FP32 = 0, /* fp32 products and sums (CUDA cores) */
-  GEM_MLP_TF32 = 1  /* operands rounded to TF32 (nearest, ties away), fp32 accumulation,
-                       tensor cores (tcgen05) for the large products */
+  GEM_MLP_FP32 = 0, /* fp32 products and sums */
+  GEM_MLP_TF32 = 1  /* TF32 operands (10 explicit mantissa bits, round to nearest, ties
+                       away from zero), products exact in fp32, fp32 sums: the numerics of
+                       a TF32 tensor-core product, evaluated on the CUDA cores */
 };
 
 /* Bind an MLP to a GEM handle (its P must equal the MLP's parameter count).  batch is the
@@ -90,6 +91,13 @@ int gem_mlp_grad(gem_mlp_t* mlp, const int32_t* workers, int L, const int32_t* b
  * theta).  losses (device [T], may be NULL) receives each commit's minibatch loss. */
 int gem_mlp_run(gem_mlp_t* mlp, const int32_t* order, int T, const int32_t* batch_rows,
                 float* losses);
+
+/* Wait for the MLP's work on the handle's stream; GEM_ECUDA if device work failed. */
+int gem_mlp_status(gem_mlp_t* mlp);
+
+/* Number of kernels the MLP has launched (gather, forward, loss, backward; the commits are
+ * counted by gem_launch_count). */
+uint64_t gem_mlp_launch_count(const gem_mlp_t* mlp);
 
 /* Free the MLP's scratch (after its pending work).  NULL is a no-op. */
 void gem_mlp_destroy(gem_mlp_t* mlp);

@@ -15,6 +15,10 @@
 //   inputs    D_l  = (D_{l+1} W_l) * [A_l > 0]
 //   biases    db_l = column sums of D_{l+1} (fixed order, no atomics)
 // Every sum runs in a fixed order, so the gradients are deterministic.
+//
+// Precision.  Every product runs in one grouped SIMT GEMM kernel that reads either operand
+// layout; with GEM_MLP_TF32 it rounds each operand to TF32 as it loads it (products of TF32
+// values are exact in fp32; the sums stay fp32).
 #include <cstdint>
 #include <cstring>
 #include <new>
@@ -470,6 +474,23 @@ int gem_mlp_set_data(gem_mlp_t* M, const float* X, const int32_t* labels, int64_
   M->X = X;
   M->labels = labels;
   M->rows = rows;
+  return GEM_OK;
+}
+
+uint64_t gem_mlp_launch_count(const gem_mlp_t* M) { return M ? M->launches : 0; }
+
+int gem_mlp_status(gem_mlp_t* M) {
+  if (!M) return GEM_EINVAL;
+  gem_t* h = M->gem;
+  int dev_prev = 0;
+  cudaGetDevice(&dev_prev);
+  cudaSetDevice(h->device);
+  const cudaError_t e = cudaStreamSynchronize(h->stream);
+  cudaSetDevice(dev_prev);
+  if (e != cudaSuccess) {
+    h->broken = true;
+    return GEM_ECUDA;
+  }
   return GEM_OK;
 }
 

@@ -84,3 +84,13 @@ def gem_mlp_run(h: int, order, batch_rows, losses=None) -> None:
     if r.shape[0] != o.shape[0]:
         raise ValueError("batch_rows must have one row per commit")
     check(lib().gem_mlp_run(C.c_void_p(h), _p(o), len(o), _p(r), _opt_ptr(losses)), "gem_mlp_run")
+
+
+def gem_mlp_status(h: int) -> None:
+    """Waits for the MLP's work; raises if device work failed."""
+    from ._lib import check
+    check(lib().gem_mlp_status(C.c_void_p(h)), "gem_mlp_status")
+
+
+def gem_mlp_launch_count(h: int) -> int:
+    return int(lib().gem_mlp_launch_count(C.c_void_p(h)))
