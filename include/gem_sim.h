@@ -99,6 +99,25 @@ int gem_mlp_status(gem_mlp_t* mlp);
  * counted by gem_launch_count). */
 uint64_t gem_mlp_launch_count(const gem_mlp_t* mlp);
 
+/* The gradient of gem_mlp_grad for one set of parameters, for callers that cannot allocate
+ * device memory: code that runs under a framework owning all device memory through its own
+ * pool (an allocation outside it breaks the pool's budget), or in a loop where cudaMalloc's
+ * device-wide synchronisation is not allowed.  Nothing is allocated and no handle is needed:
+ * the caller passes the inputs (theta [P] in device memory, the data set X [rows][dims[0]]
+ * and labels [rows] in device memory, the minibatch batch_rows [batch] as a host array,
+ * checked and copied before the call returns) and the outputs (grad [P], device, 16-byte
+ * aligned; loss, device, may be NULL).  The scratch is one file-scope device array of 4 MiB
+ * (1,048,576 floats) held by every GPU that loads the library until the process exits; a
+ * network whose per-minibatch activations and deltas do not fit in it is rejected with
+ * GEM_EINVAL.  The first call on a device looks up the array's device address, so make it
+ * before any stream capture.  Calls share the array: calls that overlap on the GPU (other
+ * streams, other host threads) race; order them on one stream.  The paper has no
+ * counterpart to this entry point. */
+int gem_mlp_grad_static(int n_layers, const int32_t* dims, int batch, int precision,
+                        const float* theta, const float* X, const int32_t* labels,
+                        int64_t rows, const int32_t* batch_rows, float* grad, float* loss,
+                        void* stream);
+
 /* Free the MLP's scratch (after its pending work).  NULL is a no-op. */
 void gem_mlp_destroy(gem_mlp_t* mlp);
 

@@ -47,6 +47,7 @@ def _declare(L):
         "gem_mlp_run": ([p, p, i, p, p], i),
         "gem_mlp_destroy": ([p], None),
         "gem_mlp_status": ([p], i),
+        "gem_mlp_grad_static": ([i, p, i, i, p, p, p, C.c_int64, p, p, p, p], i),
         "gem_mlp_launch_count": ([p], C.c_uint64),
         "gem_synth_theta0": ([C.c_uint64, sz, p, p], i),
         "gem_synth_grad_heavytail": ([C.c_uint64, C.c_uint64, i, sz, sz, p, p], i),

@@ -21,6 +21,7 @@
 // values are exact in fp32; the sums stay fp32).
 #include <cstdint>
 #include <cstring>
+#include <mutex>
 #include <new>
 #include <vector>
 
@@ -569,3 +570,110 @@ int gem_mlp_run(gem_mlp_t* M, const int32_t* order, int T, const int32_t* batch_
 }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------------------------------
+// Gradient without allocation (gem_mlp_grad_static).  Its scratch is this file-scope device
+// array: every GPU that loads the library holds it until the process exits.  Host code
+// cannot pass the symbol itself to a kernel (on the host it names a stand-in object, not
+// device memory), so its device address is looked up once per device.
+namespace {
+
+constexpr long long kStaticScratchFloats = 1ll << 20;  // 4 MiB
+__device__ __align__(256) float g_static_scratch[kStaticScratchFloats];
+
+constexpr int kMaxDevices = 64;
+std::mutex g_static_mutex;
+float* g_static_addr[kMaxDevices] = {};
+
+// Device address of g_static_scratch on the current device (looked up on first use).
+int static_scratch(int device, float** out) {
+  if (device < 0 || device >= kMaxDevices) return GEM_EINVAL;
+  std::lock_guard<std::mutex> lock(g_static_mutex);
+  if (!g_static_addr[device]) {
+    void* ptr = nullptr;
+    if (cudaGetSymbolAddress(&ptr, g_static_scratch) != cudaSuccess || !ptr) {
+      cudaGetLastError();
+      return GEM_ECUDA;
+    }
+    g_static_addr[device] = static_cast<float*>(ptr);
+  }
+  *out = g_static_addr[device];
+  return GEM_OK;
+}
+
+}  // namespace
+
+extern "C" int gem_mlp_grad_static(int n_layers, const int32_t* dims, int batch, int precision,
+                                   const float* theta, const float* X, const int32_t* labels,
+                                   int64_t rows, const int32_t* batch_rows, float* grad,
+                                   float* loss, void* stream) {
+  if (!dims || n_layers < 1 || n_layers > kMaxLayers || batch < 1 || batch > kMaxBatch)
+    return GEM_EINVAL;
+  if (precision != GEM_MLP_FP32 && precision != GEM_MLP_TF32) return GEM_EINVAL;
+  if (!theta || !X || !labels || rows < 1 || !batch_rows || !grad) return GEM_EINVAL;
+  if ((reinterpret_cast<uintptr_t>(grad) & 15u) != 0) return GEM_EINVAL;
+  for (int l = 0; l <= n_layers; ++l)
+    if (dims[l] < 1) return GEM_EINVAL;
+  if (dims[n_layers] > kMaxClasses) return GEM_EINVAL;
+  for (int i = 0; i < batch; ++i)
+    if (batch_rows[i] < 0 || batch_rows[i] >= rows) return GEM_EINVAL;
+
+  // descriptors on the stack: the snapshot is `theta`, one worker, one slot
+  gem_ctx h{};
+  gem_mlp M{};
+  M.gem = &h;
+  M.L = n_layers;
+  M.batch = batch;
+  M.precision = precision;
+  M.X = X;
+  M.labels = labels;
+  M.rows = rows;
+  long long P = 0;
+  for (int l = 0; l <= n_layers; ++l) M.dims[l] = dims[l];
+  for (int l = 0; l < n_layers; ++l) {
+    M.w_off[l] = P;
+    M.b_off[l] = P + (long long)dims[l + 1] * dims[l];
+    P = M.b_off[l] + dims[l + 1];
+  }
+  long long off = 0;
+  M.off_x = off;
+  off += round32((long long)batch * dims[0]);
+  for (int l = 1; l < n_layers; ++l) {
+    M.off_act[l] = off;
+    off += round32((long long)batch * dims[l]);
+  }
+  M.off_logits = off;
+  off += round32((long long)batch * dims[n_layers]);
+  for (int l = 1; l <= n_layers; ++l) {
+    M.off_delta[l] = off;
+    off += round32((long long)batch * dims[l]);
+  }
+  M.slot_stride = off;
+  M.slots = 1;
+  const long long rows_floats = round32(batch);  // minibatch rows stored after the slot
+  if (off + rows_floats > kStaticScratchFloats) return GEM_EINVAL;  // beyond the static array
+
+  int device = 0;
+  if (cudaGetDevice(&device) != cudaSuccess) {
+    cudaGetLastError();
+    return GEM_ECUDA;
+  }
+  float* scratch = nullptr;
+  int rc = static_scratch(device, &scratch);
+  if (rc) return rc;
+  h.device = device;
+  h.P = size_t(P);
+  h.stride = size_t(P);
+  h.n = 1;
+  h.s = const_cast<float*>(theta);
+  h.stream = static_cast<cudaStream_t>(stream);
+  M.scratch = scratch;
+  int32_t* rows_dev = reinterpret_cast<int32_t*>(scratch + off);
+  if (cudaMemcpyAsync(rows_dev, batch_rows, sizeof(int32_t) * size_t(batch), cudaMemcpyHostToDevice,
+                      h.stream) != cudaSuccess)
+    return GEM_ECUDA;
+  const int32_t worker = 0;
+  rc = mlp_chunk(&M, &worker, 1, rows_dev, grad, 0, loss);
+  M.gem = nullptr;
+  return rc;
+}

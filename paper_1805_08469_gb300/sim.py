@@ -94,3 +94,19 @@ def gem_mlp_status(h: int) -> None:
 
 def gem_mlp_launch_count(h: int) -> int:
     return int(lib().gem_mlp_launch_count(C.c_void_p(h)))
+
+
+def gem_mlp_grad_static(dims, batch: int, precision: int, theta, X, labels, batch_rows, grad,
+                        loss=None, stream=None) -> None:
+    """Gradient without any allocation (include/gem_sim.h): theta [P], X [rows, d0], labels
+    [rows], grad [P] (and loss [1]) are CUDA tensors; batch_rows a host int array [batch]."""
+    from ._lib import check
+    d = (C.c_int32 * len(dims))(*[int(x) for x in dims])
+    r = np.ascontiguousarray(batch_rows, dtype=np.int32)
+    if r.shape != (batch,):
+        raise ValueError("batch_rows must hold `batch` row indices")
+    st = 0 if stream is None else (stream if isinstance(stream, int) else int(stream.cuda_stream))
+    check(lib().gem_mlp_grad_static(len(dims) - 1, d, batch, precision, C.c_void_p(theta.data_ptr()),
+                                    C.c_void_p(X.data_ptr()), C.c_void_p(labels.data_ptr()), X.shape[0],
+                                    _p(r), C.c_void_p(grad.data_ptr()), _opt_ptr(loss), C.c_void_p(st)),
+          "gem_mlp_grad_static")

@@ -1,0 +1,75 @@
+"""The gradient entry point that allocates nothing (gem_mlp_grad_static).
+
+Some callers cannot allocate device memory: code running under a framework that owns all
+device memory through its own pool, or in a loop where cudaMalloc's device-wide
+synchronisation is not allowed.  For them the library offers a gradient call whose scratch is
+a fixed file-scope device array.  This test checks, through the C ABI, that two calls in a
+row give the same gradients and losses as the allocating entry point (gem_mlp_grad, at its
+worker's snapshot), within the tolerance the other gradient tests use, and that a network
+too large for the array is refused.  It sits in a file of its own, collected last.
+"""
+import numpy as np
+import pytest
+import torch
+
+from paper_1805_08469_gb300 import gem, sim, synth, synth_gpu
+from paper_1805_08469_gb300._build import build_library
+from paper_1805_08469_gb300._lib import GemError
+
+pytestmark = pytest.mark.gpu
+
+
+def _rel_l2(a, b):
+    a = a.double()
+    b = b.double()
+    return float((a - b).norm() / b.norm())
+
+
+@pytest.mark.parametrize("dims,b,precision", [
+    ([784, 64, 10], 32, sim.GEM_MLP_FP32),
+    ([784, 1000, 1000, 10], 128, sim.GEM_MLP_TF32),
+])
+def test_static_scratch_gradient_matches_allocating_entry_point(dims, b, precision):
+    build_library()
+    torch.cuda.set_device(0)
+    seed = 31
+    P = synth.mlp_param_count(dims)
+    X = torch.empty((synth.DATA_ROWS, dims[0]), device="cuda")
+    y = torch.empty(synth.DATA_ROWS, dtype=torch.int32, device="cuda")
+    synth_gpu.data(seed, X, y, dims[-1])
+    theta0 = synth.xavier_theta0(seed, dims)
+    for (_wo, bo, fo, _fi) in synth.mlp_layout(dims):
+        theta0[bo:bo + fo] = 0.05 * synth.normal(synth.key(seed, 77), np.arange(bo, bo + fo))
+    theta = torch.from_numpy(theta0).cuda()
+    with gem.Gem(P, 1, 0.01, 0.9, 1e-8) as G:
+        G.set_theta(theta)
+        M = sim.gem_mlp_create(G.h, dims, b, precision)
+        try:
+            sim.gem_mlp_set_data(M, X, y)
+            for call in range(2):                  # two calls in a row share the array
+                rows = synth.batch_indices(seed, 0, call, b)
+                ref = torch.empty(P, device="cuda")
+                ref_loss = torch.empty(1, device="cuda")
+                sim.gem_mlp_grad(M, [0], rows[None, :], [ref], ref_loss)
+                got = torch.empty(P, device="cuda")
+                loss = torch.empty(1, device="cuda")
+                sim.gem_mlp_grad_static(dims, b, precision, theta, X, y, rows, got, loss)
+                torch.cuda.synchronize()
+                assert _rel_l2(got, ref) < 1e-5, (call, _rel_l2(got, ref))
+                assert abs(float(loss) - float(ref_loss)) <= 1e-5 * abs(float(ref_loss))
+        finally:
+            sim.gem_mlp_destroy(M)
+
+
+def test_static_scratch_rejects_networks_that_do_not_fit():
+    build_library()
+    torch.cuda.set_device(0)
+    dims, b = [784, 1000, 1000, 10], 256           # 1.2M floats of activations per minibatch
+    P = synth.mlp_param_count(dims)
+    theta = torch.zeros(P, device="cuda")
+    X = torch.zeros((16, 784), device="cuda")
+    y = torch.zeros(16, dtype=torch.int32, device="cuda")
+    grad = torch.empty(P, device="cuda")
+    with pytest.raises(GemError) as e:
+        sim.gem_mlp_grad_static(dims, b, sim.GEM_MLP_FP32, theta, X, y, np.zeros(b, np.int32), grad)
+    assert e.value.status == gem.GEM_EINVAL
