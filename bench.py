@@ -322,8 +322,9 @@ def run_gem(args, world, rank, local, pg):
         total_ms = max_over_ranks(pg, total_ms)
         barrier(pg)
 
-        # end to end through the public API: gradients in pinned host memory, copied in
-        # each step, and theta read back to the host after each step
+        # end to end through the public API: gradients in pinned host memory, read by the
+        # commit kernel in place over the host link every step, and theta read back to the
+        # host after each step
         e2e = None
         if not args.no_e2e:
             host_rows = 16
@@ -348,7 +349,8 @@ def run_gem(args, world, rank, local, pg):
             e2e = {"value": round(world * BYTES_PER_BATCH * e2e_steps / e2e_s / 1e9, 1), "unit": "GB/s",
                    "h2d_bytes_per_step": K_BATCH * P_FULL * 4, "d2h_bytes_per_step": P_FULL * 4,
                    "steps": e2e_steps, "commits_per_s": round(world * K_BATCH * e2e_steps / e2e_s, 1),
-                   "host_gradients": f"{host_rows} distinct pinned host buffers reused cyclically"}
+                   "host_gradients": f"{host_rows} distinct pinned host buffers reused cyclically, "
+                                     "read in place by the commit kernel (host link about 210 GB/s)"}
         G.close()
     del pool
     torch.cuda.empty_cache()

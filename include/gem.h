@@ -94,12 +94,13 @@ int gem_commit(gem_t* h, int worker, const float* grad);
  * no-op) and 0 <= order[k] < n. */
 int gem_commit_batch(gem_t* h, const int* order, const float* const* grads, int K);
 
-/* As gem_commit_batch, with each grads[k] in host memory instead (page-locked memory
- * gives full copy bandwidth).  The gradients are copied to library-owned device staging
- * buffers on a second stream, in chunks that overlap with the commits of earlier chunks.
- * The host buffers must stay valid and unmodified until the handle's stream has
- * finished the batch.  The staging buffers are allocated by the first call (at most 16
- * gradients of `stride` floats). */
+/* As gem_commit_batch, with each grads[k] in host memory instead.  When every gradient is
+ * page-locked (cudaHostAlloc / cudaHostRegister) and 16-byte aligned, the commit kernel
+ * reads them in place over the host link and nothing is copied.  Otherwise the gradients
+ * are copied to library-owned device staging buffers on a second stream, in chunks that
+ * overlap with the commits of earlier chunks; those buffers are allocated by the first such
+ * call (16 gradients of `stride` floats).  Either way the host buffers must stay valid and
+ * unmodified until the handle's stream has finished the batch. */
 int gem_commit_batch_host(gem_t* h, const int* order, const float* const* grads, int K);
 
 /* *theta receives the device address of theta [P] (borrowed, read-only, valid until

@@ -3,6 +3,7 @@
 #include <cstdint>
 #include <cstdlib>
 #include <new>
+#include <vector>
 
 #include "gem_internal.h"
 
@@ -265,6 +266,24 @@ int gem_commit_batch_host(gem_t* h, const int* order, const float* const* grads,
   if (K == 0) return GEM_OK;
   DeviceScope scope(h->device);
   if (!scope.ok()) return GEM_ECUDA;
+  // Page-locked host memory is readable by the device in place (over the host link): when
+  // every gradient is, the commit kernel reads them there and nothing is staged.
+  {
+    std::vector<const float*> dev(static_cast<size_t>(K));
+    bool in_place = true;
+    for (int k = 0; k < K && in_place; ++k) {
+      cudaPointerAttributes attr;
+      if (cudaPointerGetAttributes(&attr, grads[k]) != cudaSuccess) {
+        cudaGetLastError();
+        in_place = false;
+        break;
+      }
+      in_place = attr.type == cudaMemoryTypeHost && attr.devicePointer != nullptr &&
+                 aligned16(attr.devicePointer);
+      dev[size_t(k)] = static_cast<const float*>(attr.devicePointer);
+    }
+    if (in_place) return launch_commits(h, order, dev.data(), K);
+  }
   rc = ensure_staging(h);
   if (rc) return rc;
   // Chunk j uses staging half j % 2: the copy stream fills it once the commits that last

@@ -11,15 +11,35 @@
 //
 // Per coordinate and commit the kernel streams 12 bytes in (g, m_w, s_w) and 8 bytes
 // out (m_w, s_w); theta adds 8 bytes per launch.  The path is HBM-bound (about 0.5 flop
-// per byte), so the design goals are coalesced 128-bit accesses, enough independent
-// loads in flight per SM, and evict-first cache hints on the streamed vectors so that
-// theta and the next batch's lines are not pushed out of L2.
+// per byte), so the design goals are coalesced 128-bit accesses and enough independent
+// loads in flight per SM (one 16-byte lane per thread, 512 threads per block).  The
+// gradients are read with an evict-first hint (a gradient is used once per batch); the
+// rows of m_w and s_w are cached normally, so a worker that commits again a few commits
+// later in the same batch finds them in L2 and DRAM traffic drops below the algorithmic
+// 20 bytes per parameter and commit.
 #include "gem_internal.h"
+
+// Launch shape: threads per block, 16-byte lanes per thread, and a minimum number of
+// resident blocks per SM (0: let the compiler choose registers freely).
+#ifndef GEM_COMMIT_THREADS
+#define GEM_COMMIT_THREADS 512
+#endif
+#ifndef GEM_COMMIT_LANES
+#define GEM_COMMIT_LANES 1
+#endif
+#ifndef GEM_COMMIT_MIN_BLOCKS
+#define GEM_COMMIT_MIN_BLOCKS 0
+#endif
+// Cache policy of the moment and snapshot rows: 1 streams them (evict-first), 0 caches them
+// normally so that a worker that commits again soon finds its rows in L2.
+#ifndef GEM_COMMIT_STREAM_STATE
+#define GEM_COMMIT_STREAM_STATE 0
+#endif
 
 namespace gem {
 namespace {
 
-constexpr int kThreads = 256;
+constexpr int kThreads = GEM_COMMIT_THREADS;
 
 // One coordinate of one commit.  One IEEE fp32 operation per step, rounded to nearest,
 // no contraction into FMA (the __f*_rn intrinsics are never fused), IEEE division.
@@ -36,6 +56,22 @@ __device__ __forceinline__ void commit_coord(float& theta, float& m, float& s, f
   s = theta;                                                     // s <- theta
 }
 
+__device__ __forceinline__ float4 load_state(const float4* p) {
+#if GEM_COMMIT_STREAM_STATE
+  return __ldcs(p);
+#else
+  return *p;
+#endif
+}
+
+__device__ __forceinline__ void store_state(float4* p, float4 v) {
+#if GEM_COMMIT_STREAM_STATE
+  __stcs(p, v);
+#else
+  *p = v;
+#endif
+}
+
 __device__ __forceinline__ void commit_vec(float4& th, float4& m, float4& s, const float4 g,
                                            float eta, float mu, float eps) {
   commit_coord(th.x, m.x, s.x, g.x, eta, mu, eps);
@@ -47,7 +83,7 @@ __device__ __forceinline__ void commit_vec(float4& th, float4& m, float4& s, con
 // L independent 16-byte lanes per thread, strided by the grid so that each warp
 // touches 512 contiguous bytes per lane and array.
 template <int L>
-__global__ void __launch_bounds__(kThreads)
+__global__ void __launch_bounds__(kThreads, GEM_COMMIT_MIN_BLOCKS)
 commit_batch_kernel(const __grid_constant__ BatchArgs a) {
   const size_t nvec = a.P >> 2;
   const size_t nthreads = size_t(gridDim.x) * kThreads;
@@ -72,8 +108,8 @@ commit_batch_kernel(const __grid_constant__ BatchArgs a) {
         const size_t i = base + size_t(l) * nthreads;
         if (i < nvec) {
           g[l] = __ldcs(g4 + i);
-          m[l] = __ldcs(m4 + i);
-          s[l] = __ldcs(s4 + i);
+          m[l] = load_state(m4 + i);
+          s[l] = load_state(s4 + i);
         }
       }
 #pragma unroll
@@ -81,8 +117,8 @@ commit_batch_kernel(const __grid_constant__ BatchArgs a) {
         const size_t i = base + size_t(l) * nthreads;
         if (i < nvec) {
           commit_vec(th[l], m[l], s[l], g[l], a.eta, a.mu, a.eps);
-          __stcs(m4 + i, m[l]);
-          __stcs(s4 + i, s[l]);
+          store_state(m4 + i, m[l]);
+          store_state(s4 + i, s[l]);
         }
       }
     }
@@ -110,7 +146,7 @@ commit_batch_kernel(const __grid_constant__ BatchArgs a) {
   }
 }
 
-constexpr int kLanes = 2;
+constexpr int kLanes = GEM_COMMIT_LANES;
 
 }  // namespace
 

@@ -102,17 +102,21 @@ def test_host_gradient_batch_equals_device_batch():
     host = [torch.from_numpy(grads[k].copy()).pin_memory() if k % 2 else torch.from_numpy(grads[k].copy())
             for k in range(K)]
     g_dev = _padded(grads)
-    with gem.Gem(P, n, ETA, MU, EPS) as A, gem.Gem(P, n, ETA, MU, EPS) as B:
-        A.set_theta(torch.from_numpy(theta0).cuda())
-        B.set_theta(torch.from_numpy(theta0).cuda())
+    pinned = [torch.from_numpy(grads[k].copy()).pin_memory() for k in range(K)]
+    with gem.Gem(P, n, ETA, MU, EPS) as A, gem.Gem(P, n, ETA, MU, EPS) as B, \
+            gem.Gem(P, n, ETA, MU, EPS) as Z:
+        for H in (A, B, Z):
+            H.set_theta(torch.from_numpy(theta0).cuda())
         A.commit_batch(order, [g_dev[k, :P] for k in range(K)])
-        B.commit_batch_host(order, host)
-        A.sync()
-        B.sync()
-        assert torch.equal(A.theta(), B.theta())
-        for w in range(n):
-            assert torch.equal(A.moment(w), B.moment(w))
-            assert torch.equal(A.snapshot(w), B.snapshot(w))
+        B.commit_batch_host(order, host)      # some pageable: staged copies
+        Z.commit_batch_host(order, pinned)    # all page-locked: read in place
+        for H in (A, B, Z):
+            H.sync()
+        for H in (B, Z):
+            assert torch.equal(A.theta(), H.theta())
+            for w in range(n):
+                assert torch.equal(A.moment(w), H.moment(w))
+                assert torch.equal(A.snapshot(w), H.snapshot(w))
         out = torch.empty(P, dtype=torch.float32).pin_memory()
         gem.gem_read_theta(B.h, out)
         B.sync()
