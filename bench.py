@@ -44,8 +44,8 @@ FALLBACK_HBM_GBS = 6800.0
 # DRAM traffic of one launch of the batched commit kernel, from an ncu capture of the
 # same workload (see profiles/commit_batch_p25m_n100.md).  Valid only for the kernel
 # source it was taken on; reported as null once that source changes.
-NCU_TRAFFIC_BYTES_PER_LAUNCH = None
-NCU_TRAFFIC_SOURCE_SHA = None
+NCU_TRAFFIC_BYTES_PER_LAUNCH = 44_734_500_000   # mean of two full-size launches
+NCU_TRAFFIC_SOURCE_SHA = "24881a78b514977c"
 
 
 def kernel_source_sha() -> str:
