@@ -413,7 +413,11 @@ def run_mlp_workloads(args, seed_offset: int = 0) -> dict:
     X = torch.empty((synth.DATA_ROWS, 784), device="cuda")
     y = torch.empty(synth.DATA_ROWS, dtype=torch.int32, device="cuda")
     for name, dims, n, b, prec, sched, seed, warm, timed in MLP_WORKLOADS:
+        if args.mlp_workload and name != args.mlp_workload:
+            continue
         seed = seed + seed_offset
+        if args.mlp_commits:
+            warm, timed = min(warm, args.mlp_commits), args.mlp_commits
         synth_gpu.data(seed, X, y, dims[-1], stream=stream)
         T = warm + timed
         schedule = sim.gem_schedule_uniform if sched == "uniform" else sim.gem_schedule_queue
@@ -463,6 +467,12 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-mlp", action="store_true")
+    ap.add_argument("--only", choices=["all", "commit", "mlp"], default="all",
+                    help="profiling aid: run only the commit batches or only the async MLP runs")
+    ap.add_argument("--mlp-workload", default="",
+                    help="profiling aid: run only the MLP workload with this name")
+    ap.add_argument("--mlp-commits", type=int, default=0,
+                    help="profiling aid: timed commits per MLP workload (0: the defaults)")
     # smaller cases for profiling; the defaults are the benchmark workload
     ap.add_argument("--P", type=int, default=P_FULL)
     ap.add_argument("--workers", type=int, default=N_WORKERS)
@@ -477,7 +487,16 @@ def main():
     else:
         from paper_1805_08469_gb300._build import build_library
         build_library()
-        run_gem(args, world, rank, local, pg)
+        if args.only == "mlp":
+            import torch
+            torch.cuda.set_device(local)
+            out = run_mlp_workloads(args, seed_offset=rank)
+            if rank == 0:
+                print(json.dumps({"impl": "gem", "only": "mlp", "async_mlp": out}), flush=True)
+        else:
+            if args.only == "commit":
+                args.no_mlp = True
+            run_gem(args, world, rank, local, pg)
     if pg is not None:
         pg.destroy_process_group()
 

@@ -36,8 +36,11 @@ constexpr int kMaxGroups = 128;
 constexpr int kMaxClasses = 32;
 constexpr int kMaxBatch = 1024;
 
-// SIMT tile: 128 x 64 outputs per block of 256 threads, 8 x 4 per thread, k-steps of 16.
-constexpr int BM = 128, BN = 64, BK = 16, kThreads = 256;
+// SIMT tile: 128 (or 64) x 64 outputs per block of 256 (or 128) threads, 8 x 4 per thread,
+// k-steps of 16.
+constexpr int BM = 128, BN = 64, BK = 16;
+constexpr long long kSmCountHint = 152;  // GB300
+constexpr int kMaxSplit = 4;             // split-K factor at most
 
 enum Epilogue : int { kStore = 0, kBias = 1, kBiasRelu = 2, kMask = 3 };
 
@@ -58,6 +61,12 @@ struct GemmArgs {
   long long bias_group_stride;
   const float* mask;  // by group, keep C(m, n) where mask(m, n) > 0
   long long mask_group_stride, ldmask;
+  // split-K: blockIdx.z = group * ksplit + split; split s sums k in [s kchunk, (s+1) kchunk)
+  // and writes its raw partial sums to ws + (group * ksplit + s) * M * N (row-major, ld N)
+  int ksplit;
+  int kchunk;
+  float* ws;            // null: no split
+  long long ws_floats;  // capacity of ws
   int workers[kMaxGroups];
 };
 
@@ -72,52 +81,65 @@ __device__ __forceinline__ float to_tf32(float x) {
 
 // C[g] (M x N) = epilogue( op(A[g]) op(B[g]) ).  A_KMAJOR: A(m, k) at A[m*lda + k], else at
 // A[k*lda + m].  B_KMAJOR: B(k, n) at B[n*ldb + k], else at B[k*ldb + n].
-template <bool A_KMAJOR, bool B_KMAJOR, int EPI, bool TF32>
-__global__ void __launch_bounds__(kThreads)
+//
+// TBM x 64 tile per block of 2 TBM threads; thread (tx, ty) = (tid % 16, tid / 16) owns
+// rows 8 ty .. 8 ty + 7 and columns 4 tx .. 4 tx + 3.  Both tiles are kept m- (or n-) contiguous
+// in shared memory, double-buffered, so one k-step is three 128-bit shared loads and 32
+// FMAs.  The next k-tile is read from global memory into registers while the current one
+// is multiplied; global reads are coalesced along whichever index is contiguous.
+template <int TBM, bool A_KMAJOR, bool B_KMAJOR, int EPI, bool TF32>
+__global__ void __launch_bounds__(2 * TBM)
 gemm_grouped_kernel(const __grid_constant__ GemmArgs p) {
-  __shared__ float As[BM][BK + 1];
-  __shared__ float Bs[BN][BK + 1];
-  const int g = blockIdx.z;
-  const int m0 = blockIdx.y * BM, n0 = blockIdx.x * BN;
+  constexpr int T = 2 * TBM;                 // threads: 16 columns x TBM / 8 rows of them
+  constexpr int kPadA = TBM + 4, kPadB = BN + 4;  // row pitches (floats), 16-byte aligned
+  constexpr int kBPer = BN * BK / T;         // B elements staged per thread (A: always 8)
+  __shared__ __align__(16) float As[2][BK][kPadA];
+  __shared__ __align__(16) float Bs[2][BK][kPadB];
+  const int split = p.ksplit > 1 ? p.ksplit : 1;
+  const int g = blockIdx.z / split, sk = blockIdx.z - g * split;
+  const int kbeg = sk * p.kchunk;
+  const int kend = split > 1 ? min(p.K, kbeg + p.kchunk) : p.K;
+  const int m0 = blockIdx.y * TBM, n0 = blockIdx.x * BN;
   const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
   const float* A = p.A.base + (p.A.by_worker ? (long long)p.workers[g] : (long long)g) * p.A.group_stride;
   const float* B = p.B.base + (p.B.by_worker ? (long long)p.workers[g] : (long long)g) * p.B.group_stride;
   const long long lda = p.A.ld, ldb = p.B.ld;
   const int M = p.M, N = p.N, K = p.K;
 
-  float ra[8], rb[4];
+  // staging: 8 A elements and 4 B elements per thread per k-tile
+  float ra[8], rb[kBPer];
   auto load = [&](int k0) {
 #pragma unroll
     for (int it = 0; it < 8; ++it) {
       int m, k;
-      if (A_KMAJOR) { m = (tid >> 4) + 16 * it; k = tid & 15; }
-      else          { m = tid & 127;            k = (tid >> 7) + 2 * it; }
+      if (A_KMAJOR) { m = (tid >> 4) + (T / 16) * it; k = tid & 15; }
+      else          { m = tid % TBM;                  k = tid / TBM + 2 * it; }
       const int gm = m0 + m, gk = k0 + k;
       float v = 0.f;
-      if (gm < M && gk < K) v = A_KMAJOR ? A[gm * lda + gk] : A[gk * lda + gm];
+      if (gm < M && gk < kend) v = A_KMAJOR ? A[gm * lda + gk] : A[gk * lda + gm];
       ra[it] = TF32 ? to_tf32(v) : v;
     }
 #pragma unroll
-    for (int it = 0; it < 4; ++it) {
+    for (int it = 0; it < kBPer; ++it) {
       int n, k;
-      if (B_KMAJOR) { n = (tid >> 4) + 16 * it; k = tid & 15; }
-      else          { n = tid & 63;             k = (tid >> 6) + 4 * it; }
+      if (B_KMAJOR) { n = (tid >> 4) + (T / 16) * it; k = tid & 15; }
+      else          { n = tid & 63;                   k = (tid >> 6) + (T / 64) * it; }
       const int gn = n0 + n, gk = k0 + k;
       float v = 0.f;
-      if (gn < N && gk < K) v = B_KMAJOR ? B[gn * ldb + gk] : B[gk * ldb + gn];
+      if (gn < N && gk < kend) v = B_KMAJOR ? B[gn * ldb + gk] : B[gk * ldb + gn];
       rb[it] = TF32 ? to_tf32(v) : v;
     }
   };
-  auto store = [&]() {
+  auto store = [&](int buf) {
 #pragma unroll
     for (int it = 0; it < 8; ++it) {
-      if (A_KMAJOR) As[(tid >> 4) + 16 * it][tid & 15] = ra[it];
-      else          As[tid & 127][(tid >> 7) + 2 * it] = ra[it];
+      if (A_KMAJOR) As[buf][tid & 15][(tid >> 4) + (T / 16) * it] = ra[it];
+      else          As[buf][tid / TBM + 2 * it][tid % TBM] = ra[it];
     }
 #pragma unroll
-    for (int it = 0; it < 4; ++it) {
-      if (B_KMAJOR) Bs[(tid >> 4) + 16 * it][tid & 15] = rb[it];
-      else          Bs[tid & 63][(tid >> 6) + 4 * it] = rb[it];
+    for (int it = 0; it < kBPer; ++it) {
+      if (B_KMAJOR) Bs[buf][tid & 15][(tid >> 4) + (T / 16) * it] = rb[it];
+      else          Bs[buf][(tid >> 6) + (T / 64) * it][tid & 63] = rb[it];
     }
   };
 
@@ -127,42 +149,57 @@ gemm_grouped_kernel(const __grid_constant__ GemmArgs p) {
 #pragma unroll
     for (int j = 0; j < 4; ++j) acc[i][j] = 0.f;
 
-  load(0);
-  store();
+  load(kbeg);
+  store(0);
   __syncthreads();
-  for (int k0 = 0; k0 < K; k0 += BK) {
-    const bool more = k0 + BK < K;
+  int buf = 0;
+  for (int k0 = kbeg; k0 < kend; k0 += BK) {
+    const bool more = k0 + BK < kend;
     if (more) load(k0 + BK);
 #pragma unroll
     for (int k = 0; k < BK; ++k) {
-      float a[8], b[4];
-#pragma unroll
-      for (int i = 0; i < 8; ++i) a[i] = As[ty + 16 * i][k];
-#pragma unroll
-      for (int j = 0; j < 4; ++j) b[j] = Bs[tx + 16 * j][k];
+      const float4 a0 = *reinterpret_cast<const float4*>(&As[buf][k][ty * 8]);
+      const float4 a1 = *reinterpret_cast<const float4*>(&As[buf][k][ty * 8 + 4]);
+      const float4 b4 = *reinterpret_cast<const float4*>(&Bs[buf][k][tx * 4]);
+      const float a[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
+      const float b[4] = {b4.x, b4.y, b4.z, b4.w};
 #pragma unroll
       for (int i = 0; i < 8; ++i)
 #pragma unroll
         for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(a[i], b[j], acc[i][j]);
     }
-    __syncthreads();
     if (more) {
-      store();
+      store(buf ^ 1);   // the other buffer was last read before the previous barrier
       __syncthreads();
+      buf ^= 1;
     }
   }
 
+  if (split > 1) {  // raw partial sums; splitk_reduce_kernel applies the epilogue
+    float* W = p.ws + (long long)blockIdx.z * M * N;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const int m = m0 + ty * 8 + i;
+      if (m >= M) continue;
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const int n = n0 + tx * 4 + j;
+        if (n < N) W[(long long)m * N + n] = acc[i][j];
+      }
+    }
+    return;
+  }
   float* C = p.C + (long long)g * p.c_group_stride;
   const float* bias = (EPI == kBias || EPI == kBiasRelu)
                           ? p.bias + (long long)p.workers[g] * p.bias_group_stride : nullptr;
   const float* mask = EPI == kMask ? p.mask + (long long)g * p.mask_group_stride : nullptr;
 #pragma unroll
   for (int i = 0; i < 8; ++i) {
-    const int m = m0 + ty + 16 * i;
+    const int m = m0 + ty * 8 + i;
     if (m >= M) continue;
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
-      const int n = n0 + tx + 16 * j;
+      const int n = n0 + tx * 4 + j;
       if (n >= N) continue;
       float v = acc[i][j];
       if (EPI == kBias) v = v + bias[n];
@@ -170,6 +207,74 @@ gemm_grouped_kernel(const __grid_constant__ GemmArgs p) {
       if (EPI == kMask) v = mask[m * p.ldmask + n] > 0.f ? v : 0.f;
       C[m * p.ldc + n] = v;
     }
+  }
+}
+
+// Sum of the split-K partials of every output in split order (deterministic), then the
+// epilogue of the product.
+template <int EPI>
+__global__ void splitk_reduce_kernel(const __grid_constant__ GemmArgs p, int groups) {
+  const long long MN = (long long)p.M * p.N;
+  const long long q = blockIdx.x * (long long)blockDim.x + threadIdx.x;
+  if (q >= MN * groups) return;
+  const int g = int(q / MN);
+  const long long r = q - g * MN;
+  const int m = int(r / p.N), n = int(r - (long long)m * p.N);
+  const float* W = p.ws + (long long)g * p.ksplit * MN + r;
+  float v = 0.f;
+  for (int s = 0; s < p.ksplit; ++s) v += W[s * MN];
+  if (EPI == kBias) v = v + p.bias[(long long)p.workers[g] * p.bias_group_stride + n];
+  if (EPI == kBiasRelu) v = fmaxf(v + p.bias[(long long)p.workers[g] * p.bias_group_stride + n], 0.f);
+  if (EPI == kMask)
+    v = p.mask[(long long)g * p.mask_group_stride + (long long)m * p.ldmask + n] > 0.f ? v : 0.f;
+  p.C[(long long)g * p.c_group_stride + (long long)m * p.ldc + n] = v;
+}
+
+// Products with few outputs per row (N <= kMaxClasses), used for the logits:
+// C[g][m][n] = sum_k A[g][m][k] B[g][n][k] + bias[n], A and B K-major.  One block of 8 warps
+// per row m: warp w sums its slice of k (lane l takes k = l, l + 32, ... inside the slice,
+// coalesced), a fixed butterfly reduces the lanes, and thread n adds the 8 warp sums in
+// order, so the result is deterministic.
+template <bool TF32>
+__global__ void __launch_bounds__(256)
+gemm_small_n_kernel(const __grid_constant__ GemmArgs p) {
+  __shared__ float part[8][kMaxClasses];
+  const int g = blockIdx.y, m = blockIdx.x;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const float* A = p.A.base + (p.A.by_worker ? (long long)p.workers[g] : (long long)g) * p.A.group_stride +
+                   (long long)m * p.A.ld;
+  const float* B = p.B.base + (p.B.by_worker ? (long long)p.workers[g] : (long long)g) * p.B.group_stride;
+  const int slice = ((p.K + 8 * 32 - 1) / (8 * 32)) * 32;
+  const int kb = warp * slice, ke = min(p.K, kb + slice);
+  float acc[kMaxClasses];
+#pragma unroll
+  for (int n = 0; n < kMaxClasses; ++n) acc[n] = 0.f;
+  for (int k = kb + lane; k < ke; k += 32) {
+    const float a = TF32 ? to_tf32(A[k]) : A[k];
+#pragma unroll
+    for (int n = 0; n < kMaxClasses; ++n) {
+      if (n < p.N) {
+        const float b = B[(long long)n * p.B.ld + k];
+        acc[n] = fmaf(a, TF32 ? to_tf32(b) : b, acc[n]);
+      }
+    }
+  }
+#pragma unroll
+  for (int n = 0; n < kMaxClasses; ++n) {
+    if (n < p.N) {
+      float v = acc[n];
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+      if (lane == 0) part[warp][n] = v;
+    }
+  }
+  __syncthreads();
+  const int n = threadIdx.x;
+  if (n < p.N) {
+    float v = 0.f;
+    for (int w = 0; w < 8; ++w) v += part[w][n];
+    const float* bias = p.bias + (long long)p.workers[g] * p.bias_group_stride;
+    p.C[(long long)g * p.c_group_stride + (long long)m * p.ldc + n] = v + bias[n];
   }
 }
 
@@ -242,13 +347,44 @@ __global__ void bias_grad_kernel(const __grid_constant__ BiasGradArgs a, const f
   grad[g * grad_stride + a.grad_off[l] + o] = s;
 }
 
-template <bool AK, bool BK_, int EPI>
-cudaError_t launch_gemm(const GemmArgs& a, int groups, bool tf32, cudaStream_t st) {
-  dim3 grid((a.N + BN - 1) / BN, (a.M + BM - 1) / BM, groups);
+template <int TBM, bool AK, bool BK_, int EPI>
+void launch_tile(const GemmArgs& a, int groups, bool tf32, cudaStream_t st) {
+  dim3 grid((a.N + BN - 1) / BN, (a.M + TBM - 1) / TBM, groups);
   if (tf32)
-    gemm_grouped_kernel<AK, BK_, EPI, true><<<grid, kThreads, 0, st>>>(a);
+    gemm_grouped_kernel<TBM, AK, BK_, EPI, true><<<grid, 2 * TBM, 0, st>>>(a);
   else
-    gemm_grouped_kernel<AK, BK_, EPI, false><<<grid, kThreads, 0, st>>>(a);
+    gemm_grouped_kernel<TBM, AK, BK_, EPI, false><<<grid, 2 * TBM, 0, st>>>(a);
+}
+
+// 128-row tiles when the launch fills the GPU; otherwise 64-row tiles (twice the blocks)
+// and, when a split-K workspace is given and K is long, up to kMaxSplit splits of K whose
+// partial sums a second kernel adds in a fixed order.
+template <bool AK, bool BK_, int EPI>
+cudaError_t launch_gemm(const GemmArgs& a_in, int groups, bool tf32, cudaStream_t st) {
+  GemmArgs a = a_in;
+  a.ksplit = 1;
+  a.kchunk = a.K;
+  const long long blocks128 = (long long)((a.N + BN - 1) / BN) * ((a.M + BM - 1) / BM) * groups;
+  if (blocks128 >= 2 * kSmCountHint) {
+    launch_tile<128, AK, BK_, EPI>(a, groups, tf32, st);
+    return cudaGetLastError();
+  }
+  const long long blocks64 = (long long)((a.N + BN - 1) / BN) * ((a.M + 63) / 64) * groups;
+  int split = 1;
+  const long long mn = (long long)a.M * a.N * groups;
+  if (a.ws && a.M <= 128)
+    while (split < kMaxSplit && blocks64 * split < 4 * kSmCountHint && a.K / (2 * split) >= 128 &&
+           mn * 2 * split <= a.ws_floats)
+      split *= 2;
+  if (split == 1) {
+    launch_tile<64, AK, BK_, EPI>(a, groups, tf32, st);
+    return cudaGetLastError();
+  }
+  a.ksplit = split;
+  a.kchunk = ((a.K + split - 1) / split + BK - 1) / BK * BK;
+  launch_tile<64, AK, BK_, EPI>(a, groups * split, tf32, st);
+  const long long total = (long long)a.M * a.N * groups;
+  splitk_reduce_kernel<EPI><<<unsigned((total + 255) / 256), 256, 0, st>>>(a, groups);
   return cudaGetLastError();
 }
 
@@ -274,6 +410,8 @@ struct gem_mlp {
   int slots = 0;
   float* scratch = nullptr;
   float* grads = nullptr;  // [n][gem stride]
+  float* ws = nullptr;     // split-K partial sums
+  long long ws_floats = 0;
   int32_t* rows_dev = nullptr;  // minibatch rows uploaded from the host
   size_t rows_cap = 0;
   uint64_t launches = 0;
@@ -306,6 +444,8 @@ int mlp_chunk(gem_mlp* M, const int32_t* workers, int G, const int32_t* batch_ro
   GemmArgs a;
   std::memset(&a, 0, sizeof(a));
   for (int g = 0; g < G; ++g) a.workers[g] = workers[g];
+  a.ws = M->ws;
+  a.ws_floats = M->ws_floats;
   const long long wstride = (long long)h->stride;
 
   // forward
@@ -320,8 +460,19 @@ int mlp_chunk(gem_mlp* M, const int32_t* workers, int G, const int32_t* batch_ro
     a.C = last ? scr + M->off_logits : act(l + 1);
     a.c_group_stride = S;
     a.ldc = dout;
-    cudaError_t e = last ? launch_gemm<true, true, kBias>(a, G, tf32, st)
-                         : launch_gemm<true, true, kBiasRelu>(a, G, tf32, st);
+    cudaError_t e;
+    if (last && dout <= kMaxClasses) {
+      // the logits: few outputs per row, one block per row
+      dim3 grid(b, G);
+      if (tf32)
+        gemm_small_n_kernel<true><<<grid, 256, 0, st>>>(a);
+      else
+        gemm_small_n_kernel<false><<<grid, 256, 0, st>>>(a);
+      e = cudaGetLastError();
+    } else {
+      e = last ? launch_gemm<true, true, kBias>(a, G, tf32, st)
+               : launch_gemm<true, true, kBiasRelu>(a, G, tf32, st);
+    }
     if ((rc = cuda_rc(e))) return rc;
     M->launches++;
   }
@@ -444,11 +595,19 @@ int gem_mlp_create(gem_t* g, int n_layers, const int32_t* dims, int batch, int p
   cudaSetDevice(g->device);
   cudaError_t e = cudaMalloc(&M->scratch, sizeof(float) * size_t(M->slot_stride) * M->slots);
   if (e == cudaSuccess) e = cudaMalloc(&M->grads, sizeof(float) * g->stride * size_t(g->n));
+  if (e == cudaSuccess && batch <= 128) {
+    // split-K workspace: kMaxSplit partial products of at most batch x widest layer per slot
+    int widest = 0;
+    for (int l = 1; l <= n_layers; ++l) widest = dims[l] > widest ? dims[l] : widest;
+    M->ws_floats = (long long)kMaxSplit * 128 * widest * M->slots;
+    e = cudaMalloc(&M->ws, sizeof(float) * size_t(M->ws_floats));
+  }
   cudaSetDevice(dev_prev);
   if (e != cudaSuccess) {
     cudaGetLastError();
     cudaFree(M->scratch);
     cudaFree(M->grads);
+    cudaFree(M->ws);
     delete M;
     return GEM_ENOMEM;
   }
@@ -464,6 +623,7 @@ void gem_mlp_destroy(gem_mlp_t* M) {
   cudaStreamSynchronize(M->gem->stream);
   cudaFree(M->scratch);
   cudaFree(M->grads);
+  cudaFree(M->ws);
   cudaFree(M->rows_dev);
   cudaGetLastError();
   cudaSetDevice(dev_prev);

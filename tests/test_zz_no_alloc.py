@@ -5,7 +5,7 @@ device memory through its own pool, or in a loop where cudaMalloc's device-wide
 synchronisation is not allowed.  For them the library offers a gradient call whose scratch is
 a fixed file-scope device array.  This test checks, through the C ABI, that two calls in a
 row give the same gradients and losses as the allocating entry point (gem_mlp_grad, at its
-worker's snapshot), within the tolerance the other gradient tests use, and that a network
+worker's snapshot), within the precision's rounding tolerance, and that a network
 too large for the array is refused.  It sits in a file of its own, collected last.
 """
 import numpy as np
@@ -55,8 +55,15 @@ def test_static_scratch_gradient_matches_allocating_entry_point(dims, b, precisi
                 loss = torch.empty(1, device="cuda")
                 sim.gem_mlp_grad_static(dims, b, precision, theta, X, y, rows, got, loss)
                 torch.cuda.synchronize()
-                assert _rel_l2(got, ref) < 1e-5, (call, _rel_l2(got, ref))
-                assert abs(float(loss) - float(ref_loss)) <= 1e-5 * abs(float(ref_loss))
+                # The allocating entry point splits long K sums across blocks (split-K with a
+                # workspace); this one has no workspace and sums each K in one block.  The
+                # orders differ, so the results agree to rounding: 1e-5 in fp32, and in TF32
+                # (operands rounded to 10 mantissa bits, which amplifies order differences in
+                # the deep layers) 1e-3 over the whole gradient, between the last-layer (1e-4) and
+                # deep-layer (1e-2) bars of the TF32 gradient tests.
+                bar = 1e-5 if precision == sim.GEM_MLP_FP32 else 1e-3
+                assert _rel_l2(got, ref) < bar, (call, _rel_l2(got, ref))
+                assert abs(float(loss) - float(ref_loss)) <= bar * abs(float(ref_loss))
         finally:
             sim.gem_mlp_destroy(M)
 
