@@ -128,6 +128,54 @@ int gem_sync(gem_t* h);
 /* Layout query: P, n and the row stride (in floats) of m and s.  Any output may be NULL. */
 int gem_shape(const gem_t* h, size_t* P, int* n, size_t* stride);
 
+/* Commit rules.  GEM_MODE_GEM is the rule at the top of this file and the default; the
+ * others are the comparison rules of the paper's experiments and the high-energy proxies
+ * of its Appendix B.  Each is computed in fp32, one IEEE operation per step:
+ *
+ *   GEM_MODE_GEM           Algorithm 1: the five steps above.
+ *   GEM_MODE_DOWNPOUR      the DOWNPOUR rule: theta = theta + dtheta (pi = 1), s_w = theta;
+ *                          m_w is not read or changed.
+ *   GEM_MODE_ADAPTIVE      adaptive staleness (experiments section): the update is rescaled
+ *                          by 1 / (tau + 1), pi = 1 / (tau + 1) rounded to fp32 and
+ *                          theta = theta + pi * dtheta, s_w = theta; m_w is not read or
+ *                          changed.  tau is the commit's staleness on the handle's clock
+ *                          (gem_staleness).
+ *   GEM_MODE_KAPPA_SQRT    App. B, Eq. pi_with_kappa: as GEM with |m_w| replaced by
+ *                          sqrt(kappa) * |m_w| (sqrt(kappa) rounded to fp32 first).
+ *   GEM_MODE_KAPPA_LINEAR  App. B, the modified form used in its study: as GEM with |m_w|
+ *                          replaced by kappa * |m_w|. */
+enum gem_mode {
+  GEM_MODE_GEM = 0,
+  GEM_MODE_DOWNPOUR = 1,
+  GEM_MODE_ADAPTIVE = 2,
+  GEM_MODE_KAPPA_SQRT = 3,
+  GEM_MODE_KAPPA_LINEAR = 4
+};
+
+/* Select the rule of every later commit.  kappa is the proxy's energy factor: required
+ * finite and > 0 for the two kappa modes, ignored (and reported as 1) for the others.
+ * Host-side only: takes effect for commits issued after the call. */
+int gem_set_mode(gem_t* h, int mode, float kappa);
+
+/* Current rule and kappa.  Either output may be NULL. */
+int gem_get_mode(const gem_t* h, int* mode, float* kappa);
+
+/* Staleness bookkeeping.  The handle numbers commits 0, 1, 2, ... in the order they are
+ * issued (its clock, reset to 0 by gem_set_theta).  A worker pulls right after its own
+ * commit, so the staleness of a commit by w at clock t is the number of commits by the
+ * other workers since then: tau = t - last_w - 1, with last_w the clock value of w's
+ * previous commit, or -1 before its first.  *tau receives the staleness that w's next
+ * commit will have. */
+int gem_staleness(const gem_t* h, int worker, int64_t* tau);
+
+/* The clock and last[w] for each of the n workers (last may be NULL); with gem_save_state
+ * this is the whole of a checkpoint. */
+int gem_get_clock(const gem_t* h, int64_t* clock, int64_t* last);
+
+/* Restore the clock: clock >= 0 and -1 <= last[w] < clock for every worker (last NULL: -1
+ * for all).  Returns GEM_EINVAL and changes nothing if a value is out of range. */
+int gem_set_clock(gem_t* h, int64_t clock, const int64_t* last);
+
 /* Number of kernels this handle has launched since it was created. */
 uint64_t gem_launch_count(const gem_t* h);
 

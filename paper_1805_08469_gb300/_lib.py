@@ -37,6 +37,11 @@ def _declare(L):
         "gem_sync": ([p], i),
         "gem_shape": ([p, p, p, p], i),
         "gem_launch_count": ([p], C.c_uint64),
+        "gem_set_mode": ([p, i, C.c_float], i),
+        "gem_get_mode": ([p, p, p], i),
+        "gem_staleness": ([p, i, p], i),
+        "gem_get_clock": ([p, p, p], i),
+        "gem_set_clock": ([p, C.c_int64, p], i),
         "gem_status_string": ([i], C.c_char_p),
         "gem_schedule_uniform": ([C.c_uint64, i, i, p, p], i),
         "gem_schedule_queue": ([C.c_uint64, i, i, C.c_double, p, p], i),

@@ -1,5 +1,6 @@
 // Host side of the GEM commit ABI (include/gem.h): handle life cycle, argument checks,
 // stream plumbing and the staging of host-resident gradients.
+#include <cmath>
 #include <cstdint>
 #include <cstdlib>
 #include <new>
@@ -43,35 +44,9 @@ int check_handle(const gem_t* h) {
   return GEM_OK;
 }
 
-gem::BatchArgs base_args(const gem_t* h) {
-  gem::BatchArgs a;
-  a.theta = h->theta;
-  a.m = h->m;
-  a.s = h->s;
-  a.P = h->P;
-  a.stride = h->stride;
-  a.eta = h->eta;
-  a.mu = h->mu;
-  a.eps = h->eps;
-  a.K = 0;
-  return a;
-}
-
-// Launch the commits [0, K) in chunks of at most kMaxBatchPerLaunch, in order.
+// Launch the commits [0, K) in order; GEM_ECUDA marks the handle broken.
 int launch_commits(gem_t* h, const int* order, const float* const* grads, int K) {
-  gem::BatchArgs a = base_args(h);
-  for (int k0 = 0; k0 < K; k0 += gem::kMaxBatchPerLaunch) {
-    const int kc = (K - k0) < gem::kMaxBatchPerLaunch ? (K - k0) : gem::kMaxBatchPerLaunch;
-    a.K = kc;
-    for (int k = 0; k < kc; ++k) {
-      a.worker[k] = order[k0 + k];
-      a.grad[k] = grads[k0 + k];
-    }
-    const int rc = cuda_status(h, gem::launch_commit_batch(a, h->sm_count, h->stream));
-    if (rc) return rc;
-    h->launches += 1;
-  }
-  return GEM_OK;
+  return cuda_status(h, gem::commit_ordered(h, order, grads, K));
 }
 
 int check_batch(const gem_t* h, const int* order, const float* const* grads, int K) {
@@ -102,6 +77,59 @@ int ensure_staging(gem_t* h) {
 
 }  // namespace
 
+namespace gem {
+
+cudaError_t commit_ordered(gem_ctx* h, const int* order, const float* const* grads, int K) {
+  BatchArgs a;
+  a.theta = h->theta;
+  a.m = h->m;
+  a.s = h->s;
+  a.P = h->P;
+  a.stride = h->stride;
+  a.eta = h->eta;
+  a.mu = h->mu;
+  a.eps = h->eps;
+  a.energy_scale = 1.f;
+  switch (h->mode) {
+    case GEM_MODE_KAPPA_SQRT:
+      a.rule = kRuleScaled;
+      a.energy_scale = sqrtf(h->kappa);  // correctly rounded fp32 square root
+      break;
+    case GEM_MODE_KAPPA_LINEAR:
+      a.rule = kRuleScaled;
+      a.energy_scale = h->kappa;
+      break;
+    case GEM_MODE_DOWNPOUR:
+    case GEM_MODE_ADAPTIVE:
+      a.rule = kRuleFixed;
+      break;
+    default:
+      a.rule = kRuleGem;
+      break;
+  }
+  for (int k0 = 0; k0 < K; k0 += kMaxBatchPerLaunch) {
+    const int kc = (K - k0) < kMaxBatchPerLaunch ? (K - k0) : kMaxBatchPerLaunch;
+    a.K = kc;
+    for (int k = 0; k < kc; ++k) {
+      const int w = order[k0 + k];
+      a.worker[k] = w;
+      a.grad[k] = grads[k0 + k];
+      // staleness: commits by the other workers since w's last commit (and pull)
+      const int64_t tau = h->clock - h->last[size_t(w)] - 1;
+      h->last[size_t(w)] = h->clock;
+      h->clock += 1;
+      // adaptive staleness: pi = 1 / (tau + 1) in fp32 (IEEE division); DOWNPOUR: pi = 1
+      a.pi[k] = h->mode == GEM_MODE_ADAPTIVE ? 1.0f / (static_cast<float>(tau) + 1.0f) : 1.0f;
+    }
+    const cudaError_t e = launch_commit_batch(a, h->sm_count, h->stream);
+    if (e != cudaSuccess) return e;
+    h->launches += 1;
+  }
+  return cudaSuccess;
+}
+
+}  // namespace gem
+
 extern "C" {
 
 const char* gem_status_string(int status) {
@@ -130,6 +158,12 @@ int gem_create(size_t P, int n, float eta, float mu, float eps, gem_t** out) {
   h->eta = eta;
   h->mu = mu;
   h->eps = eps;
+  try {
+    h->last.assign(size_t(n), -1);
+  } catch (...) {
+    delete h;
+    return GEM_ENOMEM;
+  }
   if (cudaGetDevice(&h->device) != cudaSuccess ||
       cudaDeviceGetAttribute(&h->sm_count, cudaDevAttrMultiProcessorCount, h->device) !=
           cudaSuccess) {
@@ -200,7 +234,54 @@ int gem_set_theta(gem_t* h, const float* theta0) {
     e = cudaMemcpyAsync(h->s + size_t(w) * h->stride, h->theta, row, cudaMemcpyDeviceToDevice,
                         h->stream);
   if (e == cudaSuccess) e = cudaMemsetAsync(h->m, 0, size_t(h->n) * row, h->stream);
+  h->clock = 0;
+  for (auto& t : h->last) t = -1;
   return cuda_status(h, e);
+}
+
+int gem_set_mode(gem_t* h, int mode, float kappa) {
+  int rc = check_handle(h);
+  if (rc) return rc;
+  if (mode < GEM_MODE_GEM || mode > GEM_MODE_KAPPA_LINEAR) return GEM_EINVAL;
+  if ((mode == GEM_MODE_KAPPA_SQRT || mode == GEM_MODE_KAPPA_LINEAR) &&
+      !(kappa > 0.0f && kappa <= 3.0e38f))
+    return GEM_EINVAL;
+  h->mode = mode;
+  h->kappa = (mode == GEM_MODE_KAPPA_SQRT || mode == GEM_MODE_KAPPA_LINEAR) ? kappa : 1.0f;
+  return GEM_OK;
+}
+
+int gem_get_mode(const gem_t* h, int* mode, float* kappa) {
+  if (!h) return GEM_EINVAL;
+  if (mode) *mode = h->mode;
+  if (kappa) *kappa = h->kappa;
+  return GEM_OK;
+}
+
+int gem_get_clock(const gem_t* h, int64_t* clock, int64_t* last) {
+  if (!h) return GEM_EINVAL;
+  if (clock) *clock = h->clock;
+  if (last)
+    for (int w = 0; w < h->n; ++w) last[w] = h->last[size_t(w)];
+  return GEM_OK;
+}
+
+int gem_set_clock(gem_t* h, int64_t clock, const int64_t* last) {
+  int rc = check_handle(h);
+  if (rc) return rc;
+  if (clock < 0) return GEM_EINVAL;
+  if (last)
+    for (int w = 0; w < h->n; ++w)
+      if (last[w] < -1 || last[w] >= clock) return GEM_EINVAL;
+  h->clock = clock;
+  for (int w = 0; w < h->n; ++w) h->last[size_t(w)] = last ? last[w] : -1;
+  return GEM_OK;
+}
+
+int gem_staleness(const gem_t* h, int worker, int64_t* tau) {
+  if (!h || !tau || worker < 0 || worker >= h->n) return GEM_EINVAL;
+  *tau = h->clock - h->last[size_t(worker)] - 1;
+  return GEM_OK;
 }
 
 int gem_pull(gem_t* h, int worker, const float** snapshot) {

@@ -43,17 +43,30 @@ constexpr int kThreads = GEM_COMMIT_THREADS;
 
 // One coordinate of one commit.  One IEEE fp32 operation per step, rounded to nearest,
 // no contraction into FMA (the __f*_rn intrinsics are never fused), IEEE division.
+// RULE kRuleGem takes |m_w| as the root of twice the proxy energy (Eq. proxy_estimate);
+// kRuleScaled multiplies it by `scale` first (sqrt(kappa) or kappa, App. B).
+template <int RULE>
 __device__ __forceinline__ void commit_coord(float& theta, float& m, float& s, float g,
-                                             float eta, float mu, float eps) {
+                                             float eta, float mu, float eps, float scale) {
   const float dtheta = -__fmul_rn(eta, g);                       // -eta grad L(s)
   const float m_new = __fadd_rn(__fmul_rn(mu, m), dtheta);       // m <- mu m + dtheta
   const float drift = fabsf(__fsub_rn(theta, s));                // |theta - s|
-  float pi = __fdiv_rn(__fsub_rn(fabsf(m_new), drift),           // (|m| - |theta - s|)
+  const float energy = RULE == kRuleScaled ? __fmul_rn(scale, fabsf(m_new)) : fabsf(m_new);
+  float pi = __fdiv_rn(__fsub_rn(energy, drift),                 // (|m| - |theta - s|)
                        __fadd_rn(fabsf(dtheta), eps));           //   / (|dtheta| + eps)
   pi = pi > 0.0f ? pi : 0.0f;                                    // pi >= 0
   theta = __fadd_rn(theta, __fmul_rn(pi, dtheta));               // theta + pi dtheta
   m = m_new;
   s = theta;                                                     // s <- theta
+}
+
+// A commit with a given scaling factor (kRuleFixed): theta + pi dtheta, s <- theta; the
+// moment is not part of these rules.
+__device__ __forceinline__ void commit_coord_fixed(float& theta, float& s, float g, float eta,
+                                                   float pi) {
+  const float dtheta = -__fmul_rn(eta, g);
+  theta = __fadd_rn(theta, __fmul_rn(pi, dtheta));
+  s = theta;
 }
 
 __device__ __forceinline__ float4 load_state(const float4* p) {
@@ -72,17 +85,27 @@ __device__ __forceinline__ void store_state(float4* p, float4 v) {
 #endif
 }
 
+template <int RULE>
 __device__ __forceinline__ void commit_vec(float4& th, float4& m, float4& s, const float4 g,
-                                           float eta, float mu, float eps) {
-  commit_coord(th.x, m.x, s.x, g.x, eta, mu, eps);
-  commit_coord(th.y, m.y, s.y, g.y, eta, mu, eps);
-  commit_coord(th.z, m.z, s.z, g.z, eta, mu, eps);
-  commit_coord(th.w, m.w, s.w, g.w, eta, mu, eps);
+                                           float eta, float mu, float eps, float scale) {
+  commit_coord<RULE>(th.x, m.x, s.x, g.x, eta, mu, eps, scale);
+  commit_coord<RULE>(th.y, m.y, s.y, g.y, eta, mu, eps, scale);
+  commit_coord<RULE>(th.z, m.z, s.z, g.z, eta, mu, eps, scale);
+  commit_coord<RULE>(th.w, m.w, s.w, g.w, eta, mu, eps, scale);
+}
+
+__device__ __forceinline__ void commit_vec_fixed(float4& th, float4& s, const float4 g, float eta,
+                                                 float pi) {
+  commit_coord_fixed(th.x, s.x, g.x, eta, pi);
+  commit_coord_fixed(th.y, s.y, g.y, eta, pi);
+  commit_coord_fixed(th.z, s.z, g.z, eta, pi);
+  commit_coord_fixed(th.w, s.w, g.w, eta, pi);
 }
 
 // L independent 16-byte lanes per thread, strided by the grid so that each warp
-// touches 512 contiguous bytes per lane and array.
-template <int L>
+// touches 512 contiguous bytes per lane and array.  The fixed-factor rules read only the
+// gradient and write only s_w (12 bytes less per coordinate and commit).
+template <int L, int RULE>
 __global__ void __launch_bounds__(kThreads, GEM_COMMIT_MIN_BLOCKS)
 commit_batch_kernel(const __grid_constant__ BatchArgs a) {
   const size_t nvec = a.P >> 2;
@@ -108,16 +131,22 @@ commit_batch_kernel(const __grid_constant__ BatchArgs a) {
         const size_t i = base + size_t(l) * nthreads;
         if (i < nvec) {
           g[l] = __ldcs(g4 + i);
-          m[l] = load_state(m4 + i);
-          s[l] = load_state(s4 + i);
+          if (RULE != kRuleFixed) {
+            m[l] = load_state(m4 + i);
+            s[l] = load_state(s4 + i);
+          }
         }
       }
 #pragma unroll
       for (int l = 0; l < L; ++l) {
         const size_t i = base + size_t(l) * nthreads;
         if (i < nvec) {
-          commit_vec(th[l], m[l], s[l], g[l], a.eta, a.mu, a.eps);
-          store_state(m4 + i, m[l]);
+          if (RULE == kRuleFixed) {
+            commit_vec_fixed(th[l], s[l], g[l], a.eta, a.pi[k]);
+          } else {
+            commit_vec<RULE>(th[l], m[l], s[l], g[l], a.eta, a.mu, a.eps, a.energy_scale);
+            store_state(m4 + i, m[l]);
+          }
           store_state(s4 + i, s[l]);
         }
       }
@@ -137,9 +166,15 @@ commit_batch_kernel(const __grid_constant__ BatchArgs a) {
     float th = a.theta[j];
     for (int k = 0; k < a.K; ++k) {
       const size_t row = size_t(a.worker[k]) * a.stride;
-      float m = a.m[row + j], s = a.s[row + j];
-      commit_coord(th, m, s, a.grad[k][j], a.eta, a.mu, a.eps);
-      a.m[row + j] = m;
+      float s;
+      if (RULE == kRuleFixed) {
+        commit_coord_fixed(th, s, a.grad[k][j], a.eta, a.pi[k]);
+      } else {
+        float m = a.m[row + j];
+        s = a.s[row + j];
+        commit_coord<RULE>(th, m, s, a.grad[k][j], a.eta, a.mu, a.eps, a.energy_scale);
+        a.m[row + j] = m;
+      }
       a.s[row + j] = s;
     }
     a.theta[j] = th;
@@ -148,13 +183,12 @@ commit_batch_kernel(const __grid_constant__ BatchArgs a) {
 
 constexpr int kLanes = GEM_COMMIT_LANES;
 
-}  // namespace
-
-cudaError_t launch_commit_batch(const BatchArgs& a, int sm_count, cudaStream_t stream) {
+template <int RULE>
+cudaError_t launch_rule(const BatchArgs& a, int sm_count, cudaStream_t stream) {
   static int blocks_per_sm = 0;
   if (blocks_per_sm == 0) {
     cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(
-        &blocks_per_sm, commit_batch_kernel<kLanes>, kThreads, 0);
+        &blocks_per_sm, commit_batch_kernel<kLanes, RULE>, kThreads, 0);
     if (e != cudaSuccess) return e;
     if (blocks_per_sm < 1) blocks_per_sm = 1;
   }
@@ -169,8 +203,19 @@ cudaError_t launch_commit_batch(const BatchArgs& a, int sm_count, cudaStream_t s
     grid = (nvec + rounds * per_block - 1) / (rounds * per_block);
   }
   if (grid < 1) grid = 1;
-  commit_batch_kernel<kLanes><<<unsigned(grid), kThreads, 0, stream>>>(a);
+  commit_batch_kernel<kLanes, RULE><<<unsigned(grid), kThreads, 0, stream>>>(a);
   return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_commit_batch(const BatchArgs& a, int sm_count, cudaStream_t stream) {
+  switch (a.rule) {
+    case kRuleGem: return launch_rule<kRuleGem>(a, sm_count, stream);
+    case kRuleScaled: return launch_rule<kRuleScaled>(a, sm_count, stream);
+    case kRuleFixed: return launch_rule<kRuleFixed>(a, sm_count, stream);
+    default: return cudaErrorInvalidValue;
+  }
 }
 
 }  // namespace gem

@@ -5,6 +5,7 @@
 
 #include <cstddef>
 #include <cstdint>
+#include <vector>
 
 #include "../../include/gem.h"
 
@@ -21,6 +22,13 @@ constexpr size_t kStrideAlign = 32;
 // Host-gradient staging for gem_commit_batch_host: two halves of kStageChunk slots.
 constexpr int kStageChunk = 8;
 
+// How a launch scales each commit.
+enum RuleKind : int {
+  kRuleGem = 0,     // pi from energy matching with the proxy |m_w| (Algorithm 1)
+  kRuleScaled = 1,  // the same with the proxy energy_scale |m_w| (App. B, high-energy proxies)
+  kRuleFixed = 2,   // pi[k] given per commit; m_w untouched (DOWNPOUR, adaptive staleness)
+};
+
 struct BatchArgs {
   float* theta;                            // [stride]
   float* m;                                // [n][stride]
@@ -29,8 +37,11 @@ struct BatchArgs {
   size_t stride;
   float eta, mu, eps;
   int K;                                   // commits in this launch, 1..kMaxBatchPerLaunch
+  int rule;                                // RuleKind
+  float energy_scale;                      // kRuleScaled: factor on |m_w|
   const float* grad[kMaxBatchPerLaunch];   // gradient of commit k, P floats
   int worker[kMaxBatchPerLaunch];          // worker of commit k
+  float pi[kMaxBatchPerLaunch];            // kRuleFixed: scaling factor of commit k
 };
 
 // Launch the fused commit kernel for a.K commits on `stream`.
@@ -51,9 +62,23 @@ struct gem_ctx {
   cudaStream_t stream = nullptr;
   uint64_t launches = 0;
   bool broken = false;
+  // commit rule (gem_set_mode) and the commit clock the staleness is counted on
+  int mode = GEM_MODE_GEM;
+  float kappa = 1.f;
+  int64_t clock = 0;           // commits issued since gem_set_theta
+  std::vector<int64_t> last;   // [n] clock value of worker w's last commit, -1 before its first
   // staging of host gradients (gem_commit_batch_host), allocated on first use
   float* stage = nullptr;
   cudaStream_t copy_stream = nullptr;
   cudaEvent_t stage_filled[2] = {nullptr, nullptr};
   cudaEvent_t stage_free[2] = {nullptr, nullptr};
 };
+
+namespace gem {
+
+// Launch commits [0, K) of the handle in order, in chunks of kMaxBatchPerLaunch, with the
+// handle's commit rule; advances the commit clock and counts the launches.  The arguments
+// must have been checked.
+cudaError_t commit_ordered(gem_ctx* h, const int* order, const float* const* grads, int K);
+
+}  // namespace gem

@@ -696,15 +696,7 @@ int gem_mlp_run(gem_mlp_t* M, const int32_t* order, int T, const int32_t* batch_
   cudaGetDevice(&dev_prev);
   cudaSetDevice(h->device);
   int rc = upload_rows(M, batch_rows, (long long)T * M->batch);
-  gem::BatchArgs ca;
-  ca.theta = h->theta;
-  ca.m = h->m;
-  ca.s = h->s;
-  ca.P = h->P;
-  ca.stride = h->stride;
-  ca.eta = h->eta;
-  ca.mu = h->mu;
-  ca.eps = h->eps;
+  std::vector<const float*> gptr(size_t(T) > 0 ? size_t(T) : 1);
   for (int i = 0; i < S && rc == GEM_OK; ++i) {
     const int a = seg[i], e = seg[i + 1];
     for (int c0 = a; c0 < e && rc == GEM_OK; c0 += M->slots) {
@@ -713,15 +705,9 @@ int gem_mlp_run(gem_mlp_t* M, const int32_t* order, int T, const int32_t* batch_
                      M->grads + (long long)(c0 - a) * h->stride, (long long)h->stride,
                      losses ? losses + c0 : nullptr);
     }
-    for (int k0 = a; k0 < e && rc == GEM_OK; k0 += gem::kMaxBatchPerLaunch) {
-      const int kc = (e - k0) < gem::kMaxBatchPerLaunch ? (e - k0) : gem::kMaxBatchPerLaunch;
-      ca.K = kc;
-      for (int k = 0; k < kc; ++k) {
-        ca.worker[k] = order[k0 + k];
-        ca.grad[k] = M->grads + (long long)(k0 + k - a) * h->stride;
-      }
-      rc = cuda_rc(gem::launch_commit_batch(ca, h->sm_count, h->stream));
-      h->launches++;
+    if (rc == GEM_OK) {
+      for (int k = a; k < e; ++k) gptr[size_t(k)] = M->grads + (long long)(k - a) * h->stride;
+      rc = cuda_rc(gem::commit_ordered(h, order + a, gptr.data() + a, e - a));
     }
   }
   if (rc == GEM_ECUDA) h->broken = true;

@@ -17,6 +17,12 @@ GEM_ENOMEM = -2
 GEM_ECUDA = -3
 GEM_ESTATE = -4
 
+GEM_MODE_GEM = 0
+GEM_MODE_DOWNPOUR = 1
+GEM_MODE_ADAPTIVE = 2
+GEM_MODE_KAPPA_SQRT = 3
+GEM_MODE_KAPPA_LINEAR = 4
+
 
 def _dev_ptr(t, what: str) -> int:
     """Address of a contiguous fp32 CUDA tensor (or an int address)."""
@@ -167,6 +173,36 @@ def gem_launch_count(h: int) -> int:
     return int(lib().gem_launch_count(C.c_void_p(h)))
 
 
+def gem_set_mode(h: int, mode: int, kappa: float = 1.0) -> None:
+    check(lib().gem_set_mode(C.c_void_p(h), int(mode), float(kappa)), "gem_set_mode")
+
+
+def gem_get_mode(h: int) -> tuple[int, float]:
+    mode = C.c_int()
+    kappa = C.c_float()
+    check(lib().gem_get_mode(C.c_void_p(h), C.byref(mode), C.byref(kappa)), "gem_get_mode")
+    return int(mode.value), float(kappa.value)
+
+
+def gem_staleness(h: int, worker: int) -> int:
+    tau = C.c_int64()
+    check(lib().gem_staleness(C.c_void_p(h), int(worker), C.byref(tau)), "gem_staleness")
+    return int(tau.value)
+
+
+def gem_get_clock(h: int, n: int):
+    """(clock, last[n]) of the handle's commit clock."""
+    clock = C.c_int64()
+    last = (C.c_int64 * n)()
+    check(lib().gem_get_clock(C.c_void_p(h), C.byref(clock), last), "gem_get_clock")
+    return int(clock.value), [int(x) for x in last]
+
+
+def gem_set_clock(h: int, clock: int, last=None) -> None:
+    arr = None if last is None else (C.c_int64 * len(last))(*[int(x) for x in last])
+    check(lib().gem_set_clock(C.c_void_p(h), int(clock), arr), "gem_set_clock")
+
+
 class _DeviceArray:
     """Exposes a borrowed device address as a CUDA array (zero-copy torch view)."""
 
@@ -235,3 +271,15 @@ class Gem:
 
     def launches(self) -> int:
         return gem_launch_count(self.h)
+
+    def set_mode(self, mode: int, kappa: float = 1.0):
+        gem_set_mode(self.h, mode, kappa)
+
+    def staleness(self, worker: int) -> int:
+        return gem_staleness(self.h, worker)
+
+    def clock(self):
+        return gem_get_clock(self.h, self.n)
+
+    def set_clock(self, clock: int, last=None):
+        gem_set_clock(self.h, clock, last)
