@@ -37,9 +37,11 @@ enum Mode : int {
 };
 
 // One worker's commit on one coordinate (Algorithm 1, procedures Worker and Psi_GEM,
-// followed by the master's update of Eq. update_psi).
+// followed by the master's update of Eq. update_psi).  Returns the scaling factor pi the
+// commit applied to this coordinate (the per-parameter value whose median the experiments
+// section reports).
 template <typename T>
-inline void commit_coordinate(T& theta, T& m, T& s, T g, T eta, T mu, T eps, int mode,
+inline T commit_coordinate(T& theta, T& m, T& s, T g, T eta, T mu, T eps, int mode,
                               T kappa, int tau, int precommit_snapshot) {
   // Worker: the update is plain SGD on the snapshot, dtheta = -eta * grad L(s).
   const T dtheta = -(eta * g);
@@ -67,6 +69,7 @@ inline void commit_coordinate(T& theta, T& m, T& s, T g, T eta, T mu, T eps, int
   theta = theta_pulled + pi * dtheta;
   // s <- theta: the worker's next gradient is taken at the post-commit central variable.
   s = precommit_snapshot ? theta_pulled : theta;
+  return pi;
 }
 
 template <typename T>
@@ -74,7 +77,7 @@ int run(int64_t P, int n, int T_commits, const int32_t* order, const int32_t* ta
         const T* grads, int64_t grad_stride, const int32_t* grad_index, T* theta, T* m,
         T* s, int64_t state_stride, double eta_d, double mu_d, double eps_d, int mode,
         double kappa_d, int precommit_snapshot, const int64_t* record_cols, int n_record,
-        T* record) {
+        T* record, T* pi_record) {
   if (P < 0 || n < 1 || T_commits < 0 || !order || !grads || !theta || !m || !s) return -1;
   if (state_stride < P) return -1;
   const T eta = T(eta_d), mu = T(mu_d), eps = T(eps_d), kappa = T(kappa_d);
@@ -86,9 +89,12 @@ int run(int64_t P, int n, int T_commits, const int32_t* order, const int32_t* ta
     T* mw = m + int64_t(w) * state_stride;
     T* sw = s + int64_t(w) * state_stride;
     const int tw = tau ? tau[t] : 0;
-    for (int64_t j = 0; j < P; ++j)
-      commit_coordinate<T>(theta[j], mw[j], sw[j], g[j], eta, mu, eps, mode, kappa, tw,
-                           precommit_snapshot);
+    T* pi_row = pi_record ? pi_record + int64_t(t) * P : nullptr;
+    for (int64_t j = 0; j < P; ++j) {
+      const T pi = commit_coordinate<T>(theta[j], mw[j], sw[j], g[j], eta, mu, eps, mode, kappa,
+                                        tw, precommit_snapshot);
+      if (pi_row) pi_row[j] = pi;
+    }
     if (record && n_record > 0)
       for (int r = 0; r < n_record; ++r) record[int64_t(t) * n_record + r] = theta[record_cols[r]];
   }
@@ -112,7 +118,7 @@ int oracle_gem_run_f32(int64_t P, int n, int T, const int32_t* order, const int3
                        float* record) {
   return run<float>(P, n, T, order, tau, grads, grad_stride, grad_index, theta, m, s,
                     state_stride, eta, mu, eps, mode, kappa, precommit_snapshot,
-                    record_cols, n_record, record);
+                    record_cols, n_record, record, nullptr);
 }
 
 int oracle_gem_run_f64(int64_t P, int n, int T, const int32_t* order, const int32_t* tau,
@@ -123,7 +129,29 @@ int oracle_gem_run_f64(int64_t P, int n, int T, const int32_t* order, const int3
                        double* record) {
   return run<double>(P, n, T, order, tau, grads, grad_stride, grad_index, theta, m, s,
                      state_stride, eta, mu, eps, mode, kappa, precommit_snapshot,
-                     record_cols, n_record, record);
+                     record_cols, n_record, record, nullptr);
+}
+
+// As oracle_gem_run_f32 / _f64, and when pi_record is not NULL the scaling factor pi of
+// every coordinate of commit t is written to pi_record[t][0..P).
+int oracle_gem_run_pi_f32(int64_t P, int n, int T, const int32_t* order, const int32_t* tau,
+                          const float* grads, int64_t grad_stride, const int32_t* grad_index,
+                          float* theta, float* m, float* s, int64_t state_stride, double eta,
+                          double mu, double eps, int mode, double kappa,
+                          int precommit_snapshot, float* pi_record) {
+  return run<float>(P, n, T, order, tau, grads, grad_stride, grad_index, theta, m, s,
+                    state_stride, eta, mu, eps, mode, kappa, precommit_snapshot, nullptr, 0,
+                    nullptr, pi_record);
+}
+
+int oracle_gem_run_pi_f64(int64_t P, int n, int T, const int32_t* order, const int32_t* tau,
+                          const double* grads, int64_t grad_stride, const int32_t* grad_index,
+                          double* theta, double* m, double* s, int64_t state_stride,
+                          double eta, double mu, double eps, int mode, double kappa,
+                          int precommit_snapshot, double* pi_record) {
+  return run<double>(P, n, T, order, tau, grads, grad_stride, grad_index, theta, m, s,
+                     state_stride, eta, mu, eps, mode, kappa, precommit_snapshot, nullptr, 0,
+                     nullptr, pi_record);
 }
 
 }  // extern "C"

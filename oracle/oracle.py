@@ -28,6 +28,10 @@ def lib():
             fn = getattr(_lib, name)
             fn.argtypes = run_args
             fn.restype = C.c_int
+        for name in ("oracle_gem_run_pi_f32", "oracle_gem_run_pi_f64"):
+            fn = getattr(_lib, name)
+            fn.argtypes = run_args[:17] + [p]
+            fn.restype = C.c_int
         _lib.oracle_splitmix64_raw.argtypes = [C.c_uint64, C.c_uint64]
         _lib.oracle_splitmix64_raw.restype = C.c_uint64
         _lib.oracle_splitmix64_draw.argtypes = [C.c_uint64, C.c_uint64, C.c_uint64]
@@ -59,12 +63,16 @@ def _need(a, dtype, name):
 
 
 def gem_run(theta, m, s, grads, order, *, eta, mu, eps, grad_index=None, tau=None,
-            mode=MODE_GEM, kappa=1.0, precommit_snapshot=False, record_cols=None):
+            mode=MODE_GEM, kappa=1.0, precommit_snapshot=False, record_cols=None,
+            record_pi=False):
     """Apply len(order) commits in place (fp32 or fp64 state, chosen by theta's dtype).
 
     theta [P]; m, s [n, P]; grads [R, P] (row grad_index[t], or row t); returns the
-    [T, len(record_cols)] trajectory of theta at record_cols when asked for.
+    [T, len(record_cols)] trajectory of theta at record_cols when asked for, or with
+    record_pi the [T, P] scaling factors pi that the commits applied.
     """
+    if record_pi and record_cols is not None:
+        raise ValueError("record_pi and record_cols are separate runs")
     dt = theta.dtype
     if dt not in (np.float32, np.float64):
         raise TypeError("theta must be float32 or float64")
@@ -88,12 +96,42 @@ def gem_run(theta, m, s, grads, order, *, eta, mu, eps, grad_index=None, tau=Non
         rc_cols = np.ascontiguousarray(record_cols, dtype=np.int64)
         nrec = rc_cols.shape[0]
         rec = np.empty((T, nrec), dtype=dt)
+    if record_pi:
+        fn = lib().oracle_gem_run_pi_f32 if dt == np.float32 else lib().oracle_gem_run_pi_f64
+        pi = np.empty((T, P), dtype=dt)
+        rc = fn(P, n, T, _ptr(order), _ptr(tau_a), _ptr(grads), P, _ptr(gi), _ptr(theta), _ptr(m),
+                _ptr(s), P, eta, mu, eps, mode, kappa, int(precommit_snapshot), _ptr(pi))
+        if rc:
+            raise ValueError(f"oracle_gem_run_pi failed ({rc})")
+        return pi
     rc = fn(P, n, T, _ptr(order), _ptr(tau_a), _ptr(grads), P, _ptr(gi), _ptr(theta), _ptr(m),
             _ptr(s), P, eta, mu, eps, mode, kappa, int(precommit_snapshot), _ptr(rc_cols), nrec,
             _ptr(rec))
     if rc:
         raise ValueError(f"oracle_gem_run failed ({rc})")
     return rec
+
+
+def pi_median(pi, seg):
+    """Per-segment lower and upper medians of the scaling factors of one commit (the median
+    per-parameter pi of the experiments section, per tensor when the segments are the
+    tensors of the flat layout).
+
+    pi [P]; seg [nseg + 1] increasing offsets into pi.  Segment i is pi[seg[i]:seg[i+1]]
+    with N elements, sorted ascending; its lower median is element (N - 1) // 2 and its
+    upper median element N // 2 (equal for odd N; numpy's median is their mean).  Empty
+    segments give NaN.  Returns two float arrays [nseg] in pi's dtype.
+    """
+    seg = np.asarray(seg, dtype=np.int64)
+    lo = np.full(len(seg) - 1, np.nan, dtype=pi.dtype)
+    hi = np.full(len(seg) - 1, np.nan, dtype=pi.dtype)
+    for i in range(len(seg) - 1):
+        x = np.sort(pi[seg[i]:seg[i + 1]])
+        N = x.shape[0]
+        if N:
+            lo[i] = x[(N - 1) // 2]
+            hi[i] = x[N // 2]
+    return lo, hi
 
 
 def splitmix64_raw(state: int, counter: int) -> int:
