@@ -38,6 +38,10 @@ K_BATCH = 100
 POOL_ROWS = 100
 SEED = 5
 ETA, MU, EPS = 0.01, 0.9, 1e-8
+# the other commit rules (gem_mode values of include/gem.h) and kappa; bytes per parameter
+# and commit moved by each rule (theta adds 8 per batch for all)
+RULES = [("downpour", 1, 1.0), ("adaptive", 2, 1.0), ("kappa_sqrt_2", 3, 2.0), ("kappa_linear_2", 4, 2.0)]
+RULE_BYTES = {0: 20, 1: 8, 2: 8, 3: 20, 4: 20}
 BYTES_PER_BATCH = P_FULL * (20 * K_BATCH + 8)
 FALLBACK_HBM_GBS = 6800.0
 
@@ -322,6 +326,56 @@ def run_gem(args, world, rank, local, pg):
         total_ms = max_over_ranks(pg, total_ms)
         barrier(pg)
 
+        # the other commit rules on the same workload, each with its own algorithmic bytes
+        rules = None
+        if not args.no_rules:
+            rules = {}
+            rule_steps = max(3, min(args.steps, 10))
+            for name, mode, kappa in RULES:
+                G.set_mode(mode, kappa)
+                G.commit_batch(*batch(0))
+                ms = time_batches(G, [batch(i) for i in range(rule_steps)], stream)
+                bpb = P_FULL * (RULE_BYTES[mode] * K_BATCH + 8)
+                rules[name] = {"GB_per_s": round(bpb / (ms * 1e-3) / 1e9, 1),
+                               "commits_per_s": round(K_BATCH / (ms * 1e-3), 1),
+                               "ms_per_batch": round(ms, 4),
+                               "bytes_per_param_and_commit": RULE_BYTES[mode]}
+            G.set_mode(gem.GEM_MODE_GEM)
+
+        # scaling-factor statistics: every commit of a batch records its factors, then the
+        # exact median of each commit's P factors
+        pi_stats = None
+        if not args.no_rules:
+            pi_rows = torch.empty((K_BATCH, P_FULL), device="cuda")
+            rows = [pi_rows[k] for k in range(K_BATCH)]
+            lo = torch.empty((K_BATCH, 1), device="cuda")
+            hi = torch.empty((K_BATCH, 1), device="cuda")
+            G.commit_batch_pi(*batch(0), rows)
+            G.pi_median(rows, [0, P_FULL], lo, hi)
+            reps = 3
+            ev = [torch.cuda.Event(enable_timing=True) for _ in range(3 * reps)]
+            stream.synchronize()
+            for r in range(reps):
+                ev[3 * r].record(stream)
+                G.commit_batch_pi(*batch(r + 1), rows)
+                ev[3 * r + 1].record(stream)
+                G.pi_median(rows, [0, P_FULL], lo, hi)
+                ev[3 * r + 2].record(stream)
+            ev[-1].synchronize()
+            commit_ms = sum(ev[3 * r].elapsed_time(ev[3 * r + 1]) for r in range(reps)) / reps
+            select_ms = sum(ev[3 * r + 1].elapsed_time(ev[3 * r + 2]) for r in range(reps)) / reps
+            sel_bytes = 12 * K_BATCH * P_FULL
+            pi_stats = {
+                "commit_with_pi_ms": round(commit_ms, 4),
+                "commit_with_pi_GB_per_s": round(P_FULL * (24 * K_BATCH + 8) / (commit_ms * 1e-3) / 1e9, 1),
+                "median_ms": round(select_ms, 4),
+                "median_GB_per_s": round(sel_bytes / (select_ms * 1e-3) / 1e9, 1),
+                "median_bytes": "12 per factor (three radix passes of 4 bytes)",
+                "commits_per_s_with_median": round(K_BATCH / ((commit_ms + select_ms) * 1e-3), 1),
+                "median_pi_last_batch": float(lo[-1, 0]),
+            }
+            del pi_rows, rows
+
         # end to end through the public API: gradients in pinned host memory, read by the
         # commit kernel in place over the host link every step, and theta read back to the
         # host after each step
@@ -355,6 +409,7 @@ def run_gem(args, world, rank, local, pg):
     del pool
     torch.cuda.empty_cache()
 
+    flat = None if args.no_flat else run_flat_commits(seed_offset=rank)
     mlp = None if args.no_mlp else run_mlp_workloads(args, seed_offset=rank)
 
     if rank != 0:
@@ -384,6 +439,9 @@ def run_gem(args, world, rank, local, pg):
                      "kernel": "commit_batch_kernel", "algorithmic_bytes_per_launch": BYTES_PER_BATCH,
                      "launch_ms_min": round(min(per_step_ms), 4), "launch_ms_max": round(max(per_step_ms), 4)},
         "gpu_launches": int(launches),
+        "commit_rules": rules,
+        "pi_statistics": pi_stats,
+        "flat_single_commits": flat,
         "async_mlp": mlp,
         "clocks": clocks.summary(),
         "e2e": e2e,
@@ -391,6 +449,61 @@ def run_gem(args, world, rank, local, pg):
     if not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline()
     print(json.dumps(line), flush=True)
+
+
+def time_batches(G, batches, stream) -> float:
+    """Mean CUDA-event time (ms) of one gem_commit_batch call over `batches`."""
+    import torch
+    stream.synchronize()
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    t0.record(stream)
+    for order, grads in batches:
+        G.commit_batch(order, grads)
+    t1.record(stream)
+    t1.synchronize()
+    return t0.elapsed_time(t1) / len(batches)
+
+
+def run_flat_commits(seed_offset: int = 0) -> dict:
+    """Flat P = 1.2M, n = 20, 5,000 uniform-tick commits with log-uniform gradient scales
+    (sigma_j in [1e-4, 1e-1]); the gradients cycle through a device pool of 200.  The state
+    (about 0.2 GB) is L2-scale, so the GB/s are effective, not DRAM, rates."""
+    import numpy as np
+    import torch
+
+    from paper_1805_08469_gb300 import gem, sim, synth, synth_gpu
+    P, n, T, pool_rows, seed = 1_200_000, 20, 5000, 200, 2 + seed_offset
+    stream = torch.cuda.Stream()
+    order, _ = sim.gem_schedule_uniform(seed, n, T)
+    out = {}
+    with torch.cuda.stream(stream):
+        sigma = torch.from_numpy(synth.sigma_loguniform(seed, np.arange(P))).cuda()
+        pool = torch.empty((pool_rows, P), device="cuda")
+        for r in range(pool_rows):
+            synth_gpu.grad_loguniform(seed, r, sigma, pool[r], stream=stream)
+        with gem.Gem(P, n, ETA, MU, EPS, stream=stream) as G:
+            G.set_theta(synth_gpu.theta0_flat(seed, torch.empty(P, device="cuda"), stream=stream))
+            grads = [pool[t % pool_rows] for t in range(T)]
+            G.commit_batch([int(w) for w in order[:200]], grads[:200])      # warm-up
+            ms = time_batches(G, [([int(w) for w in order], grads)], stream)
+            out["batched"] = {"commits_per_s": round(T / (ms * 1e-3), 1),
+                              "effective_GB_per_s": round(P * (20 * T + 8 * ((T + 199) // 200)) / (ms * 1e-3) / 1e9, 1),
+                              "note": "gem_commit_batch of all 5,000 commits (launches of 200)"}
+            G.sync()
+            t0 = torch.cuda.Event(enable_timing=True)
+            t1 = torch.cuda.Event(enable_timing=True)
+            t0.record(stream)
+            for t in range(T):
+                G.commit(int(order[t]), grads[t])
+            t1.record(stream)
+            t1.synchronize()
+            ms = t0.elapsed_time(t1)
+            out["single"] = {"commits_per_s": round(T / (ms * 1e-3), 1),
+                             "effective_GB_per_s": round(P * 28 * T / (ms * 1e-3) / 1e9, 1),
+                             "note": "one gem_commit call per commit (host-issue bound)"}
+    out["workload"] = f"flat P={P} n={n}, {T} uniform-tick commits, log-uniform sigma, pool of {pool_rows}"
+    return out
 
 
 MLP_WORKLOADS = [
@@ -467,6 +580,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-mlp", action="store_true")
+    ap.add_argument("--no-rules", action="store_true", help="skip timing the other commit rules")
+    ap.add_argument("--no-flat", action="store_true", help="skip the flat P=1.2M single-commit run")
     ap.add_argument("--only", choices=["all", "commit", "mlp"], default="all",
                     help="profiling aid: run only the commit batches or only the async MLP runs")
     ap.add_argument("--mlp-workload", default="",
@@ -496,6 +611,8 @@ def main():
         else:
             if args.only == "commit":
                 args.no_mlp = True
+                args.no_flat = True
+                args.no_rules = True
             run_gem(args, world, rank, local, pg)
     if pg is not None:
         pg.destroy_process_group()

@@ -176,6 +176,31 @@ int gem_get_clock(const gem_t* h, int64_t* clock, int64_t* last);
  * for all).  Returns GEM_EINVAL and changes nothing if a value is out of range. */
 int gem_set_clock(gem_t* h, int64_t clock, const int64_t* last);
 
+/* Scaling-factor statistics.  The experiments section follows the median per-parameter
+ * value of pi over time (and, in the appendix, per tensor) to show how GEM rescales the
+ * commits as workers are added.  These two calls record pi and take exact medians.
+ *
+ * gem_commit_batch_pi: gem_commit_batch, and when pi is not NULL and pi[k] is not NULL,
+ * the scaling factor that commit k applied to each coordinate is written to pi[k] [P]
+ * (device memory, 16-byte aligned): the clamped pi of the GEM and kappa rules, 1 for
+ * DOWNPOUR, 1 / (tau + 1) for adaptive staleness.  The commits themselves are unchanged,
+ * bit for bit.  pi and its entries are host data read before the call returns. */
+int gem_commit_batch_pi(gem_t* h, const int* order, const float* const* grads, int K,
+                        float* const* pi);
+
+/* Exact medians of K rows of P floats (typically recorded by gem_commit_batch_pi), per
+ * segment: segment i of row k is pi[k][seg[i] .. seg[i+1]).  With its N elements sorted
+ * ascending, lo[k * nseg + i] receives element (N - 1) / 2 and hi[k * nseg + i] element
+ * N / 2 (the same for odd N; their mean is the usual median); NaN for an empty segment.
+ * pi is a host array of K device pointers (4-byte aligned); seg is a host array of nseg + 1
+ * offsets with 0 <= seg[0] <= ... <= seg[nseg] <= P, 1 <= nseg <= 64; lo and hi are device
+ * arrays of K * nseg floats.  Stream-ordered: three passes over the rows (radix selection,
+ * 11 + 11 + 10 bits of an order-preserving key).  The first call, and any call with more
+ * rows or segments than before (up to 200 rows per pass), allocates the select scratch:
+ * 16 KB per row and segment. */
+int gem_pi_median(gem_t* h, const float* const* pi, int K, const int64_t* seg, int nseg,
+                  float* lo, float* hi);
+
 /* Number of kernels this handle has launched since it was created. */
 uint64_t gem_launch_count(const gem_t* h);
 

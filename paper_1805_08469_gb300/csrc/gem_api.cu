@@ -79,7 +79,8 @@ int ensure_staging(gem_t* h) {
 
 namespace gem {
 
-cudaError_t commit_ordered(gem_ctx* h, const int* order, const float* const* grads, int K) {
+cudaError_t commit_ordered(gem_ctx* h, const int* order, const float* const* grads, int K,
+                           float* const* pi_out) {
   BatchArgs a;
   a.theta = h->theta;
   a.m = h->m;
@@ -110,6 +111,11 @@ cudaError_t commit_ordered(gem_ctx* h, const int* order, const float* const* gra
   for (int k0 = 0; k0 < K; k0 += kMaxBatchPerLaunch) {
     const int kc = (K - k0) < kMaxBatchPerLaunch ? (K - k0) : kMaxBatchPerLaunch;
     a.K = kc;
+    a.record_pi = 0;
+    for (int k = 0; k < kc; ++k) {
+      a.pi_out[k] = pi_out ? pi_out[k0 + k] : nullptr;
+      if (a.pi_out[k]) a.record_pi = 1;
+    }
     for (int k = 0; k < kc; ++k) {
       const int w = order[k0 + k];
       a.worker[k] = w;
@@ -208,6 +214,7 @@ void gem_destroy(gem_t* h) {
   }
   if (h->copy_stream) cudaStreamDestroy(h->copy_stream);
   cudaFree(h->stage);
+  cudaFree(h->select_scratch);
   cudaFree(h->theta);
   cudaFree(h->m);
   cudaFree(h->s);
@@ -336,6 +343,46 @@ int gem_commit_batch(gem_t* h, const int* order, const float* const* grads, int 
   DeviceScope scope(h->device);
   if (!scope.ok()) return GEM_ECUDA;
   return launch_commits(h, order, grads, K);
+}
+
+int gem_commit_batch_pi(gem_t* h, const int* order, const float* const* grads, int K,
+                        float* const* pi) {
+  int rc = check_handle(h);
+  if (rc) return rc;
+  rc = check_batch(h, order, grads, K);
+  if (rc) return rc;
+  if (pi)
+    for (int k = 0; k < K; ++k)
+      if (pi[k] && !aligned16(pi[k])) return GEM_EINVAL;
+  if (K == 0) return GEM_OK;
+  DeviceScope scope(h->device);
+  if (!scope.ok()) return GEM_ECUDA;
+  return cuda_status(h, gem::commit_ordered(h, order, grads, K, pi));
+}
+
+int gem_pi_median(gem_t* h, const float* const* pi, int K, const int64_t* seg, int nseg,
+                  float* lo, float* hi) {
+  int rc = check_handle(h);
+  if (rc) return rc;
+  if (K < 0 || nseg < 1 || nseg > gem::kMaxPiSegments || !seg) return GEM_EINVAL;
+  if (seg[0] < 0 || seg[nseg] > int64_t(h->P)) return GEM_EINVAL;
+  for (int i = 0; i < nseg; ++i)
+    if (seg[i + 1] < seg[i] || seg[i + 1] - seg[i] > int64_t(UINT32_MAX)) return GEM_EINVAL;
+  if (K == 0) return GEM_OK;
+  if (!pi || !lo || !hi) return GEM_EINVAL;
+  const uintptr_t align4 = 3u;
+  if ((reinterpret_cast<uintptr_t>(lo) & align4) || (reinterpret_cast<uintptr_t>(hi) & align4))
+    return GEM_EINVAL;
+  for (int k = 0; k < K; ++k)
+    if (!pi[k] || (reinterpret_cast<uintptr_t>(pi[k]) & align4)) return GEM_EINVAL;
+  DeviceScope scope(h->device);
+  if (!scope.ok()) return GEM_ECUDA;
+  const cudaError_t e = gem::pi_median_ordered(h, pi, K, seg, nseg, lo, hi);
+  if (e == cudaErrorMemoryAllocation) {
+    cudaGetLastError();
+    return GEM_ENOMEM;
+  }
+  return cuda_status(h, e);
 }
 
 int gem_commit_batch_host(gem_t* h, const int* order, const float* const* grads, int K) {

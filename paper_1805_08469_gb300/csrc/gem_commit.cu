@@ -46,8 +46,8 @@ constexpr int kThreads = GEM_COMMIT_THREADS;
 // RULE kRuleGem takes |m_w| as the root of twice the proxy energy (Eq. proxy_estimate);
 // kRuleScaled multiplies it by `scale` first (sqrt(kappa) or kappa, App. B).
 template <int RULE>
-__device__ __forceinline__ void commit_coord(float& theta, float& m, float& s, float g,
-                                             float eta, float mu, float eps, float scale) {
+__device__ __forceinline__ float commit_coord(float& theta, float& m, float& s, float g,
+                                              float eta, float mu, float eps, float scale) {
   const float dtheta = -__fmul_rn(eta, g);                       // -eta grad L(s)
   const float m_new = __fadd_rn(__fmul_rn(mu, m), dtheta);       // m <- mu m + dtheta
   const float drift = fabsf(__fsub_rn(theta, s));                // |theta - s|
@@ -58,6 +58,7 @@ __device__ __forceinline__ void commit_coord(float& theta, float& m, float& s, f
   theta = __fadd_rn(theta, __fmul_rn(pi, dtheta));               // theta + pi dtheta
   m = m_new;
   s = theta;                                                     // s <- theta
+  return pi;
 }
 
 // A commit with a given scaling factor (kRuleFixed): theta + pi dtheta, s <- theta; the
@@ -86,12 +87,14 @@ __device__ __forceinline__ void store_state(float4* p, float4 v) {
 }
 
 template <int RULE>
-__device__ __forceinline__ void commit_vec(float4& th, float4& m, float4& s, const float4 g,
-                                           float eta, float mu, float eps, float scale) {
-  commit_coord<RULE>(th.x, m.x, s.x, g.x, eta, mu, eps, scale);
-  commit_coord<RULE>(th.y, m.y, s.y, g.y, eta, mu, eps, scale);
-  commit_coord<RULE>(th.z, m.z, s.z, g.z, eta, mu, eps, scale);
-  commit_coord<RULE>(th.w, m.w, s.w, g.w, eta, mu, eps, scale);
+__device__ __forceinline__ float4 commit_vec(float4& th, float4& m, float4& s, const float4 g,
+                                             float eta, float mu, float eps, float scale) {
+  float4 pi;
+  pi.x = commit_coord<RULE>(th.x, m.x, s.x, g.x, eta, mu, eps, scale);
+  pi.y = commit_coord<RULE>(th.y, m.y, s.y, g.y, eta, mu, eps, scale);
+  pi.z = commit_coord<RULE>(th.z, m.z, s.z, g.z, eta, mu, eps, scale);
+  pi.w = commit_coord<RULE>(th.w, m.w, s.w, g.w, eta, mu, eps, scale);
+  return pi;
 }
 
 __device__ __forceinline__ void commit_vec_fixed(float4& th, float4& s, const float4 g, float eta,
@@ -105,8 +108,12 @@ __device__ __forceinline__ void commit_vec_fixed(float4& th, float4& s, const fl
 // L independent 16-byte lanes per thread, strided by the grid so that each warp
 // touches 512 contiguous bytes per lane and array.  The fixed-factor rules read only the
 // gradient and write only s_w (12 bytes less per coordinate and commit).
-template <int L, int RULE>
-__global__ void __launch_bounds__(kThreads, GEM_COMMIT_MIN_BLOCKS)
+// The scaled rule asks for two resident blocks per SM: left free, the compiler fits it in
+// 40 registers for three blocks and spills, which costs about 4% of its bandwidth.
+// REC: the commits whose pi_out[k] is set also store their scaling factors there (4 more
+// bytes per coordinate).
+template <int L, int RULE, bool REC>
+__global__ void __launch_bounds__(kThreads, RULE == kRuleScaled ? 2 : GEM_COMMIT_MIN_BLOCKS)
 commit_batch_kernel(const __grid_constant__ BatchArgs a) {
   const size_t nvec = a.P >> 2;
   const size_t nthreads = size_t(gridDim.x) * kThreads;
@@ -141,13 +148,16 @@ commit_batch_kernel(const __grid_constant__ BatchArgs a) {
       for (int l = 0; l < L; ++l) {
         const size_t i = base + size_t(l) * nthreads;
         if (i < nvec) {
+          float4 pi;
           if (RULE == kRuleFixed) {
             commit_vec_fixed(th[l], s[l], g[l], a.eta, a.pi[k]);
+            pi = make_float4(a.pi[k], a.pi[k], a.pi[k], a.pi[k]);
           } else {
-            commit_vec<RULE>(th[l], m[l], s[l], g[l], a.eta, a.mu, a.eps, a.energy_scale);
+            pi = commit_vec<RULE>(th[l], m[l], s[l], g[l], a.eta, a.mu, a.eps, a.energy_scale);
             store_state(m4 + i, m[l]);
           }
           store_state(s4 + i, s[l]);
+          if (REC && a.pi_out[k]) reinterpret_cast<float4*>(a.pi_out[k])[i] = pi;
         }
       }
     }
@@ -166,16 +176,18 @@ commit_batch_kernel(const __grid_constant__ BatchArgs a) {
     float th = a.theta[j];
     for (int k = 0; k < a.K; ++k) {
       const size_t row = size_t(a.worker[k]) * a.stride;
-      float s;
+      float s, pi;
       if (RULE == kRuleFixed) {
         commit_coord_fixed(th, s, a.grad[k][j], a.eta, a.pi[k]);
+        pi = a.pi[k];
       } else {
         float m = a.m[row + j];
         s = a.s[row + j];
-        commit_coord<RULE>(th, m, s, a.grad[k][j], a.eta, a.mu, a.eps, a.energy_scale);
+        pi = commit_coord<RULE>(th, m, s, a.grad[k][j], a.eta, a.mu, a.eps, a.energy_scale);
         a.m[row + j] = m;
       }
       a.s[row + j] = s;
+      if (REC && a.pi_out[k]) a.pi_out[k][j] = pi;
     }
     a.theta[j] = th;
   }
@@ -183,12 +195,12 @@ commit_batch_kernel(const __grid_constant__ BatchArgs a) {
 
 constexpr int kLanes = GEM_COMMIT_LANES;
 
-template <int RULE>
+template <int RULE, bool REC>
 cudaError_t launch_rule(const BatchArgs& a, int sm_count, cudaStream_t stream) {
   static int blocks_per_sm = 0;
   if (blocks_per_sm == 0) {
     cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(
-        &blocks_per_sm, commit_batch_kernel<kLanes, RULE>, kThreads, 0);
+        &blocks_per_sm, commit_batch_kernel<kLanes, RULE, REC>, kThreads, 0);
     if (e != cudaSuccess) return e;
     if (blocks_per_sm < 1) blocks_per_sm = 1;
   }
@@ -203,17 +215,25 @@ cudaError_t launch_rule(const BatchArgs& a, int sm_count, cudaStream_t stream) {
     grid = (nvec + rounds * per_block - 1) / (rounds * per_block);
   }
   if (grid < 1) grid = 1;
-  commit_batch_kernel<kLanes, RULE><<<unsigned(grid), kThreads, 0, stream>>>(a);
+  commit_batch_kernel<kLanes, RULE, REC><<<unsigned(grid), kThreads, 0, stream>>>(a);
   return cudaGetLastError();
 }
 
 }  // namespace
 
 cudaError_t launch_commit_batch(const BatchArgs& a, int sm_count, cudaStream_t stream) {
+  if (a.record_pi) {
+    switch (a.rule) {
+      case kRuleGem: return launch_rule<kRuleGem, true>(a, sm_count, stream);
+      case kRuleScaled: return launch_rule<kRuleScaled, true>(a, sm_count, stream);
+      case kRuleFixed: return launch_rule<kRuleFixed, true>(a, sm_count, stream);
+      default: return cudaErrorInvalidValue;
+    }
+  }
   switch (a.rule) {
-    case kRuleGem: return launch_rule<kRuleGem>(a, sm_count, stream);
-    case kRuleScaled: return launch_rule<kRuleScaled>(a, sm_count, stream);
-    case kRuleFixed: return launch_rule<kRuleFixed>(a, sm_count, stream);
+    case kRuleGem: return launch_rule<kRuleGem, false>(a, sm_count, stream);
+    case kRuleScaled: return launch_rule<kRuleScaled, false>(a, sm_count, stream);
+    case kRuleFixed: return launch_rule<kRuleFixed, false>(a, sm_count, stream);
     default: return cudaErrorInvalidValue;
   }
 }

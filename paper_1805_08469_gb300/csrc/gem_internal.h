@@ -42,6 +42,8 @@ struct BatchArgs {
   const float* grad[kMaxBatchPerLaunch];   // gradient of commit k, P floats
   int worker[kMaxBatchPerLaunch];          // worker of commit k
   float pi[kMaxBatchPerLaunch];            // kRuleFixed: scaling factor of commit k
+  int record_pi;                           // 1: pi_out[k] (when not null) receives pi
+  float* pi_out[kMaxBatchPerLaunch];       // scaling factors of commit k, P floats, or null
 };
 
 // Launch the fused commit kernel for a.K commits on `stream`.
@@ -67,6 +69,9 @@ struct gem_ctx {
   float kappa = 1.f;
   int64_t clock = 0;           // commits issued since gem_set_theta
   std::vector<int64_t> last;   // [n] clock value of worker w's last commit, -1 before its first
+  // scratch of the pi median select: histograms and per-problem state, grown on demand
+  void* select_scratch = nullptr;
+  size_t select_bytes = 0;
   // staging of host gradients (gem_commit_batch_host), allocated on first use
   float* stage = nullptr;
   cudaStream_t copy_stream = nullptr;
@@ -79,6 +84,18 @@ namespace gem {
 // Launch commits [0, K) of the handle in order, in chunks of kMaxBatchPerLaunch, with the
 // handle's commit rule; advances the commit clock and counts the launches.  The arguments
 // must have been checked.
-cudaError_t commit_ordered(gem_ctx* h, const int* order, const float* const* grads, int K);
+cudaError_t commit_ordered(gem_ctx* h, const int* order, const float* const* grads, int K,
+                           float* const* pi_out = nullptr);
+
+// Segments per median call and commits per select launch.
+constexpr int kMaxPiSegments = 64;
+constexpr int kMaxPiBatch = 200;
+
+// Exact lower and upper medians of each segment of each of K scaling-factor rows
+// (segments seg[0..nseg] shared by all rows), written to lo/hi [K][nseg] on the handle's
+// stream.  Uses the handle's select scratch (grown on demand).  Arguments checked by the
+// caller.
+cudaError_t pi_median_ordered(gem_ctx* h, const float* const* pi, int K, const int64_t* seg,
+                              int nseg, float* lo, float* hi);
 
 }  // namespace gem

@@ -1,0 +1,241 @@
+// Exact medians of the scaling factors pi, per commit and per segment (the statistic of the
+// experiments section: the median per-parameter value of pi, over time, and per tensor in
+// the ImageNet figures of the appendix).
+//
+// Selection by radix on an order-preserving 32-bit key of each float, most significant
+// digit first, in three passes of 11, 11 and 10 bits.  Every problem (commit k, segment s)
+// has two targets, the lower and upper middle elements (ranks (N - 1) / 2 and N / 2 of the
+// N elements sorted ascending).  A target is a (prefix, mask, rank) triple: the key bits
+// fixed so far and the rank of the target among the elements that share them.
+//   - select_hist_kernel: blocks of 16,384 elements of one segment count, in shared memory,
+//     the next digit of every element that matches a target's prefix, and add their
+//     counts to the problem's histogram in global memory.  Counts are aggregated per warp
+//     (one shared-memory atomic per distinct digit), because clamped factors put many
+//     equal keys (pi = 0) into one bin.  While both targets share their prefix, which is
+//     always true in the first pass, one histogram serves both.
+//   - select_pick_kernel: one block per problem scans the histogram, finds the bin that
+//     holds each target's rank, extends the prefix and reduces the rank, then clears the
+//     histogram for the next pass.
+// After the third pass the prefix is the target's key, which maps back to its float.
+// Each pass reads the factors once (4 bytes per element), so 12 bytes per element.
+#include <cmath>
+
+#include "gem_internal.h"
+
+namespace gem {
+namespace {
+
+constexpr int kThreads = 256;
+constexpr int kBins = 2048;                 // 11-bit digits (the last pass uses 1024)
+constexpr int kUnroll = 8;                  // independent loads per thread and step
+constexpr int kChunk = kThreads * kUnroll * 8;   // elements per histogram block
+constexpr int kPasses = 3;
+
+__host__ __device__ constexpr int digit_shift(int pass) { return pass == 0 ? 21 : (pass == 1 ? 10 : 0); }
+__host__ __device__ constexpr int digit_bits(int pass) { return pass == 2 ? 10 : 11; }
+
+struct SelectArgs {
+  const float* pi[kMaxPiBatch];             // row k: P floats
+  long long seg[kMaxPiSegments + 1];        // segment offsets, shared by all rows
+  int block_start[kMaxPiSegments + 1];      // first histogram block of each segment
+  int K, nseg, pass;
+  unsigned* hist;                           // [K][nseg][2][kBins]
+  unsigned* state;                          // [K][nseg][2][3]: prefix, mask, rank
+  float* lo;                                // [K][nseg]
+  float* hi;                                // [K][nseg]
+};
+
+// Unsigned order of the keys equals the order of the floats (-0 below +0, NaNs outermost).
+__device__ __forceinline__ unsigned order_key(float x) {
+  const unsigned u = __float_as_uint(x);
+  return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+
+__device__ __forceinline__ float key_value(unsigned k) {
+  return __uint_as_float((k & 0x80000000u) ? (k & 0x7fffffffu) : ~k);
+}
+
+__global__ void select_init_kernel(const __grid_constant__ SelectArgs a) {
+  const int q = blockIdx.x * blockDim.x + threadIdx.x;     // problem k * nseg + s
+  if (q >= a.K * a.nseg) return;
+  const int s = q % a.nseg;
+  const long long N = a.seg[s + 1] - a.seg[s];
+  unsigned* st = a.state + size_t(q) * 6;
+  st[0] = 0u;
+  st[1] = 0u;
+  st[2] = N > 0 ? unsigned((N - 1) / 2) : 0u;
+  st[3] = 0u;
+  st[4] = 0u;
+  st[5] = unsigned(N / 2);
+}
+
+// Adds one element's digit to a shared histogram when its key matches the prefix; every
+// lane of the warp must call it (the match is warp-wide).
+__device__ __forceinline__ void count_digit(unsigned* h, bool valid, unsigned key, unsigned prefix,
+                                            unsigned mask, unsigned digit, int lane) {
+  const unsigned bin = (valid && (key & mask) == prefix) ? digit : 0xffffffffu;
+  const unsigned peers = __match_any_sync(0xffffffffu, bin);
+  if (bin != 0xffffffffu && lane == __ffs(peers) - 1) atomicAdd(h + bin, unsigned(__popc(peers)));
+}
+
+__global__ void __launch_bounds__(kThreads) select_hist_kernel(const __grid_constant__ SelectArgs a) {
+  __shared__ unsigned h[2 * kBins];
+  const int b = blockIdx.x, k = blockIdx.y;
+  int s = 0;
+  while (b >= a.block_start[s + 1]) ++s;
+  const int q = k * a.nseg + s;
+  const unsigned* st = a.state + size_t(q) * 6;
+  const unsigned p0 = st[0], m0 = st[1], p1 = st[3], m1 = st[4];
+  const bool two = p0 != p1 || m0 != m1;
+  for (int i = threadIdx.x; i < 2 * kBins; i += kThreads) h[i] = 0u;
+  __syncthreads();
+
+  const int shift = digit_shift(a.pass);
+  const unsigned dmask = (1u << digit_bits(a.pass)) - 1u;
+  const long long beg = a.seg[s] + (long long)(b - a.block_start[s]) * kChunk;
+  const long long end = beg + kChunk < a.seg[s + 1] ? beg + kChunk : a.seg[s + 1];
+  const float* x = a.pi[k];
+  const int lane = threadIdx.x & 31;
+  // the loop bounds are uniform across the block, so whole warps reach count_digit
+  for (long long base = beg; base < end; base += kThreads * kUnroll) {
+    unsigned key[kUnroll];
+#pragma unroll
+    for (int u = 0; u < kUnroll; ++u) {
+      const long long i = base + u * kThreads + threadIdx.x;
+      key[u] = i < end ? order_key(x[i]) : 0u;
+    }
+#pragma unroll
+    for (int u = 0; u < kUnroll; ++u) {
+      const bool valid = base + u * kThreads + threadIdx.x < end;
+      const unsigned d = (key[u] >> shift) & dmask;
+      count_digit(h, valid, key[u], p0, m0, d, lane);
+      if (two) count_digit(h + kBins, valid, key[u], p1, m1, d, lane);
+    }
+  }
+  __syncthreads();
+  unsigned* g = a.hist + size_t(q) * 2 * kBins;
+  const int used = two ? 2 * kBins : kBins;
+  for (int i = threadIdx.x; i < used; i += kThreads) {
+    const unsigned c = h[i];
+    if (c) atomicAdd(g + i, c);
+  }
+}
+
+__global__ void __launch_bounds__(kThreads) select_pick_kernel(const __grid_constant__ SelectArgs a) {
+  constexpr int kPer = kBins / kThreads;     // bins per thread (8)
+  __shared__ unsigned wsum[kThreads / 32];
+  __shared__ unsigned sst[6];
+  const int q = blockIdx.x;
+  const int s = q % a.nseg;
+  const long long N = a.seg[s + 1] - a.seg[s];
+  unsigned* st = a.state + size_t(q) * 6;
+  unsigned* g = a.hist + size_t(q) * 2 * kBins;
+  if (threadIdx.x < 6) sst[threadIdx.x] = st[threadIdx.x];
+  __syncthreads();
+  const bool two = sst[0] != sst[3] || sst[1] != sst[4];
+  const int shift = digit_shift(a.pass);
+  const unsigned nb = 1u << digit_bits(a.pass);
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+
+  for (int t = 0; t < 2; ++t) {
+    const unsigned* hh = g + (two ? t : 0) * kBins;
+    unsigned local[kPer];
+    unsigned sum = 0;
+#pragma unroll
+    for (int j = 0; j < kPer; ++j) {
+      local[j] = hh[threadIdx.x * kPer + j];
+      sum += local[j];
+    }
+    unsigned incl = sum;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+      const unsigned v = __shfl_up_sync(0xffffffffu, incl, off);
+      if (lane >= off) incl += v;
+    }
+    if (lane == 31) wsum[warp] = incl;
+    __syncthreads();
+    unsigned before = 0;
+    for (int w = 0; w < warp; ++w) before += wsum[w];
+    const unsigned excl = before + incl - sum;
+    const unsigned r = sst[3 * t + 2];
+    if (N > 0 && r >= excl && r - excl < sum) {
+      unsigned c = excl;
+      int d = 0;
+#pragma unroll
+      for (int j = 0; j < kPer; ++j) {
+        if (r - c < local[j]) {
+          d = threadIdx.x * kPer + j;
+          break;
+        }
+        c += local[j];
+      }
+      const unsigned prefix = sst[3 * t] | (unsigned(d) << shift);
+      st[3 * t] = prefix;
+      st[3 * t + 1] = sst[3 * t + 1] | ((nb - 1u) << shift);
+      st[3 * t + 2] = r - c;
+      if (a.pass == kPasses - 1) (t == 0 ? a.lo : a.hi)[q] = key_value(prefix);
+    }
+    __syncthreads();   // wsum is reused by the next target
+  }
+  for (int i = threadIdx.x; i < 2 * kBins; i += kThreads) g[i] = 0u;
+  if (N == 0 && a.pass == kPasses - 1 && threadIdx.x == 0) {
+    a.lo[q] = __int_as_float(0x7fc00000);
+    a.hi[q] = __int_as_float(0x7fc00000);
+  }
+}
+
+}  // namespace
+
+cudaError_t pi_median_ordered(gem_ctx* h, const float* const* pi, int K, const int64_t* seg,
+                              int nseg, float* lo, float* hi) {
+  if (K <= 0) return cudaSuccess;
+  const int kc_max = K < kMaxPiBatch ? K : kMaxPiBatch;
+  const size_t hist_bytes = size_t(kc_max) * nseg * 2 * kBins * sizeof(unsigned);
+  const size_t need = hist_bytes + size_t(kc_max) * nseg * 6 * sizeof(unsigned);
+  if (need > h->select_bytes) {
+    cudaFree(h->select_scratch);   // waits for work still using the old buffer
+    h->select_scratch = nullptr;
+    h->select_bytes = 0;
+    cudaError_t e = cudaMalloc(&h->select_scratch, need);
+    if (e != cudaSuccess) return e;
+    h->select_bytes = need;
+  }
+  SelectArgs a;
+  a.nseg = nseg;
+  a.block_start[0] = 0;
+  for (int s = 0; s <= nseg; ++s) a.seg[s] = seg[s];
+  for (int s = 0; s < nseg; ++s) {
+    const long long N = seg[s + 1] - seg[s];
+    a.block_start[s + 1] = a.block_start[s] + int((N + kChunk - 1) / kChunk);
+  }
+  const int blocks = a.block_start[nseg];
+  a.hist = static_cast<unsigned*>(h->select_scratch);
+  a.state = reinterpret_cast<unsigned*>(static_cast<char*>(h->select_scratch) + hist_bytes);
+  for (int k0 = 0; k0 < K; k0 += kMaxPiBatch) {
+    const int kc = (K - k0) < kMaxPiBatch ? (K - k0) : kMaxPiBatch;
+    a.K = kc;
+    for (int k = 0; k < kc; ++k) a.pi[k] = pi[k0 + k];
+    a.lo = lo + size_t(k0) * nseg;
+    a.hi = hi + size_t(k0) * nseg;
+    a.pass = 0;
+    cudaError_t e = cudaMemsetAsync(a.hist, 0, size_t(kc) * nseg * 2 * kBins * sizeof(unsigned),
+                                    h->stream);
+    if (e != cudaSuccess) return e;
+    select_init_kernel<<<(kc * nseg + 127) / 128, 128, 0, h->stream>>>(a);
+    h->launches += 1;
+    for (int p = 0; p < kPasses; ++p) {
+      a.pass = p;
+      if (blocks > 0) {
+        select_hist_kernel<<<dim3(unsigned(blocks), unsigned(kc)), kThreads, 0, h->stream>>>(a);
+        h->launches += 1;
+      }
+      select_pick_kernel<<<unsigned(kc * nseg), kThreads, 0, h->stream>>>(a);
+      h->launches += 1;
+    }
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
+}
+
+}  // namespace gem

@@ -105,6 +105,27 @@ def gem_commit_batch(h: int, order: Sequence[int], grads: Sequence) -> None:
     check(lib().gem_commit_batch(C.c_void_p(h), o, g, K), "gem_commit_batch")
 
 
+def gem_commit_batch_pi(h: int, order: Sequence[int], grads: Sequence, pi: Sequence) -> None:
+    """gem_commit_batch that also writes each commit's scaling factors to pi[k] (a [P]
+    float32 CUDA tensor, or None for a commit whose factors are not wanted)."""
+    o, g, K = _batch_arrays(order, [_dev_ptr(x, "grads[k]") for x in grads])
+    if len(pi) != K:
+        raise ValueError("order and pi differ in length")
+    pp = (C.c_void_p * max(K, 1))(*[None if x is None else _dev_ptr(x, "pi[k]") for x in pi])
+    check(lib().gem_commit_batch_pi(C.c_void_p(h), o, g, K, pp), "gem_commit_batch_pi")
+
+
+def gem_pi_median(h: int, pi: Sequence, seg: Sequence[int], lo, hi) -> None:
+    """Per-segment lower / upper medians of the rows pi[k] into lo, hi [K, nseg] (float32
+    CUDA tensors); seg holds nseg + 1 offsets.  Stream-ordered."""
+    K = len(pi)
+    rows = (C.c_void_p * max(K, 1))(*[_dev_ptr(x, "pi[k]") for x in pi])
+    sg = (C.c_int64 * len(seg))(*[int(x) for x in seg])
+    check(lib().gem_pi_median(C.c_void_p(h), rows, K, sg, len(seg) - 1,
+                              C.c_void_p(_dev_ptr(lo, "lo")), C.c_void_p(_dev_ptr(hi, "hi"))),
+          "gem_pi_median")
+
+
 def gem_commit_batch_host(h: int, order: Sequence[int], grads: Sequence) -> None:
     ptrs = []
     for x in grads:
@@ -256,6 +277,12 @@ class Gem:
 
     def commit_batch_host(self, order, grads):
         gem_commit_batch_host(self.h, order, grads)
+
+    def commit_batch_pi(self, order, grads, pi):
+        gem_commit_batch_pi(self.h, order, grads, pi)
+
+    def pi_median(self, pi, seg, lo, hi):
+        gem_pi_median(self.h, pi, seg, lo, hi)
 
     def sync(self):
         gem_sync(self.h)
