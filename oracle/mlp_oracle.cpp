@@ -30,6 +30,12 @@ extern "C" int oracle_gem_run_f32(int64_t P, int n, int T, const int32_t* order,
                                   double eta, double mu, double eps, int mode, double kappa,
                                   int precommit_snapshot, const int64_t* record_cols,
                                   int n_record, float* record);
+extern "C" int oracle_gem_run_pi_f32(int64_t P, int n, int T, const int32_t* order,
+                                     const int32_t* tau, const float* grads,
+                                     int64_t grad_stride, const int32_t* grad_index,
+                                     float* theta, float* m, float* s, int64_t state_stride,
+                                     double eta, double mu, double eps, int mode, double kappa,
+                                     int precommit_snapshot, float* pi_record);
 
 namespace {
 
@@ -181,6 +187,14 @@ double oracle_mlp_loss_grad_f64(int L, const int32_t* dims, const double* theta,
 // theta [P], m and s [n][state_stride] fp32 are updated in place.  X [x_rows][dims[0]],
 // labels [x_rows].  After commit t = record_at[r] theta is copied to record[r][0..P).
 // losses[t] (optional) receives the minibatch loss of commit t.
+int oracle_mlp_sim_run_pi(int L, const int32_t* dims, int n, int T, const int32_t* order,
+                          const int32_t* tau, const float* X, int64_t x_rows,
+                          const int32_t* labels, const int32_t* batch_rows, int b,
+                          float* theta, float* m, float* s, int64_t state_stride, double eta,
+                          double mu, double eps, int mode, double kappa, int tf32,
+                          int n_record, const int32_t* record_at, float* record,
+                          double* losses, float* pi_record);
+
 int oracle_mlp_sim_run(int L, const int32_t* dims, int n, int T, const int32_t* order,
                        const int32_t* tau, const float* X, int64_t x_rows,
                        const int32_t* labels, const int32_t* batch_rows, int b,
@@ -188,6 +202,20 @@ int oracle_mlp_sim_run(int L, const int32_t* dims, int n, int T, const int32_t* 
                        double mu, double eps, int mode, double kappa, int tf32,
                        int n_record, const int32_t* record_at, float* record,
                        double* losses) {
+  return oracle_mlp_sim_run_pi(L, dims, n, T, order, tau, X, x_rows, labels, batch_rows, b,
+                               theta, m, s, state_stride, eta, mu, eps, mode, kappa, tf32,
+                               n_record, record_at, record, losses, nullptr);
+}
+
+// As oracle_mlp_sim_run; when pi_record is not NULL, the scaling factors of commit t are
+// written to pi_record[t][0..P).
+int oracle_mlp_sim_run_pi(int L, const int32_t* dims, int n, int T, const int32_t* order,
+                          const int32_t* tau, const float* X, int64_t x_rows,
+                          const int32_t* labels, const int32_t* batch_rows, int b,
+                          float* theta, float* m, float* s, int64_t state_stride, double eta,
+                          double mu, double eps, int mode, double kappa, int tf32,
+                          int n_record, const int32_t* record_at, float* record,
+                          double* losses, float* pi_record) {
   if (L < 1 || n < 1 || T < 0 || b < 1 || !order || !X || !labels || !batch_rows) return -1;
   const int64_t P = param_count(L, dims);
   if (state_stride < P) return -1;
@@ -213,9 +241,9 @@ int oracle_mlp_sim_run(int L, const int32_t* dims, int n, int T, const int32_t* 
     for (int64_t j = 0; j < P; ++j) g32[j] = float(grad[j]);
     const int32_t one_w = w;
     const int32_t one_tau = tau ? tau[t] : 0;
-    const int rc = oracle_gem_run_f32(P, n, 1, &one_w, &one_tau, g32.data(), P, nullptr,
-                                      theta, m, s, state_stride, eta, mu, eps, mode, kappa,
-                                      0, nullptr, 0, nullptr);
+    const int rc = oracle_gem_run_pi_f32(P, n, 1, &one_w, &one_tau, g32.data(), P, nullptr,
+                                         theta, m, s, state_stride, eta, mu, eps, mode, kappa,
+                                         0, pi_record ? pi_record + int64_t(t) * P : nullptr);
     if (rc) return rc;
     while (record && r < n_record && record_at[r] == t) {
       std::memcpy(record + int64_t(r) * P, theta, size_t(P) * sizeof(float));

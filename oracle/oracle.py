@@ -49,6 +49,8 @@ def lib():
         _lib.oracle_mlp_sim_run.argtypes = [i32, p, i32, i32, p, p, p, i64, p, p, i32, p, p,
                                             p, i64, f64, f64, f64, i32, f64, i32, i32, p, p, p]
         _lib.oracle_mlp_sim_run.restype = C.c_int
+        _lib.oracle_mlp_sim_run_pi.argtypes = _lib.oracle_mlp_sim_run.argtypes + [p]
+        _lib.oracle_mlp_sim_run_pi.restype = C.c_int
     return _lib
 
 
@@ -179,9 +181,11 @@ def mlp_loss_grad(dims, theta, X, y, *, tf32=False):
 
 
 def mlp_sim_run(dims, theta, m, s, order, X, labels, batch_rows, *, eta, mu, eps, tau=None,
-                mode=MODE_GEM, kappa=1.0, tf32=False, record_at=(), want_losses=False):
+                mode=MODE_GEM, kappa=1.0, tf32=False, record_at=(), want_losses=False,
+                record_pi=False):
     """End-to-end GEM on the MLP; fp32 state updated in place.  X [rows, d0] holds the
-    rows that batch_rows [T, b] index.  Returns (records [len(record_at), P], losses)."""
+    rows that batch_rows [T, b] index.  Returns (records [len(record_at), P], losses), and
+    with record_pi a third item, the scaling factors [T, P] of every commit."""
     dims_a = np.ascontiguousarray(dims, dtype=np.int32)
     for a, nm in ((theta, "theta"), (m, "m"), (s, "s")):
         _need(a, np.float32, nm)
@@ -197,10 +201,12 @@ def mlp_sim_run(dims, theta, m, s, order, X, labels, batch_rows, *, eta, mu, eps
     rec = np.empty((len(rec_at), P), dtype=np.float32)
     losses = np.empty(T, dtype=np.float64) if want_losses else None
     tau_a = None if tau is None else np.ascontiguousarray(tau, dtype=np.int32)
-    rc = lib().oracle_mlp_sim_run(len(dims) - 1, _ptr(dims_a), n, T, _ptr(order), _ptr(tau_a),
-                                  _ptr(X), X.shape[0], _ptr(labels), _ptr(batch_rows), b,
-                                  _ptr(theta), _ptr(m), _ptr(s), P, eta, mu, eps, mode, kappa,
-                                  int(tf32), len(rec_at), _ptr(rec_at), _ptr(rec), _ptr(losses))
+    pi = np.empty((T, P), dtype=np.float32) if record_pi else None
+    rc = lib().oracle_mlp_sim_run_pi(len(dims) - 1, _ptr(dims_a), n, T, _ptr(order), _ptr(tau_a),
+                                     _ptr(X), X.shape[0], _ptr(labels), _ptr(batch_rows), b,
+                                     _ptr(theta), _ptr(m), _ptr(s), P, eta, mu, eps, mode, kappa,
+                                     int(tf32), len(rec_at), _ptr(rec_at), _ptr(rec), _ptr(losses),
+                                     _ptr(pi))
     if rc:
         raise ValueError(f"oracle_mlp_sim_run failed ({rc})")
-    return rec, losses
+    return (rec, losses, pi) if record_pi else (rec, losses)

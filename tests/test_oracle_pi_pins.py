@@ -133,3 +133,27 @@ def test_median_segments_empty_and_rank_counts():
         for val, r in ((lo[i], (N - 1) // 2), (hi[i], N // 2)):
             assert (v < val).sum() <= r < (v <= val).sum()
         assert np.float64(lo[i]) / 2 + np.float64(hi[i]) / 2 == pytest.approx(np.median(v), rel=1e-15)
+
+
+def test_mlp_simulator_records_the_factors_of_its_commits():
+    """The simulator's first commit applies the gradient at theta_0 (every snapshot is
+    theta_0); its recorded factors equal those of a flat commit of that gradient, which the
+    tests above pin."""
+    from paper_1805_08469_gb300 import synth
+    dims, n, b, seed = [12, 7, 3], 3, 5, 21
+    P = synth.mlp_param_count(dims)
+    rng = np.random.default_rng(seed)
+    X = rng.standard_normal((40, dims[0])).astype(np.float32)
+    y = rng.integers(0, dims[-1], 40).astype(np.int32)
+    rows = rng.integers(0, 40, (4, b)).astype(np.int32)
+    theta0 = (0.3 * rng.standard_normal(P)).astype(np.float32)
+    order = np.array([2, 0, 2, 1], np.int32)
+    th, m, s = theta0.copy(), np.zeros((n, P), np.float32), np.tile(theta0, (n, 1))
+    _r, _l, pi = oracle.mlp_sim_run(dims, th, m, s, order, X, y, rows, eta=0.05, mu=0.9, eps=1e-8,
+                                    record_pi=True)
+    _loss, g = oracle.mlp_loss_grad(dims, theta0.astype(np.float64), X[rows[0]].astype(np.float64), y[rows[0]])
+    th2, m2, s2 = theta0.copy(), np.zeros((n, P), np.float32), np.tile(theta0, (n, 1))
+    ref = oracle.gem_run(th2, m2, s2, g.astype(np.float32)[None, :], [2], eta=0.05, mu=0.9, eps=1e-8,
+                         record_pi=True)
+    assert np.array_equal(pi[0], ref[0])
+    assert pi.shape == (4, P) and np.all(pi >= 0)
