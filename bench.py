@@ -532,7 +532,8 @@ def run_mlp_workloads(args, seed_offset: int = 0) -> dict:
         if args.mlp_commits:
             warm, timed = min(warm, args.mlp_commits), args.mlp_commits
         synth_gpu.data(seed, X, y, dims[-1], stream=stream)
-        T = warm + timed
+        pi_commits = min(timed, 500)      # then per-tensor factor medians on further commits
+        T = warm + timed + pi_commits
         schedule = sim.gem_schedule_uniform if sched == "uniform" else sim.gem_schedule_queue
         order = schedule(seed, n, T)[0]
         batches = synth.schedule_batches(seed, order, b)
@@ -546,17 +547,29 @@ def run_mlp_workloads(args, seed_offset: int = 0) -> dict:
             losses = torch.empty(T, device="cuda")
             sim.gem_mlp_run(M, order[:warm], batches[:warm], losses[:warm])
             stream.synchronize()
-            segs = len(sim.gem_plan_segments(order[warm:], n)) - 1
+            segs = len(sim.gem_plan_segments(order[warm:warm + timed], n)) - 1
             l0 = G.launches()
             e0 = torch.cuda.Event(enable_timing=True)
             e1 = torch.cuda.Event(enable_timing=True)
             e0.record(stream)
-            sim.gem_mlp_run(M, order[warm:], batches[warm:], losses[warm:])
+            sim.gem_mlp_run(M, order[warm:warm + timed], batches[warm:warm + timed],
+                            losses[warm:warm + timed])
             e1.record(stream)
             stream.synchronize()
             ms = e0.elapsed_time(e1)
             commit_launches = G.launches() - l0
-            lh = losses.cpu().numpy()
+            lh = losses[:warm + timed].cpu().numpy()
+            nt = 2 * (len(dims) - 1)
+            pi_lo = torch.empty((pi_commits, nt), device="cuda")
+            pi_hi = torch.empty((pi_commits, nt), device="cuda")
+            a = warm + timed
+            sim.gem_mlp_run_pi(M, order[a:a + 1], batches[a:a + 1], pi_lo[:1], pi_hi[:1])
+            e0.record(stream)   # the first call allocated the factor rows and select scratch
+            sim.gem_mlp_run_pi(M, order[a + 1:], batches[a + 1:], pi_lo[1:], pi_hi[1:], losses[a + 1:])
+            e1.record(stream)
+            stream.synchronize()
+            ms_pi = e0.elapsed_time(e1)
+            med = pi_lo.cpu().numpy()[-100:].mean(axis=0)
             sim.gem_mlp_destroy(M)
             G.close()
         gflop = 2.0 * b * sum(dims[l] * dims[l + 1] for l in range(len(dims) - 1)) * 3 - \
@@ -567,7 +580,10 @@ def run_mlp_workloads(args, seed_offset: int = 0) -> dict:
                      "achieved_tflops": round(gflop * timed / (ms * 1e-3) / 1e12, 2),
                      "commit_launches": int(commit_launches),
                      "loss_first_100": round(float(lh[:100].mean()), 4),
-                     "loss_last_100": round(float(lh[-100:].mean()), 4)}
+                     "loss_last_100": round(float(lh[-100:].mean()), 4),
+                     "with_pi_medians": {"commits_per_s": round((pi_commits - 1) / (ms_pi * 1e-3), 1),
+                                         "commits": pi_commits - 1,
+                                         "median_pi_per_tensor_last_100": [round(float(v), 5) for v in med]}}
     return out
 
 

@@ -92,6 +92,16 @@ int gem_mlp_grad(gem_mlp_t* mlp, const int32_t* workers, int L, const int32_t* b
 int gem_mlp_run(gem_mlp_t* mlp, const int32_t* order, int T, const int32_t* batch_rows,
                 float* losses);
 
+/* gem_mlp_run that also follows the scaling factors, as the experiments section does: for
+ * each commit t, the lower and upper medians (gem_pi_median) of the factors pi that the
+ * commit applied to each tensor of the flat layout [W_1, b_1, ..., W_L, b_L] are written
+ * to pi_lo[t][2L] and pi_hi[t][2L] (device arrays of T * 2 * n_layers floats; tensor 2l is
+ * W_(l+1), 2l + 1 is b_(l+1)).  The commits are the same, bit for bit.  The first call
+ * allocates a factor buffer of n rows of `stride` floats (the size of the gradient
+ * buffers) and the select scratch. */
+int gem_mlp_run_pi(gem_mlp_t* mlp, const int32_t* order, int T, const int32_t* batch_rows,
+                   float* losses, float* pi_lo, float* pi_hi);
+
 /* Wait for the MLP's work on the handle's stream; GEM_ECUDA if device work failed. */
 int gem_mlp_status(gem_mlp_t* mlp);
 

@@ -52,6 +52,7 @@ def _declare(L):
         "gem_mlp_set_data": ([p, p, p, C.c_int64], i),
         "gem_mlp_grad": ([p, p, i, p, p, p], i),
         "gem_mlp_run": ([p, p, i, p, p], i),
+        "gem_mlp_run_pi": ([p, p, i, p, p, p, p], i),
         "gem_mlp_destroy": ([p], None),
         "gem_mlp_status": ([p], i),
         "gem_mlp_grad_static": ([i, p, i, i, p, p, p, C.c_int64, p, p, p, p], i),

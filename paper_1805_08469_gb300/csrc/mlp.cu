@@ -411,6 +411,7 @@ struct gem_mlp {
   float* scratch = nullptr;
   float* grads = nullptr;  // [n][gem stride]
   float* ws = nullptr;     // split-K partial sums
+  float* pi_rows = nullptr;  // [n][gem stride] scaling factors of a segment's commits
   long long ws_floats = 0;
   int32_t* rows_dev = nullptr;  // minibatch rows uploaded from the host
   size_t rows_cap = 0;
@@ -624,6 +625,7 @@ void gem_mlp_destroy(gem_mlp_t* M) {
   cudaFree(M->scratch);
   cudaFree(M->grads);
   cudaFree(M->ws);
+  cudaFree(M->pi_rows);
   cudaFree(M->rows_dev);
   cudaGetLastError();
   cudaSetDevice(dev_prev);
@@ -682,13 +684,29 @@ int gem_mlp_grad(gem_mlp_t* M, const int32_t* workers, int L, const int32_t* bat
   return rc;
 }
 
-int gem_mlp_run(gem_mlp_t* M, const int32_t* order, int T, const int32_t* batch_rows,
-                float* losses) {
+}  // extern "C"
+
+namespace {
+
+// gem_mlp_run, with per-tensor factor medians when pi_lo is not null.
+int mlp_run(gem_mlp_t* M, const int32_t* order, int T, const int32_t* batch_rows,
+            float* losses, float* pi_lo, float* pi_hi) {
   if (!M || T < 0 || (T > 0 && (!order || !batch_rows))) return GEM_EINVAL;
   if (!M->X) return GEM_EINVAL;
   gem_t* h = M->gem;
   if (h->broken) return GEM_ESTATE;
   if (T == 0) return GEM_OK;
+  const bool want_pi = pi_lo != nullptr;
+  int64_t tensors[2 * kMaxLayers + 1];   // offsets of the tensors in the flat layout
+  const int nseg = 2 * M->L;
+  if (want_pi) {
+    if (!pi_hi) return GEM_EINVAL;
+    tensors[0] = 0;
+    for (int l = 0; l < M->L; ++l) {
+      tensors[2 * l + 1] = M->b_off[l];                     // end of W_l
+      tensors[2 * l + 2] = M->b_off[l] + M->dims[l + 1];    // end of b_l
+    }
+  }
   std::vector<int32_t> seg(size_t(T) + 1);
   const int S = gem_plan_segments(order, T, h->n, seg.data());
   if (S < 0) return GEM_EINVAL;
@@ -696,7 +714,15 @@ int gem_mlp_run(gem_mlp_t* M, const int32_t* order, int T, const int32_t* batch_
   cudaGetDevice(&dev_prev);
   cudaSetDevice(h->device);
   int rc = upload_rows(M, batch_rows, (long long)T * M->batch);
+  if (rc == GEM_OK && want_pi && !M->pi_rows) {
+    if (cudaMalloc(&M->pi_rows, sizeof(float) * h->stride * size_t(h->n)) != cudaSuccess) {
+      cudaGetLastError();
+      M->pi_rows = nullptr;
+      rc = GEM_ENOMEM;
+    }
+  }
   std::vector<const float*> gptr(size_t(T) > 0 ? size_t(T) : 1);
+  std::vector<float*> pptr(want_pi ? size_t(T) : 1, nullptr);
   for (int i = 0; i < S && rc == GEM_OK; ++i) {
     const int a = seg[i], e = seg[i + 1];
     for (int c0 = a; c0 < e && rc == GEM_OK; c0 += M->slots) {
@@ -706,13 +732,38 @@ int gem_mlp_run(gem_mlp_t* M, const int32_t* order, int T, const int32_t* batch_
                      losses ? losses + c0 : nullptr);
     }
     if (rc == GEM_OK) {
-      for (int k = a; k < e; ++k) gptr[size_t(k)] = M->grads + (long long)(k - a) * h->stride;
-      rc = cuda_rc(gem::commit_ordered(h, order + a, gptr.data() + a, e - a));
+      for (int k = a; k < e; ++k) {
+        gptr[size_t(k)] = M->grads + (long long)(k - a) * h->stride;
+        if (want_pi) pptr[size_t(k)] = M->pi_rows + (long long)(k - a) * h->stride;
+      }
+      rc = cuda_rc(gem::commit_ordered(h, order + a, gptr.data() + a, e - a,
+                                       want_pi ? pptr.data() + a : nullptr));
+    }
+    if (rc == GEM_OK && want_pi) {
+      const cudaError_t ce = gem::pi_median_ordered(h, pptr.data() + a, e - a, tensors, nseg,
+                                                     pi_lo + (long long)a * nseg,
+                                                     pi_hi + (long long)a * nseg);
+      rc = ce == cudaErrorMemoryAllocation ? GEM_ENOMEM : cuda_rc(ce);
     }
   }
   if (rc == GEM_ECUDA) h->broken = true;
   cudaSetDevice(dev_prev);
   return rc;
+}
+
+}  // namespace
+
+extern "C" {
+
+int gem_mlp_run(gem_mlp_t* M, const int32_t* order, int T, const int32_t* batch_rows,
+                float* losses) {
+  return mlp_run(M, order, T, batch_rows, losses, nullptr, nullptr);
+}
+
+int gem_mlp_run_pi(gem_mlp_t* M, const int32_t* order, int T, const int32_t* batch_rows,
+                   float* losses, float* pi_lo, float* pi_hi) {
+  if (!pi_lo || !pi_hi) return GEM_EINVAL;
+  return mlp_run(M, order, T, batch_rows, losses, pi_lo, pi_hi);
 }
 
 }  // extern "C"

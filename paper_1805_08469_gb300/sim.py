@@ -86,6 +86,18 @@ def gem_mlp_run(h: int, order, batch_rows, losses=None) -> None:
     check(lib().gem_mlp_run(C.c_void_p(h), _p(o), len(o), _p(r), _opt_ptr(losses)), "gem_mlp_run")
 
 
+def gem_mlp_run_pi(h: int, order, batch_rows, pi_lo, pi_hi, losses=None) -> None:
+    """gem_mlp_run that also writes each commit's per-tensor factor medians to pi_lo and
+    pi_hi (float32 CUDA tensors [T, 2 * n_layers])."""
+    from ._lib import check
+    o = np.ascontiguousarray(order, dtype=np.int32)
+    r = np.ascontiguousarray(batch_rows, dtype=np.int32)
+    if r.shape[0] != o.shape[0]:
+        raise ValueError("batch_rows must have one row per commit")
+    check(lib().gem_mlp_run_pi(C.c_void_p(h), _p(o), len(o), _p(r), _opt_ptr(losses),
+                               _opt_ptr(pi_lo), _opt_ptr(pi_hi)), "gem_mlp_run_pi")
+
+
 def gem_mlp_status(h: int) -> None:
     """Waits for the MLP's work; raises if device work failed."""
     from ._lib import check

@@ -180,3 +180,141 @@ def test_argument_checks():
         with pytest.raises(GemError):
             G.commit_batch_pi([0], [g[:P]], [g[1:P + 1]])  # unaligned pi row
         G.sync()
+
+
+def _mlp_setup(dims, n, b, T, seed):
+    from test_gpu_mlp import device_data
+    order, tau = oracle.schedule_uniform(seed, n, T)
+    batches = synth.schedule_batches(seed, order, b)
+    theta0 = synth.xavier_theta0(seed, dims)
+    X, y = device_data(seed)
+    tensors = [0]
+    for (wo, bo, fo, fi) in synth.mlp_layout(dims):
+        tensors += [wo + fo * fi, bo + fo]
+    return order, tau, batches, theta0, X, y, tensors
+
+
+def test_mlp_run_pi_equals_the_flat_calls_bitwise():
+    """gem_mlp_run_pi against the same segments replayed through the public flat calls
+    (gem_mlp_grad for the segment's workers, gem_commit_batch_pi, gem_pi_median over the
+    tensors of the flat layout): identical medians and theta, bit for bit."""
+    from paper_1805_08469_gb300 import sim
+    dims, n, b, T, seed = [784, 64, 10], 4, 32, 60, 1
+    order, _tau, batches, theta0, X, y, tensors = _mlp_setup(dims, n, b, T, seed)
+    P = synth.mlp_param_count(dims)
+    nseg = len(tensors) - 1
+    lo_a = torch.empty((T, nseg), device="cuda")
+    hi_a = torch.empty((T, nseg), device="cuda")
+    with gem.Gem(P, n, ETA, MU, EPS) as A:
+        A.set_theta(torch.from_numpy(theta0).cuda())
+        M = sim.gem_mlp_create(A.h, dims, b)
+        try:
+            sim.gem_mlp_set_data(M, X, y)
+            sim.gem_mlp_run_pi(M, order, batches, lo_a, hi_a)
+            A.sync()
+            theta_a = A.theta().clone()
+        finally:
+            sim.gem_mlp_destroy(M)
+    segs = sim.gem_plan_segments(order, n)
+    lo_b = torch.empty((T, nseg), device="cuda")
+    hi_b = torch.empty((T, nseg), device="cuda")
+    ld = (P + 3) // 4 * 4                                 # 16-byte aligned rows
+    grads = torch.empty((n, ld), device="cuda")
+    pis = torch.empty((n, ld), device="cuda")
+    with gem.Gem(P, n, ETA, MU, EPS) as B:
+        B.set_theta(torch.from_numpy(theta0).cuda())
+        M = sim.gem_mlp_create(B.h, dims, b)
+        try:
+            sim.gem_mlp_set_data(M, X, y)
+            for a, e in zip(segs[:-1], segs[1:]):
+                k = e - a
+                sim.gem_mlp_grad(M, order[a:e], batches[a:e], [grads[i, :P] for i in range(k)])
+                B.commit_batch_pi(order[a:e].tolist(), [grads[i, :P] for i in range(k)],
+                                  [pis[i, :P] for i in range(k)])
+                B.pi_median([pis[i, :P] for i in range(k)], tensors, lo_b[a:e], hi_b[a:e])
+            B.sync()
+            theta_b = B.theta().clone()
+        finally:
+            sim.gem_mlp_destroy(M)
+    assert torch.equal(theta_a, theta_b)
+    assert torch.equal(lo_a, lo_b) and torch.equal(hi_a, hi_b)
+
+
+def test_mlp_run_pi_against_the_oracle_simulator():
+    """Per-tensor medians of the factors of every commit against the oracle simulator's
+    recorded factors (sorted on the host), n = 4, 40 commits from theta_0.  The two
+    trajectories agree to rounding (1e-4 relative over this horizon); a factor's numerator
+    |m| - |theta - s| subtracts close numbers, which amplifies that difference, and a
+    median moves by at most the largest change of the factors around it, so the bar is
+    1e-3 relative."""
+    n, T = 4, 40
+    from paper_1805_08469_gb300 import sim
+    from test_gpu_mlp import host_rows
+    dims, b, seed = [784, 64, 10], 32, 1
+    order, _tau, batches, theta0, X, y, tensors = _mlp_setup(dims, n, b, T, seed)
+    P = synth.mlp_param_count(dims)
+    nseg = len(tensors) - 1
+    lo = torch.empty((T, nseg), device="cuda")
+    hi = torch.empty((T, nseg), device="cuda")
+    with gem.Gem(P, n, ETA, MU, EPS) as G:
+        G.set_theta(torch.from_numpy(theta0).cuda())
+        M = sim.gem_mlp_create(G.h, dims, b)
+        try:
+            sim.gem_mlp_set_data(M, X, y)
+            sim.gem_mlp_run_pi(M, order, batches, lo, hi)
+            G.sync()
+        finally:
+            sim.gem_mlp_destroy(M)
+    glo, ghi = lo.cpu().numpy(), hi.cpu().numpy()
+    Xh, yh, local = host_rows(seed, batches)
+    th, m, s = theta0.copy(), np.zeros((n, P), np.float32), np.tile(theta0, (n, 1))
+    _r, _l, pi = oracle.mlp_sim_run(dims, th, m, s, order, Xh, yh, local, eta=ETA, mu=MU, eps=EPS,
+                                    record_pi=True)
+    for t in range(T):
+        rlo, rhi = oracle.pi_median(pi[t], tensors)
+        np.testing.assert_allclose(glo[t], rlo, rtol=1e-3, atol=1e-7, err_msg=f"commit {t} lower")
+        np.testing.assert_allclose(ghi[t], rhi, rtol=1e-3, atol=1e-7, err_msg=f"commit {t} upper")
+    assert np.any(glo > 0) and np.any(glo < 1)          # the factors vary over the run
+
+
+def test_mlp_run_pi_windows_resumed_from_the_oracle():
+    """n = 16, where the drift |theta - s| is larger and the factors more sensitive: windows
+    of 4 commits resumed from the oracle's state (gem_load_state) at commits 0, 16, 32 and
+    48, so the two sides differ only by the rounding of this window's gradients; medians
+    within 1e-3 relative."""
+    from paper_1805_08469_gb300 import sim
+    from test_gpu_mlp import host_rows
+    dims, n, b, seed, W = [784, 64, 10], 16, 32, 1, 4
+    starts = [0, 16, 32, 48]
+    T = starts[-1] + W
+    order, _tau, batches, theta0, X, y, tensors = _mlp_setup(dims, n, b, T, seed)
+    P = synth.mlp_param_count(dims)
+    nseg = len(tensors) - 1
+    Xh, yh, local = host_rows(seed, batches)
+    th, m, s = theta0.copy(), np.zeros((n, P), np.float32), np.tile(theta0, (n, 1))
+    states, t = {}, 0
+    ref_pi = np.empty((T, P), np.float32)
+    for c in starts + [T]:
+        if c > t:
+            _r, _l, pi = oracle.mlp_sim_run(dims, th, m, s, order[t:c], Xh, yh, local[t:c], eta=ETA,
+                                            mu=MU, eps=EPS, record_pi=True)
+            ref_pi[t:c] = pi
+        states[c] = (th.copy(), m.copy(), s.copy())
+        t = c
+    lo = torch.empty((W, nseg), device="cuda")
+    hi = torch.empty((W, nseg), device="cuda")
+    with gem.Gem(P, n, ETA, MU, EPS) as G:
+        M = sim.gem_mlp_create(G.h, dims, b)
+        try:
+            sim.gem_mlp_set_data(M, X, y)
+            for c in starts:
+                gem.gem_load_state(G.h, *states[c])
+                sim.gem_mlp_run_pi(M, order[c:c + W], batches[c:c + W], lo, hi)
+                G.sync()
+                glo, ghi = lo.cpu().numpy(), hi.cpu().numpy()
+                for i in range(W):
+                    rlo, rhi = oracle.pi_median(ref_pi[c + i], tensors)
+                    np.testing.assert_allclose(glo[i], rlo, rtol=1e-3, atol=1e-7, err_msg=f"commit {c + i}")
+                    np.testing.assert_allclose(ghi[i], rhi, rtol=1e-3, atol=1e-7, err_msg=f"commit {c + i}")
+        finally:
+            sim.gem_mlp_destroy(M)
