@@ -48,8 +48,8 @@ FALLBACK_HBM_GBS = 6800.0
 # DRAM traffic of one launch of the batched commit kernel, from an ncu capture of the
 # same workload (see profiles/commit_batch_p25m_n100.md).  Valid only for the kernel
 # source it was taken on; reported as null once that source changes.
-NCU_TRAFFIC_BYTES_PER_LAUNCH = 44_734_500_000   # mean of two full-size launches
-NCU_TRAFFIC_SOURCE_SHA = "24881a78b514977c"
+NCU_TRAFFIC_BYTES_PER_LAUNCH = 44_737_829_120   # mean of two full-size launches
+NCU_TRAFFIC_SOURCE_SHA = "afc2bd2d841409cd"
 
 
 def kernel_source_sha() -> str:
@@ -291,7 +291,8 @@ def run_gem(args, world, rank, local, pg):
     seed = SEED + rank
     stream = torch.cuda.Stream()
     steps_total = args.warmup + args.steps
-    order, _ = sim.gem_schedule_uniform(seed, N_WORKERS, steps_total * K_BATCH)
+    # the rule and factor-statistics sections reuse batches 0..10
+    order, _ = sim.gem_schedule_uniform(seed, N_WORKERS, max(steps_total, 11) * K_BATCH)
 
     with torch.cuda.stream(stream):
         G = gem.Gem(P_FULL, N_WORKERS, ETA, MU, EPS, stream=stream)
