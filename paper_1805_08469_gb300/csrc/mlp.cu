@@ -37,8 +37,8 @@ constexpr int kMaxClasses = 32;
 constexpr int kMaxBatch = 1024;
 
 // SIMT tile: 128 (or 64) x 64 outputs per block of 256 (or 128) threads, 8 x 4 per thread,
-// k-steps of 16.
-constexpr int BM = 128, BN = 64, BK = 16;
+// k-steps of 16 (also the split-K granularity).
+constexpr int BN = 64, BK = 16;
 constexpr long long kSmCountHint = 152;  // GB300
 constexpr int kMaxSplit = 4;             // split-K factor at most
 
@@ -104,7 +104,7 @@ gemm_grouped_kernel(const __grid_constant__ GemmArgs p) {
   const float* A = p.A.base + (p.A.by_worker ? (long long)p.workers[g] : (long long)g) * p.A.group_stride;
   const float* B = p.B.base + (p.B.by_worker ? (long long)p.workers[g] : (long long)g) * p.B.group_stride;
   const long long lda = p.A.ld, ldb = p.B.ld;
-  const int M = p.M, N = p.N, K = p.K;
+  const int M = p.M, N = p.N;
 
   // staging: 8 A elements and 4 B elements per thread per k-tile
   float ra[8], rb[kBPer];
@@ -206,6 +206,335 @@ gemm_grouped_kernel(const __grid_constant__ GemmArgs p) {
       if (EPI == kBiasRelu) v = fmaxf(v + bias[n], 0.f);
       if (EPI == kMask) v = mask[m * p.ldmask + n] > 0.f ? v : 0.f;
       C[m * p.ldc + n] = v;
+    }
+  }
+}
+
+// The same products with TF32 operands on the tensor cores (warp-level mma.sync, m16n8k8,
+// fp32 accumulation), used for GEM_MLP_TF32.  Operands are rounded to TF32 exactly as the
+// CUDA-core path rounds them (to_tf32) while they are staged, so the tensor cores see the
+// same operand values; products of TF32 values are exact, and the sums are fp32 in the
+// tensor cores' order.
+//
+// 128 x TBN tile per block of 256 threads: 8 warps as 2 (m) x 4 (n), each owning a 64 x TBN/4
+// sub-tile of m16n8 accumulators.  k-tiles of 16 are staged m- (n-) major in shared memory
+// with a row pitch of 20 floats, so the fragment reads (rows gid, columns tig) of a warp hit
+// 32 different banks; double-buffered, with the next k-tile read into registers while the
+// current one is multiplied.
+constexpr int kMmaBM = 128, kMmaBK = 16, kMmaPitch = kMmaBK + 4;
+
+__device__ __forceinline__ void mma_tf32(float (&c)[4], const uint32_t (&a)[4], uint32_t b0,
+                                         uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k8.row.col.f32.tf32.tf32.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, "
+      "{%8, %9}, {%0, %1, %2, %3};"
+      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+
+template <int TBN, bool A_KMAJOR, bool B_KMAJOR, int EPI>
+__global__ void __launch_bounds__(256)
+gemm_mma_tf32_kernel(const __grid_constant__ GemmArgs p) {
+  constexpr int kT = 256;
+  constexpr int kWN = TBN / 4;            // columns per warp
+  constexpr int kNT = kWN / 8;            // n8 tiles per warp
+  constexpr int kAPer = kMmaBM * kMmaBK / kT;   // 8
+  constexpr int kBPer = TBN * kMmaBK / kT;      // 4 or 8
+  __shared__ __align__(16) float As[2][kMmaBM][kMmaPitch];
+  __shared__ __align__(16) float Bs[2][TBN][kMmaPitch];
+  const int split = p.ksplit > 1 ? p.ksplit : 1;
+  const int g = blockIdx.z / split, sk = blockIdx.z - g * split;
+  const int kbeg = sk * p.kchunk;
+  const int kend = split > 1 ? min(p.K, kbeg + p.kchunk) : p.K;
+  const int m0 = blockIdx.y * kMmaBM, n0 = blockIdx.x * TBN;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int wm = warp >> 2, wn = warp & 3;          // warp position: 2 x 4
+  const int gid = lane >> 2, tig = lane & 3;        // mma fragment coordinates
+  const float* A = p.A.base + (p.A.by_worker ? (long long)p.workers[g] : (long long)g) * p.A.group_stride;
+  const float* B = p.B.base + (p.B.by_worker ? (long long)p.workers[g] : (long long)g) * p.B.group_stride;
+  const long long lda = p.A.ld, ldb = p.B.ld;
+  const int M = p.M, N = p.N;
+
+  // staging coordinates: coalesced along k for K-major operands, along m (n) otherwise
+  float ra[kAPer], rb[kBPer];
+  auto a_coord = [&](int it, int& m, int& k) {
+    const int idx = tid + kT * it;
+    if (A_KMAJOR) { m = idx >> 4; k = idx & 15; }
+    else          { m = idx & (kMmaBM - 1); k = idx / kMmaBM; }
+  };
+  auto b_coord = [&](int it, int& n, int& k) {
+    const int idx = tid + kT * it;
+    if (B_KMAJOR) { n = idx >> 4; k = idx & 15; }
+    else          { n = idx % TBN; k = idx / TBN; }
+  };
+  auto load = [&](int k0) {
+#pragma unroll
+    for (int it = 0; it < kAPer; ++it) {
+      int m, k;
+      a_coord(it, m, k);
+      const int gm = m0 + m, gk = k0 + k;
+      float v = 0.f;
+      if (gm < M && gk < kend) v = A_KMAJOR ? A[gm * lda + gk] : A[gk * lda + gm];
+      ra[it] = to_tf32(v);
+    }
+#pragma unroll
+    for (int it = 0; it < kBPer; ++it) {
+      int n, k;
+      b_coord(it, n, k);
+      const int gn = n0 + n, gk = k0 + k;
+      float v = 0.f;
+      if (gn < N && gk < kend) v = B_KMAJOR ? B[gn * ldb + gk] : B[gk * ldb + gn];
+      rb[it] = to_tf32(v);
+    }
+  };
+  auto store = [&](int buf) {
+#pragma unroll
+    for (int it = 0; it < kAPer; ++it) {
+      int m, k;
+      a_coord(it, m, k);
+      As[buf][m][k] = ra[it];
+    }
+#pragma unroll
+    for (int it = 0; it < kBPer; ++it) {
+      int n, k;
+      b_coord(it, n, k);
+      Bs[buf][n][k] = rb[it];
+    }
+  };
+
+  float acc[4][kNT][4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i)
+#pragma unroll
+    for (int j = 0; j < kNT; ++j)
+#pragma unroll
+      for (int e = 0; e < 4; ++e) acc[i][j][e] = 0.f;
+
+  load(kbeg);
+  store(0);
+  __syncthreads();
+  int buf = 0;
+  for (int k0 = kbeg; k0 < kend; k0 += kMmaBK) {
+    const bool more = k0 + kMmaBK < kend;
+    if (more) load(k0 + kMmaBK);
+#pragma unroll
+    for (int ks = 0; ks < kMmaBK; ks += 8) {
+      uint32_t af[4][4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const int r = wm * 64 + i * 16 + gid;
+        af[i][0] = __float_as_uint(As[buf][r][ks + tig]);
+        af[i][1] = __float_as_uint(As[buf][r + 8][ks + tig]);
+        af[i][2] = __float_as_uint(As[buf][r][ks + tig + 4]);
+        af[i][3] = __float_as_uint(As[buf][r + 8][ks + tig + 4]);
+      }
+#pragma unroll
+      for (int j = 0; j < kNT; ++j) {
+        const int c = wn * kWN + j * 8 + gid;
+        const uint32_t b0 = __float_as_uint(Bs[buf][c][ks + tig]);
+        const uint32_t b1 = __float_as_uint(Bs[buf][c][ks + tig + 4]);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) mma_tf32(acc[i][j], af[i], b0, b1);
+      }
+    }
+    if (more) {
+      store(buf ^ 1);   // the other buffer was last read before the previous barrier
+      __syncthreads();
+      buf ^= 1;
+    }
+  }
+
+  // accumulator (i, j, e) holds C(row, col) with row = base + i*16 + gid + 8 (e >= 2),
+  // col = base + j*8 + 2 tig + (e & 1)
+  float* C = p.C + (long long)g * p.c_group_stride;
+  float* W = split > 1 ? p.ws + (long long)blockIdx.z * M * N : nullptr;
+  const float* bias = (EPI == kBias || EPI == kBiasRelu)
+                          ? p.bias + (long long)p.workers[g] * p.bias_group_stride : nullptr;
+  const float* mask = EPI == kMask ? p.mask + (long long)g * p.mask_group_stride : nullptr;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const int m = m0 + wm * 64 + i * 16 + gid + (e >= 2 ? 8 : 0);
+      if (m >= M) continue;
+#pragma unroll
+      for (int j = 0; j < kNT; ++j) {
+        const int n = n0 + wn * kWN + j * 8 + 2 * tig + (e & 1);
+        if (n >= N) continue;
+        float v = acc[i][j][e];
+        if (W) {  // raw partial sums; splitk_reduce_kernel applies the epilogue
+          W[(long long)m * N + n] = v;
+          continue;
+        }
+        if (EPI == kBias) v = v + bias[n];
+        if (EPI == kBiasRelu) v = fmaxf(v + bias[n], 0.f);
+        if (EPI == kMask) v = mask[m * p.ldmask + n] > 0.f ? v : 0.f;
+        C[m * p.ldc + n] = v;
+      }
+    }
+  }
+}
+
+// Pipelined variant for operands whose rows start on 16-byte boundaries (leading
+// dimensions, group strides and bases multiples of 4 floats): k-tiles of 32 are copied
+// global -> shared with cp.async (16-byte chunks, zero-filled past the operand's edge) into a
+// 3-stage ring, so the copies of the next two k-tiles are in flight while the tensor cores
+// work on the current one.  A K-major operand is staged [row][k] (pitch 36 floats), an
+// m- (n-) contiguous one [k][row] (pitch rows + 8); both give conflict-free fragment reads.
+// Operands are rounded to TF32 (cvt.rna: nearest, ties away from zero, as to_tf32) when a
+// fragment is read.
+constexpr int kPipeBK = 32, kPipeStages = 3;
+
+__host__ __device__ constexpr int pipe_tile_floats(int rows, bool kmajor) {
+  return kmajor ? rows * (kPipeBK + 4) : kPipeBK * (rows + 8);
+}
+
+__device__ __forceinline__ uint32_t tf32_bits(float x) {
+  uint32_t r;
+  asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(r) : "f"(x));
+  return r;
+}
+
+__device__ __forceinline__ void cp_async16(void* smem_dst, const void* gmem_src, int src_bytes) {
+  const uint32_t d = static_cast<uint32_t>(__cvta_generic_to_shared(smem_dst));
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(d), "l"(gmem_src), "r"(src_bytes)
+               : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
+
+// Stage the k-tile [k0, k0 + 32) of an operand tile of R rows (m or n) starting at row0:
+// element (row, k) is at src[row * ld + k] (K-major) or src[k * ld + row].  Rows >= rows_end
+// and k >= k_end are zero-filled (a chunk that straddles an edge copies its valid part).
+template <int R, bool KMAJOR>
+__device__ __forceinline__ void stage_tile(float* dst, const float* src, long long ld, int row0,
+                                           int rows_end, int k0, int k_end, int tid) {
+  constexpr int kChunks = R * kPipeBK / 4;
+#pragma unroll
+  for (int i = 0; i < kChunks / 256; ++i) {
+    const int q = tid + 256 * i;
+    int row, k, valid;
+    float* d;
+    if (KMAJOR) {
+      row = q >> 3;
+      k = (q & 7) * 4;
+      d = dst + row * (kPipeBK + 4) + k;
+      valid = (row0 + row < rows_end) ? min(4, max(0, k_end - (k0 + k))) : 0;
+    } else {
+      k = q / (R / 4);
+      row = (q % (R / 4)) * 4;
+      d = dst + k * (R + 8) + row;
+      valid = (k0 + k < k_end) ? min(4, max(0, rows_end - (row0 + row))) : 0;
+    }
+    const float* g = valid ? (KMAJOR ? src + (long long)(row0 + row) * ld + (k0 + k)
+                                     : src + (long long)(k0 + k) * ld + (row0 + row))
+                           : src;
+    cp_async16(d, g, valid * 4);
+  }
+}
+
+template <int TBN, bool A_KMAJOR, bool B_KMAJOR, int EPI>
+__global__ void __launch_bounds__(256)
+gemm_mma_pipe_kernel(const __grid_constant__ GemmArgs p) {
+  constexpr int kWN = TBN / 4, kNT = kWN / 8;
+  constexpr int kAF = pipe_tile_floats(kMmaBM, A_KMAJOR), kBF = pipe_tile_floats(TBN, B_KMAJOR);
+  constexpr int kStageF = kAF + kBF;
+  extern __shared__ __align__(16) float pipe_smem[];
+  const int split = p.ksplit > 1 ? p.ksplit : 1;
+  const int g = blockIdx.z / split, sk = blockIdx.z - g * split;
+  const int kbeg = sk * p.kchunk;
+  const int kend = split > 1 ? min(p.K, kbeg + p.kchunk) : p.K;
+  const int m0 = blockIdx.y * kMmaBM, n0 = blockIdx.x * TBN;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int wm = warp >> 2, wn = warp & 3;
+  const int gid = lane >> 2, tig = lane & 3;
+  const float* A = p.A.base + (p.A.by_worker ? (long long)p.workers[g] : (long long)g) * p.A.group_stride;
+  const float* B = p.B.base + (p.B.by_worker ? (long long)p.workers[g] : (long long)g) * p.B.group_stride;
+  const int M = p.M, N = p.N;
+  const int nkt = kend > kbeg ? (kend - kbeg + kPipeBK - 1) / kPipeBK : 0;
+
+  auto issue = [&](int kt) {
+    float* st = pipe_smem + (kt % kPipeStages) * kStageF;
+    const int k0 = kbeg + kt * kPipeBK;
+    stage_tile<kMmaBM, A_KMAJOR>(st, A, p.A.ld, m0, M, k0, kend, tid);
+    stage_tile<TBN, B_KMAJOR>(st + kAF, B, p.B.ld, n0, N, k0, kend, tid);
+  };
+  auto a_at = [&](const float* t, int row, int k) -> float {
+    return A_KMAJOR ? t[row * (kPipeBK + 4) + k] : t[k * (kMmaBM + 8) + row];
+  };
+  auto b_at = [&](const float* t, int row, int k) -> float {
+    return B_KMAJOR ? t[row * (kPipeBK + 4) + k] : t[k * (TBN + 8) + row];
+  };
+
+  float acc[4][kNT][4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i)
+#pragma unroll
+    for (int j = 0; j < kNT; ++j)
+#pragma unroll
+      for (int e = 0; e < 4; ++e) acc[i][j][e] = 0.f;
+
+#pragma unroll
+  for (int s = 0; s < kPipeStages - 1; ++s) {
+    if (s < nkt) issue(s);
+    cp_async_commit();
+  }
+  for (int kt = 0; kt < nkt; ++kt) {
+    cp_async_wait<kPipeStages - 2>();   // k-tile kt has landed (this thread's copies)
+    __syncthreads();                    // ... everyone's, and stage (kt - 1) is free
+    if (kt + kPipeStages - 1 < nkt) issue(kt + kPipeStages - 1);
+    cp_async_commit();
+    const float* ta = pipe_smem + (kt % kPipeStages) * kStageF;
+    const float* tb = ta + kAF;
+#pragma unroll
+    for (int ks = 0; ks < kPipeBK; ks += 8) {
+      uint32_t af[4][4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const int r = wm * 64 + i * 16 + gid;
+        af[i][0] = tf32_bits(a_at(ta, r, ks + tig));
+        af[i][1] = tf32_bits(a_at(ta, r + 8, ks + tig));
+        af[i][2] = tf32_bits(a_at(ta, r, ks + tig + 4));
+        af[i][3] = tf32_bits(a_at(ta, r + 8, ks + tig + 4));
+      }
+#pragma unroll
+      for (int j = 0; j < kNT; ++j) {
+        const int c = wn * kWN + j * 8 + gid;
+        const uint32_t b0 = tf32_bits(b_at(tb, c, ks + tig));
+        const uint32_t b1 = tf32_bits(b_at(tb, c, ks + tig + 4));
+#pragma unroll
+        for (int i = 0; i < 4; ++i) mma_tf32(acc[i][j], af[i], b0, b1);
+      }
+    }
+  }
+  cp_async_wait<0>();
+
+  float* C = p.C + (long long)g * p.c_group_stride;
+  float* W = split > 1 ? p.ws + (long long)blockIdx.z * M * N : nullptr;
+  const float* bias = (EPI == kBias || EPI == kBiasRelu)
+                          ? p.bias + (long long)p.workers[g] * p.bias_group_stride : nullptr;
+  const float* mask = EPI == kMask ? p.mask + (long long)g * p.mask_group_stride : nullptr;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const int m = m0 + wm * 64 + i * 16 + gid + (e >= 2 ? 8 : 0);
+      if (m >= M) continue;
+#pragma unroll
+      for (int j = 0; j < kNT; ++j) {
+        const int n = n0 + wn * kWN + j * 8 + 2 * tig + (e & 1);
+        if (n >= N) continue;
+        float v = acc[i][j][e];
+        if (W) {
+          W[(long long)m * N + n] = v;
+          continue;
+        }
+        if (EPI == kBias) v = v + bias[n];
+        if (EPI == kBiasRelu) v = fmaxf(v + bias[n], 0.f);
+        if (EPI == kMask) v = mask[m * p.ldmask + n] > 0.f ? v : 0.f;
+        C[m * p.ldc + n] = v;
+      }
     }
   }
 }
@@ -356,35 +685,69 @@ void launch_tile(const GemmArgs& a, int groups, bool tf32, cudaStream_t st) {
     gemm_grouped_kernel<TBM, AK, BK_, EPI, false><<<grid, 2 * TBM, 0, st>>>(a);
 }
 
-// 128-row tiles when the launch fills the GPU; otherwise 64-row tiles (twice the blocks)
-// and, when a split-K workspace is given and K is long, up to kMaxSplit splits of K whose
-// partial sums a second kernel adds in a fixed order.
+bool operand_16b(const Operand& o) {
+  return (reinterpret_cast<uintptr_t>(o.base) & 15u) == 0 && o.ld % 4 == 0 && o.group_stride % 4 == 0;
+}
+
+template <int TBN, bool AK, bool BK_, int EPI>
+void launch_mma(const GemmArgs& a, int groups, cudaStream_t st) {
+  dim3 grid((a.N + TBN - 1) / TBN, (a.M + kMmaBM - 1) / kMmaBM, groups);
+  if (operand_16b(a.A) && operand_16b(a.B)) {
+    constexpr int bytes = kPipeStages * 4 *
+                          (pipe_tile_floats(kMmaBM, AK) + pipe_tile_floats(TBN, BK_));
+    static bool configured[64] = {};   // one attribute call per instantiation and device
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (dev < 0 || dev >= 64 || !configured[dev]) {
+      if (cudaFuncSetAttribute(gemm_mma_pipe_kernel<TBN, AK, BK_, EPI>,
+                               cudaFuncAttributeMaxDynamicSharedMemorySize, bytes) != cudaSuccess)
+        return;   // the error is reported by the caller's cudaGetLastError
+      if (dev >= 0 && dev < 64) configured[dev] = true;
+    }
+    gemm_mma_pipe_kernel<TBN, AK, BK_, EPI><<<grid, 256, bytes, st>>>(a);
+  } else {
+    gemm_mma_tf32_kernel<TBN, AK, BK_, EPI><<<grid, 256, 0, st>>>(a);
+  }
+}
+
+// TF32 products run on the tensor cores (mma.sync), fp32 products on the CUDA cores.  The
+// large tile (128 x 128 on the tensor cores, 128 x 64 on the CUDA cores) when the launch
+// fills the GPU with at least two blocks per SM; otherwise the half-size tile and, when a
+// split-K workspace is given and K is long, up to kMaxSplit splits of K whose partial sums a
+// second kernel adds in a fixed order.
 template <bool AK, bool BK_, int EPI>
 cudaError_t launch_gemm(const GemmArgs& a_in, int groups, bool tf32, cudaStream_t st) {
   GemmArgs a = a_in;
   a.ksplit = 1;
   a.kchunk = a.K;
-  const long long blocks128 = (long long)((a.N + BN - 1) / BN) * ((a.M + BM - 1) / BM) * groups;
-  if (blocks128 >= 2 * kSmCountHint) {
-    launch_tile<128, AK, BK_, EPI>(a, groups, tf32, st);
+  const long long mt = (a.M + 127) / 128, nt64 = (a.N + 63) / 64, nt128 = (a.N + 127) / 128;
+  const long long big = (tf32 ? nt128 : nt64) * mt * groups;
+  if (big >= 2 * kSmCountHint) {
+    if (tf32)
+      launch_mma<128, AK, BK_, EPI>(a, groups, st);
+    else
+      launch_tile<128, AK, BK_, EPI>(a, groups, false, st);
     return cudaGetLastError();
   }
-  const long long blocks64 = (long long)((a.N + BN - 1) / BN) * ((a.M + 63) / 64) * groups;
+  const long long small = tf32 ? nt64 * mt * groups : nt64 * ((a.M + 63) / 64) * groups;
   int split = 1;
   const long long mn = (long long)a.M * a.N * groups;
   if (a.ws && a.M <= 128)
-    while (split < kMaxSplit && blocks64 * split < 4 * kSmCountHint && a.K / (2 * split) >= 128 &&
+    while (split < kMaxSplit && small * split < 4 * kSmCountHint && a.K / (2 * split) >= 128 &&
            mn * 2 * split <= a.ws_floats)
       split *= 2;
-  if (split == 1) {
-    launch_tile<64, AK, BK_, EPI>(a, groups, tf32, st);
-    return cudaGetLastError();
+  if (split > 1) {
+    a.ksplit = split;
+    a.kchunk = ((a.K + split - 1) / split + BK - 1) / BK * BK;
   }
-  a.ksplit = split;
-  a.kchunk = ((a.K + split - 1) / split + BK - 1) / BK * BK;
-  launch_tile<64, AK, BK_, EPI>(a, groups * split, tf32, st);
-  const long long total = (long long)a.M * a.N * groups;
-  splitk_reduce_kernel<EPI><<<unsigned((total + 255) / 256), 256, 0, st>>>(a, groups);
+  if (tf32)
+    launch_mma<64, AK, BK_, EPI>(a, groups * split, st);
+  else
+    launch_tile<64, AK, BK_, EPI>(a, groups * split, false, st);
+  if (split > 1) {
+    const long long total = (long long)a.M * a.N * groups;
+    splitk_reduce_kernel<EPI><<<unsigned((total + 255) / 256), 256, 0, st>>>(a, groups);
+  }
   return cudaGetLastError();
 }
 

@@ -57,11 +57,11 @@ def test_static_scratch_gradient_matches_allocating_entry_point(dims, b, precisi
                 torch.cuda.synchronize()
                 # The allocating entry point splits long K sums across blocks (split-K with a
                 # workspace); this one has no workspace and sums each K in one block.  The
-                # orders differ, so the results agree to rounding: 1e-5 in fp32, and in TF32
-                # (operands rounded to 10 mantissa bits, which amplifies order differences in
-                # the deep layers) 1e-3 over the whole gradient, between the last-layer (1e-4) and
-                # deep-layer (1e-2) bars of the TF32 gradient tests.
-                bar = 1e-5 if precision == sim.GEM_MLP_FP32 else 1e-3
+                # orders differ, so the results agree to rounding: 1e-5 in fp32.  In TF32 the
+                # deep layers' gradients move by about 5e-3 for a 1-ulp change of a
+                # pre-activation (the TF32-rounded softmax - onehot no longer cancels over the
+                # classes), so the bar is 1e-2, the deep-layer bar of the TF32 gradient tests.
+                bar = 1e-5 if precision == sim.GEM_MLP_FP32 else 1e-2
                 assert _rel_l2(got, ref) < bar, (call, _rel_l2(got, ref))
                 assert abs(float(loss) - float(ref_loss)) <= bar * abs(float(ref_loss))
         finally:
