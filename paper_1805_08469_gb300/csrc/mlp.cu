@@ -381,8 +381,8 @@ gemm_mma_tf32_kernel(const __grid_constant__ GemmArgs p) {
 // 3-stage ring, so the copies of the next two k-tiles are in flight while the tensor cores
 // work on the current one.  A K-major operand is staged [row][k] (pitch 36 floats), an
 // m- (n-) contiguous one [k][row] (pitch rows + 8); both give conflict-free fragment reads.
-// Operands are rounded to TF32 (cvt.rna: nearest, ties away from zero, as to_tf32) when a
-// fragment is read.
+// Each thread rounds the chunks it copied to TF32 (cvt.rna: nearest, ties away from zero, as
+// to_tf32) once they have landed; K-major fragments are then read with ldmatrix.
 constexpr int kPipeBK = 32, kPipeStages = 3;
 
 __host__ __device__ constexpr int pipe_tile_floats(int rows, bool kmajor) {
@@ -434,6 +434,35 @@ __device__ __forceinline__ void stage_tile(float* dst, const float* src, long lo
   }
 }
 
+// Round, in place, the chunks this thread copied with stage_tile (after they have landed):
+// every staged element is rounded to TF32 once, by the thread that fetched it.
+template <int R, bool KMAJOR>
+__device__ __forceinline__ void round_tile(float* dst, int tid) {
+  constexpr int kChunks = R * kPipeBK / 4;
+#pragma unroll
+  for (int i = 0; i < kChunks / 256; ++i) {
+    const int q = tid + 256 * i;
+    float* d = KMAJOR ? dst + (q >> 3) * (kPipeBK + 4) + (q & 7) * 4
+                      : dst + (q / (R / 4)) * (R + 8) + (q % (R / 4)) * 4;
+    float4 v = *reinterpret_cast<float4*>(d);
+    v.x = __uint_as_float(tf32_bits(v.x));
+    v.y = __uint_as_float(tf32_bits(v.y));
+    v.z = __uint_as_float(tf32_bits(v.z));
+    v.w = __uint_as_float(tf32_bits(v.w));
+    *reinterpret_cast<float4*>(d) = v;
+  }
+}
+
+// Four 8 x 4 blocks of 32-bit words from shared memory in the register layout of an m16n8k8
+// TF32 fragment: lane l supplies the address of row l % 8 of block l / 8; register i of
+// lane t receives word (t / 4, t % 4) of block i.
+__device__ __forceinline__ void ldsm_x4(uint32_t (&r)[4], const float* row_addr) {
+  const uint32_t a = static_cast<uint32_t>(__cvta_generic_to_shared(row_addr));
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+               : "r"(a));
+}
+
 template <int TBN, bool A_KMAJOR, bool B_KMAJOR, int EPI>
 __global__ void __launch_bounds__(256)
 gemm_mma_pipe_kernel(const __grid_constant__ GemmArgs p) {
@@ -480,31 +509,50 @@ gemm_mma_pipe_kernel(const __grid_constant__ GemmArgs p) {
     if (s < nkt) issue(s);
     cp_async_commit();
   }
+  // ldmatrix row of this lane within a 16 x 8 (A) or 16 x 8 pair-of-n-tiles (B) block
+  const int lrow = (lane & 7) + ((lane >> 3) & 1) * 8, lcol = (lane >> 4) * 4;
+  const int brow = (lane & 7) + (lane >> 4) * 8, bcol = ((lane >> 3) & 1) * 4;
   for (int kt = 0; kt < nkt; ++kt) {
-    cp_async_wait<kPipeStages - 2>();   // k-tile kt has landed (this thread's copies)
-    __syncthreads();                    // ... everyone's, and stage (kt - 1) is free
+    cp_async_wait<kPipeStages - 2>();   // this thread's copies of k-tile kt have landed
+    float* ta = pipe_smem + (kt % kPipeStages) * kStageF;
+    float* tb = ta + kAF;
+    round_tile<kMmaBM, A_KMAJOR>(ta, tid);
+    round_tile<TBN, B_KMAJOR>(tb, tid);
+    __syncthreads();                    // everyone's k-tile kt is rounded; stage kt - 1 is free
     if (kt + kPipeStages - 1 < nkt) issue(kt + kPipeStages - 1);
     cp_async_commit();
-    const float* ta = pipe_smem + (kt % kPipeStages) * kStageF;
-    const float* tb = ta + kAF;
 #pragma unroll
     for (int ks = 0; ks < kPipeBK; ks += 8) {
       uint32_t af[4][4];
 #pragma unroll
       for (int i = 0; i < 4; ++i) {
-        const int r = wm * 64 + i * 16 + gid;
-        af[i][0] = tf32_bits(a_at(ta, r, ks + tig));
-        af[i][1] = tf32_bits(a_at(ta, r + 8, ks + tig));
-        af[i][2] = tf32_bits(a_at(ta, r, ks + tig + 4));
-        af[i][3] = tf32_bits(a_at(ta, r + 8, ks + tig + 4));
+        const int r = wm * 64 + i * 16;
+        if (A_KMAJOR) {
+          ldsm_x4(af[i], ta + (r + lrow) * (kPipeBK + 4) + ks + lcol);
+        } else {
+          af[i][0] = __float_as_uint(a_at(ta, r + gid, ks + tig));
+          af[i][1] = __float_as_uint(a_at(ta, r + gid + 8, ks + tig));
+          af[i][2] = __float_as_uint(a_at(ta, r + gid, ks + tig + 4));
+          af[i][3] = __float_as_uint(a_at(ta, r + gid + 8, ks + tig + 4));
+        }
       }
 #pragma unroll
-      for (int j = 0; j < kNT; ++j) {
-        const int c = wn * kWN + j * 8 + gid;
-        const uint32_t b0 = tf32_bits(b_at(tb, c, ks + tig));
-        const uint32_t b1 = tf32_bits(b_at(tb, c, ks + tig + 4));
+      for (int j = 0; j < kNT; j += 2) {
+        uint32_t bf[4];   // b0, b1 of n-tile j, then of n-tile j + 1
+        const int c = wn * kWN + j * 8;
+        if (B_KMAJOR) {
+          ldsm_x4(bf, tb + (c + brow) * (kPipeBK + 4) + ks + bcol);
+        } else {
+          bf[0] = __float_as_uint(b_at(tb, c + gid, ks + tig));
+          bf[1] = __float_as_uint(b_at(tb, c + gid, ks + tig + 4));
+          bf[2] = __float_as_uint(b_at(tb, c + 8 + gid, ks + tig));
+          bf[3] = __float_as_uint(b_at(tb, c + 8 + gid, ks + tig + 4));
+        }
 #pragma unroll
-        for (int i = 0; i < 4; ++i) mma_tf32(acc[i][j], af[i], b0, b1);
+        for (int i = 0; i < 4; ++i) {
+          mma_tf32(acc[i][j], af[i], bf[0], bf[1]);
+          mma_tf32(acc[i][j + 1], af[i], bf[2], bf[3]);
+        }
       }
     }
   }
@@ -560,51 +608,101 @@ __global__ void splitk_reduce_kernel(const __grid_constant__ GemmArgs p, int gro
 }
 
 // Products with few outputs per row (N <= kMaxClasses), used for the logits:
-// C[g][m][n] = sum_k A[g][m][k] B[g][n][k] + bias[n], A and B K-major.  One block of 8 warps
-// per row m: warp w sums its slice of k (lane l takes k = l, l + 32, ... inside the slice,
-// coalesced), a fixed butterfly reduces the lanes, and thread n adds the 8 warp sums in
-// order, so the result is deterministic.
+// C[g][m][n] = sum_k A[g][m][k] B[g][n][k] + bias[n], A and B K-major.  The block first
+// copies the worker's B (N x K, TF32-rounded when asked) into shared memory; then each warp
+// takes whole rows m: lane l accumulates k = l, l + 32, ... (coalesced A reads, conflict-free
+// shared reads), a fixed butterfly adds the 32 lane sums, and lane 0 writes the N outputs
+// of the row.  Deterministic.  rows_per_block rows per block.
 template <bool TF32>
 __global__ void __launch_bounds__(256)
-gemm_small_n_kernel(const __grid_constant__ GemmArgs p) {
-  __shared__ float part[8][kMaxClasses];
-  const int g = blockIdx.y, m = blockIdx.x;
+gemm_small_n_kernel(const __grid_constant__ GemmArgs p, int rows_per_block) {
+  extern __shared__ __align__(16) float Bsm[];
+  const int g = blockIdx.y;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const float* A = p.A.base + (p.A.by_worker ? (long long)p.workers[g] : (long long)g) * p.A.group_stride +
-                   (long long)m * p.A.ld;
+  const float* A = p.A.base + (p.A.by_worker ? (long long)p.workers[g] : (long long)g) * p.A.group_stride;
   const float* B = p.B.base + (p.B.by_worker ? (long long)p.workers[g] : (long long)g) * p.B.group_stride;
-  const int slice = ((p.K + 8 * 32 - 1) / (8 * 32)) * 32;
-  const int kb = warp * slice, ke = min(p.K, kb + slice);
-  float acc[kMaxClasses];
-#pragma unroll
-  for (int n = 0; n < kMaxClasses; ++n) acc[n] = 0.f;
-  for (int k = kb + lane; k < ke; k += 32) {
-    const float a = TF32 ? to_tf32(A[k]) : A[k];
-#pragma unroll
-    for (int n = 0; n < kMaxClasses; ++n) {
-      if (n < p.N) {
-        const float b = B[(long long)n * p.B.ld + k];
-        acc[n] = fmaf(a, TF32 ? to_tf32(b) : b, acc[n]);
-      }
+  const int N = p.N, K = p.K;
+  const bool vec = K % 4 == 0 && p.B.ld % 4 == 0 && (reinterpret_cast<uintptr_t>(B) & 15u) == 0;
+  if (vec) {   // 16-byte asynchronous copies, all in flight at once, then rounded in place
+    const int chunks = N * K / 4;
+    for (int c = threadIdx.x; c < chunks; c += blockDim.x) {
+      const int n = (4 * c) / K, k = 4 * c - n * K;
+      cp_async16(Bsm + 4 * c, B + (long long)n * p.B.ld + k, 16);
     }
-  }
-#pragma unroll
-  for (int n = 0; n < kMaxClasses; ++n) {
-    if (n < p.N) {
-      float v = acc[n];
-#pragma unroll
-      for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
-      if (lane == 0) part[warp][n] = v;
+    cp_async_commit();
+    cp_async_wait<0>();
+    if (TF32)
+      for (int c = threadIdx.x; c < chunks; c += blockDim.x) {
+        float4 v = *reinterpret_cast<float4*>(Bsm + 4 * c);
+        v.x = to_tf32(v.x);
+        v.y = to_tf32(v.y);
+        v.z = to_tf32(v.z);
+        v.w = to_tf32(v.w);
+        *reinterpret_cast<float4*>(Bsm + 4 * c) = v;
+      }
+  } else {
+#pragma unroll 8
+    for (int i = threadIdx.x; i < N * K; i += blockDim.x) {
+      const int n = i / K, k = i - n * K;
+      const float v = B[(long long)n * p.B.ld + k];
+      Bsm[i] = TF32 ? to_tf32(v) : v;
     }
   }
   __syncthreads();
-  const int n = threadIdx.x;
-  if (n < p.N) {
-    float v = 0.f;
-    for (int w = 0; w < 8; ++w) v += part[w][n];
-    const float* bias = p.bias + (long long)p.workers[g] * p.bias_group_stride;
-    p.C[(long long)g * p.c_group_stride + (long long)m * p.ldc + n] = v + bias[n];
+  const float* bias = p.bias + (long long)p.workers[g] * p.bias_group_stride;
+  const int r0 = blockIdx.x * rows_per_block;
+  const int r1 = min(p.M, r0 + rows_per_block);
+  for (int m = r0 + warp; m < r1; m += 8) {
+    const float* a = A + (long long)m * p.A.ld;
+    float acc[kMaxClasses];
+#pragma unroll
+    for (int n = 0; n < kMaxClasses; ++n) acc[n] = 0.f;
+#pragma unroll 4
+    for (int k = lane; k < K; k += 32) {
+      const float av = TF32 ? to_tf32(a[k]) : a[k];
+#pragma unroll
+      for (int n = 0; n < kMaxClasses; ++n)
+        if (n < N) acc[n] = fmaf(av, Bsm[n * K + k], acc[n]);
+    }
+#pragma unroll
+    for (int n = 0; n < kMaxClasses; ++n) {
+      if (n < N) {
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) acc[n] += __shfl_xor_sync(0xffffffffu, acc[n], off);
+      }
+    }
+    if (lane == 0) {
+      float* c = p.C + (long long)g * p.c_group_stride + (long long)m * p.ldc;
+#pragma unroll
+      for (int n = 0; n < kMaxClasses; ++n)
+        if (n < N) c[n] = acc[n] + bias[n];
+    }
   }
+}
+
+// Launch the logits product when B fits in shared memory; false otherwise.
+template <bool TF32>
+bool launch_small_n(const GemmArgs& a, int groups, cudaStream_t st, cudaError_t* err) {
+  const size_t bytes = sizeof(float) * size_t(a.N) * size_t(a.K);
+  constexpr size_t kMaxBytes = 200 * 1024;
+  if (bytes > kMaxBytes) return false;
+  static bool configured[64] = {};
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (bytes > 48 * 1024 && (dev < 0 || dev >= 64 || !configured[dev])) {
+    *err = cudaFuncSetAttribute(gemm_small_n_kernel<TF32>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                int(kMaxBytes));
+    if (*err != cudaSuccess) return true;
+    if (dev >= 0 && dev < 64) configured[dev] = true;
+  }
+  // enough blocks to cover the SMs about twice, at least 8 rows (one per warp) each
+  long long rows_per_block = (long long)a.M * groups / (2 * kSmCountHint);
+  rows_per_block = rows_per_block < 8 ? 8 : (rows_per_block + 7) / 8 * 8;
+  const int rpb = int(rows_per_block);
+  dim3 grid(unsigned((a.M + rpb - 1) / rpb), unsigned(groups));
+  gemm_small_n_kernel<TF32><<<grid, 256, bytes, st>>>(a, rpb);
+  *err = cudaGetLastError();
+  return true;
 }
 
 // Minibatch gather: slot g's rows X[batch_rows[g][r]] -> Xs[g][r][:].
@@ -732,8 +830,9 @@ cudaError_t launch_gemm(const GemmArgs& a_in, int groups, bool tf32, cudaStream_
   const long long small = tf32 ? nt64 * mt * groups : nt64 * ((a.M + 63) / 64) * groups;
   int split = 1;
   const long long mn = (long long)a.M * a.N * groups;
+  const int min_chunk = tf32 ? 64 : 128;   // the tensor cores get through K faster
   if (a.ws && a.M <= 128)
-    while (split < kMaxSplit && small * split < 4 * kSmCountHint && a.K / (2 * split) >= 128 &&
+    while (split < kMaxSplit && small * split < 4 * kSmCountHint && a.K / (2 * split) >= min_chunk &&
            mn * 2 * split <= a.ws_floats)
       split *= 2;
   if (split > 1) {
@@ -825,14 +924,9 @@ int mlp_chunk(gem_mlp* M, const int32_t* workers, int G, const int32_t* batch_ro
     a.c_group_stride = S;
     a.ldc = dout;
     cudaError_t e;
-    if (last && dout <= kMaxClasses) {
-      // the logits: few outputs per row, one block per row
-      dim3 grid(b, G);
-      if (tf32)
-        gemm_small_n_kernel<true><<<grid, 256, 0, st>>>(a);
-      else
-        gemm_small_n_kernel<false><<<grid, 256, 0, st>>>(a);
-      e = cudaGetLastError();
+    if (last && dout <= kMaxClasses &&
+        (tf32 ? launch_small_n<true>(a, G, st, &e) : launch_small_n<false>(a, G, st, &e))) {
+      // the logits: few outputs per row, the worker's weights held in shared memory
     } else {
       e = last ? launch_gemm<true, true, kBias>(a, G, tf32, st)
                : launch_gemm<true, true, kBiasRelu>(a, G, tf32, st);
