@@ -760,18 +760,31 @@ struct BiasGradArgs {
 };
 
 // db_l[o] = sum over the batch of D_{l+1}[r][o], every layer in one launch.
-__global__ void bias_grad_kernel(const __grid_constant__ BiasGradArgs a, const float* delta,
-                                 long long slot_stride, float* grad, long long grad_stride) {
+// Block of 32 x 8 threads: lane x owns output q = 32 blockIdx.x + x; warp y sums rows
+// r = y, y + 8, ... in order, and lane x of warp 0 adds the 8 warp sums in order.
+__global__ void __launch_bounds__(256)
+bias_grad_kernel(const __grid_constant__ BiasGradArgs a, const float* delta,
+                 long long slot_stride, float* grad, long long grad_stride) {
+  __shared__ float part[8][33];
   const int g = blockIdx.y;
-  const int q = blockIdx.x * blockDim.x + threadIdx.x;
-  if (q >= a.first[a.n_layers]) return;
-  int l = 0;
-  while (q >= a.first[l + 1]) ++l;
-  const int o = q - a.first[l];
-  const float* D = delta + g * slot_stride + a.delta_off[l];
+  const int x = threadIdx.x & 31, y = threadIdx.x >> 5;
+  const int q = blockIdx.x * 32 + x;
   float s = 0.f;
-  for (int r = 0; r < a.b; ++r) s += D[(long long)r * a.width[l] + o];
-  grad[g * grad_stride + a.grad_off[l] + o] = s;
+  int l = 0, o = 0;
+  if (q < a.first[a.n_layers]) {
+    while (q >= a.first[l + 1]) ++l;
+    o = q - a.first[l];
+    const float* D = delta + g * slot_stride + a.delta_off[l];
+    for (int r = y; r < a.b; r += 8) s += D[(long long)r * a.width[l] + o];
+  }
+  part[y][x] = s;
+  __syncthreads();
+  if (y == 0 && q < a.first[a.n_layers]) {
+    float t = 0.f;
+#pragma unroll
+    for (int w = 0; w < 8; ++w) t += part[w][x];
+    grad[g * grad_stride + a.grad_off[l] + o] = t;
+  }
 }
 
 template <int TBM, bool AK, bool BK_, int EPI>
@@ -976,8 +989,8 @@ int mlp_chunk(gem_mlp* M, const int32_t* workers, int G, const int32_t* batch_ro
     ba.width[l] = M->dims[l + 1];
     ba.first[l + 1] = ba.first[l] + M->dims[l + 1];
   }
-  bias_grad_kernel<<<dim3((ba.first[L] + 255) / 256, G), 256, 0, st>>>(ba, scr, S, grads,
-                                                                        grad_stride);
+  bias_grad_kernel<<<dim3((ba.first[L] + 31) / 32, G), 256, 0, st>>>(ba, scr, S, grads,
+                                                                      grad_stride);
   if ((rc = cuda_rc(cudaGetLastError()))) return rc;
   M->launches++;
   return GEM_OK;
