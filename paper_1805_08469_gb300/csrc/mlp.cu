@@ -888,6 +888,11 @@ struct gem_mlp {
   float* ws = nullptr;     // split-K partial sums
   float* pi_rows = nullptr;  // [n][gem stride] scaling factors of a segment's commits
   long long ws_floats = 0;
+  // second stream for the weight-gradient products, which nothing waits for until the
+  // commit; ev_delta[l] marks D_l ready on the main stream, ev_side the side stream's end
+  cudaStream_t side = nullptr;
+  cudaEvent_t ev_delta[kMaxLayers + 1] = {};
+  cudaEvent_t ev_side = nullptr;
   int32_t* rows_dev = nullptr;  // minibatch rows uploaded from the host
   size_t rows_cap = 0;
   uint64_t launches = 0;
@@ -952,17 +957,27 @@ int mlp_chunk(gem_mlp* M, const int32_t* workers, int G, const int32_t* batch_ro
   if ((rc = cuda_rc(cudaGetLastError()))) return rc;
   M->launches++;
 
-  // backward
+  // backward.  The weight-gradient products go to the side stream when there is one: each
+  // waits for its delta D_{l+1} (event recorded on the main stream) and runs next to the
+  // input-gradient chain; they use no split-K workspace, which belongs to the main stream.
+  const bool two_streams = M->side != nullptr;
+  cudaStream_t wst = two_streams ? M->side : st;
   for (int l = L - 1; l >= 0; --l) {
     const int din = M->dims[l], dout = M->dims[l + 1];
+    if (two_streams) {
+      if ((rc = cuda_rc(cudaEventRecord(M->ev_delta[l + 1], st)))) return rc;
+      if ((rc = cuda_rc(cudaStreamWaitEvent(wst, M->ev_delta[l + 1], 0)))) return rc;
+    }
     // dW_l = D_{l+1}^T A_l: (m = o, k = r) from D [b x dout], (k = r, n = j) from A [b x din]
-    a.M = dout; a.N = din; a.K = b;
-    a.A = Operand{scr + M->off_delta[l + 1], S, dout, 0};
-    a.B = Operand{act(l), S, din, 0};
-    a.C = grads + M->w_off[l];
-    a.c_group_stride = grad_stride;
-    a.ldc = din;
-    if ((rc = cuda_rc(launch_gemm<false, false, kStore>(a, G, tf32, st)))) return rc;
+    GemmArgs w = a;
+    w.M = dout; w.N = din; w.K = b;
+    w.A = Operand{scr + M->off_delta[l + 1], S, dout, 0};
+    w.B = Operand{act(l), S, din, 0};
+    w.C = grads + M->w_off[l];
+    w.c_group_stride = grad_stride;
+    w.ldc = din;
+    if (two_streams) w.ws = nullptr;
+    if ((rc = cuda_rc(launch_gemm<false, false, kStore>(w, G, tf32, wst)))) return rc;
     M->launches++;
     if (l == 0) break;
     // D_l = (D_{l+1} W_l) * [A_l > 0]: (m = r, k = o) from D, (k = o, n = j) from W_l [dout x din]
@@ -993,6 +1008,10 @@ int mlp_chunk(gem_mlp* M, const int32_t* workers, int G, const int32_t* batch_ro
                                                                       grad_stride);
   if ((rc = cuda_rc(cudaGetLastError()))) return rc;
   M->launches++;
+  if (two_streams) {   // the gradients are complete once the side stream is
+    if ((rc = cuda_rc(cudaEventRecord(M->ev_side, wst)))) return rc;
+    if ((rc = cuda_rc(cudaStreamWaitEvent(st, M->ev_side, 0)))) return rc;
+  }
   return GEM_OK;
 }
 
@@ -1073,12 +1092,20 @@ int gem_mlp_create(gem_t* g, int n_layers, const int32_t* dims, int batch, int p
     M->ws_floats = (long long)kMaxSplit * 128 * widest * M->slots;
     e = cudaMalloc(&M->ws, sizeof(float) * size_t(M->ws_floats));
   }
+  if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&M->side, cudaStreamNonBlocking);
+  for (int l = 0; l <= n_layers && e == cudaSuccess; ++l)
+    e = cudaEventCreateWithFlags(&M->ev_delta[l], cudaEventDisableTiming);
+  if (e == cudaSuccess) e = cudaEventCreateWithFlags(&M->ev_side, cudaEventDisableTiming);
   cudaSetDevice(dev_prev);
   if (e != cudaSuccess) {
     cudaGetLastError();
     cudaFree(M->scratch);
     cudaFree(M->grads);
     cudaFree(M->ws);
+    for (int l = 0; l <= kMaxLayers; ++l)
+      if (M->ev_delta[l]) cudaEventDestroy(M->ev_delta[l]);
+    if (M->ev_side) cudaEventDestroy(M->ev_side);
+    if (M->side) cudaStreamDestroy(M->side);
     delete M;
     return GEM_ENOMEM;
   }
@@ -1092,6 +1119,11 @@ void gem_mlp_destroy(gem_mlp_t* M) {
   cudaGetDevice(&dev_prev);
   cudaSetDevice(M->gem->device);
   cudaStreamSynchronize(M->gem->stream);
+  if (M->side) cudaStreamSynchronize(M->side);
+  for (int l = 0; l <= kMaxLayers; ++l)
+    if (M->ev_delta[l]) cudaEventDestroy(M->ev_delta[l]);
+  if (M->ev_side) cudaEventDestroy(M->ev_side);
+  if (M->side) cudaStreamDestroy(M->side);
   cudaFree(M->scratch);
   cudaFree(M->grads);
   cudaFree(M->ws);
