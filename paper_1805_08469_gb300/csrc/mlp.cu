@@ -40,7 +40,16 @@ constexpr int kMaxBatch = 1024;
 // k-steps of 16 (also the split-K granularity).
 constexpr int BN = 64, BK = 16;
 constexpr long long kSmCountHint = 152;  // GB300
-constexpr int kMaxSplit = 4;             // split-K factor at most
+#ifndef GEM_MAX_SPLIT
+#define GEM_MAX_SPLIT 4
+#endif
+#ifndef GEM_TF32_MIN_CHUNK
+#define GEM_TF32_MIN_CHUNK 64
+#endif
+#ifndef GEM_TF32_BIG_TILE_BLOCKS   // large tensor-core tiles once a launch has this many per SM
+#define GEM_TF32_BIG_TILE_BLOCKS 1
+#endif
+constexpr int kMaxSplit = GEM_MAX_SPLIT;   // split-K factor at most
 
 enum Epilogue : int { kStore = 0, kBias = 1, kBiasRelu = 2, kMask = 3 };
 
@@ -383,7 +392,14 @@ gemm_mma_tf32_kernel(const __grid_constant__ GemmArgs p) {
 // m- (n-) contiguous one [k][row] (pitch rows + 8); both give conflict-free fragment reads.
 // Each thread rounds the chunks it copied to TF32 (cvt.rna: nearest, ties away from zero, as
 // to_tf32) once they have landed; K-major fragments are then read with ldmatrix.
-constexpr int kPipeBK = 32, kPipeStages = 3;
+#ifndef GEM_PIPE_BK
+#define GEM_PIPE_BK 32
+#endif
+#ifndef GEM_PIPE_STAGES
+#define GEM_PIPE_STAGES 3
+#endif
+constexpr int kPipeBK = GEM_PIPE_BK, kPipeStages = GEM_PIPE_STAGES;
+static_assert(kPipeBK % 8 == 0 && (64 * kPipeBK / 4) % 256 == 0, "k-tile must split into 16-byte chunks");
 
 __host__ __device__ constexpr int pipe_tile_floats(int rows, bool kmajor) {
   return kmajor ? rows * (kPipeBK + 4) : kPipeBK * (rows + 8);
@@ -417,8 +433,8 @@ __device__ __forceinline__ void stage_tile(float* dst, const float* src, long lo
     int row, k, valid;
     float* d;
     if (KMAJOR) {
-      row = q >> 3;
-      k = (q & 7) * 4;
+      row = q / (kPipeBK / 4);
+      k = (q % (kPipeBK / 4)) * 4;
       d = dst + row * (kPipeBK + 4) + k;
       valid = (row0 + row < rows_end) ? min(4, max(0, k_end - (k0 + k))) : 0;
     } else {
@@ -442,7 +458,7 @@ __device__ __forceinline__ void round_tile(float* dst, int tid) {
 #pragma unroll
   for (int i = 0; i < kChunks / 256; ++i) {
     const int q = tid + 256 * i;
-    float* d = KMAJOR ? dst + (q >> 3) * (kPipeBK + 4) + (q & 7) * 4
+    float* d = KMAJOR ? dst + (q / (kPipeBK / 4)) * (kPipeBK + 4) + (q % (kPipeBK / 4)) * 4
                       : dst + (q / (R / 4)) * (R + 8) + (q % (R / 4)) * 4;
     float4 v = *reinterpret_cast<float4*>(d);
     v.x = __uint_as_float(tf32_bits(v.x));
@@ -833,7 +849,7 @@ cudaError_t launch_gemm(const GemmArgs& a_in, int groups, bool tf32, cudaStream_
   a.kchunk = a.K;
   const long long mt = (a.M + 127) / 128, nt64 = (a.N + 63) / 64, nt128 = (a.N + 127) / 128;
   const long long big = (tf32 ? nt128 : nt64) * mt * groups;
-  if (big >= 2 * kSmCountHint) {
+  if (big >= (tf32 ? GEM_TF32_BIG_TILE_BLOCKS : 2) * kSmCountHint) {
     if (tf32)
       launch_mma<128, AK, BK_, EPI>(a, groups, st);
     else
@@ -843,7 +859,7 @@ cudaError_t launch_gemm(const GemmArgs& a_in, int groups, bool tf32, cudaStream_
   const long long small = tf32 ? nt64 * mt * groups : nt64 * ((a.M + 63) / 64) * groups;
   int split = 1;
   const long long mn = (long long)a.M * a.N * groups;
-  const int min_chunk = tf32 ? 64 : 128;   // the tensor cores get through K faster
+  const int min_chunk = tf32 ? GEM_TF32_MIN_CHUNK : 128;   // the tensor cores get through K faster
   if (a.ws && a.M <= 128)
     while (split < kMaxSplit && small * split < 4 * kSmCountHint && a.K / (2 * split) >= min_chunk &&
            mn * 2 * split <= a.ws_floats)
