@@ -51,6 +51,13 @@ def lib():
         _lib.oracle_mlp_sim_run.restype = C.c_int
         _lib.oracle_mlp_sim_run_pi.argtypes = _lib.oracle_mlp_sim_run.argtypes + [p]
         _lib.oracle_mlp_sim_run_pi.restype = C.c_int
+        _lib.oracle_cnn_param_count.argtypes = [p]
+        _lib.oracle_cnn_param_count.restype = i64
+        _lib.oracle_cnn_loss_grad_f64.argtypes = [p, p, p, p, p, i32, p, p]
+        _lib.oracle_cnn_loss_grad_f64.restype = f64
+        _lib.oracle_cnn_sim_run.argtypes = [p, i32, i32, p, p, p, i64, p, p, i32, p, p, p, p, i64,
+                                            f64, f64, f64, i32, f64, i32, p, p, p]
+        _lib.oracle_cnn_sim_run.restype = C.c_int
     return _lib
 
 
@@ -210,3 +217,63 @@ def mlp_sim_run(dims, theta, m, s, order, X, labels, batch_rows, *, eta, mu, eps
     if rc:
         raise ValueError(f"oracle_mlp_sim_run failed ({rc})")
     return (rec, losses, pi) if record_pi else (rec, losses)
+
+
+# The MNIST convolutional network of Appendix A: shape = (H, c1, c2, f1, f2, C).
+CNN_MNIST = (28, 10, 20, 128, 64, 10)
+
+
+def cnn_param_count(shape) -> int:
+    sh = np.ascontiguousarray(shape, dtype=np.int32)
+    P = int(lib().oracle_cnn_param_count(_ptr(sh)))
+    if P < 0:
+        raise ValueError(f"invalid network shape {tuple(shape)}")
+    return P
+
+
+def cnn_loss_grad(shape, theta, X, y, drop, *, want_logits=False):
+    """Mean loss, gradient [P] (double) and optionally logits [b, C] of the network at
+    theta for the samples X [b, H*H], labels y [b] and dropout scales drop [b, c2]."""
+    sh = np.ascontiguousarray(shape, dtype=np.int32)
+    theta = np.ascontiguousarray(theta, dtype=np.float64)
+    X = np.ascontiguousarray(X, dtype=np.float64)
+    y = np.ascontiguousarray(y, dtype=np.int32)
+    drop = np.ascontiguousarray(drop, dtype=np.float64)
+    b = X.shape[0]
+    grad = np.empty_like(theta)
+    logits = np.empty((b, shape[5]), dtype=np.float64) if want_logits else None
+    loss = lib().oracle_cnn_loss_grad_f64(_ptr(sh), _ptr(theta), _ptr(X), _ptr(y), _ptr(drop), b,
+                                          _ptr(grad), _ptr(logits))
+    if np.isnan(loss):
+        raise ValueError("invalid shape or label")
+    return (float(loss), grad, logits) if want_logits else (float(loss), grad)
+
+
+def cnn_sim_run(shape, theta, m, s, order, X, labels, batch_rows, drop, *, eta, mu, eps,
+                tau=None, mode=MODE_GEM, kappa=1.0, record_at=(), want_losses=False):
+    """End-to-end GEM on the CNN; fp32 state updated in place.  X [rows, H*H] holds the
+    rows that batch_rows [T, b] index; drop [T, b, c2] the dropout scales of each commit.
+    Returns (records [len(record_at), P], losses)."""
+    sh = np.ascontiguousarray(shape, dtype=np.int32)
+    for a, nm in ((theta, "theta"), (m, "m"), (s, "s")):
+        _need(a, np.float32, nm)
+    P = theta.shape[0]
+    n = m.shape[0]
+    order = np.ascontiguousarray(order, dtype=np.int32)
+    T = order.shape[0]
+    X = np.ascontiguousarray(X, dtype=np.float32)
+    labels = np.ascontiguousarray(labels, dtype=np.int32)
+    batch_rows = np.ascontiguousarray(batch_rows, dtype=np.int32)
+    drop = np.ascontiguousarray(drop, dtype=np.float32)
+    b = batch_rows.shape[1]
+    rec_at = np.ascontiguousarray(sorted(record_at), dtype=np.int32)
+    rec = np.empty((len(rec_at), P), dtype=np.float32)
+    losses = np.empty(T, dtype=np.float64) if want_losses else None
+    tau_a = None if tau is None else np.ascontiguousarray(tau, dtype=np.int32)
+    rc = lib().oracle_cnn_sim_run(_ptr(sh), n, T, _ptr(order), _ptr(tau_a), _ptr(X), X.shape[0],
+                                  _ptr(labels), _ptr(batch_rows), b, _ptr(drop), _ptr(theta),
+                                  _ptr(m), _ptr(s), P, eta, mu, eps, mode, kappa, len(rec_at),
+                                  _ptr(rec_at), _ptr(rec), _ptr(losses))
+    if rc:
+        raise ValueError(f"oracle_cnn_sim_run failed ({rc})")
+    return rec, losses
