@@ -53,6 +53,19 @@ int gem_synth_data(uint64_t seed, int rows, int d_in, int classes, float* X, int
 int gem_synth_xavier(uint64_t seed, const int32_t* dims, int n_layers, float* theta,
                      void* stream);
 
+/* Parameters of the MNIST convolutional network (gem_cnn.h) with shape {H, c1, c2, f1, f2,
+ * C}, PyTorch's default initialisation: tensor t of the flat layout (conv1.W, conv1.b,
+ * conv2.W, conv2.b, fc1.W, fc1.b, fc2.W, fc2.b, fc3.W, fc3.b) holds bound_t (2u - 1),
+ * bound_t = 1 / sqrt(fan_in_t) rounded to fp32, u = (draw(key(seed, 11 + 256 t), q) >> 40)
+ * 2^-24. */
+int gem_synth_cnn_theta0(uint64_t seed, const int32_t* shape, float* theta, void* stream);
+
+/* Channel-dropout scales of commits t0 .. t0 + T - 1: out [T][b][channels], entry
+ * ((t - t0) b + i) channels + c is 0 when (draw(key(seed, 10), (t b + i) channels + c) >> 40)
+ * 2^-24 < p, else 1 / (1 - p) rounded to fp32.  0 <= p < 1. */
+int gem_synth_dropout(uint64_t seed, uint64_t t0, int T, int b, int channels, float p,
+                      float* out, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -57,11 +57,21 @@ def _declare(L):
         "gem_mlp_status": ([p], i),
         "gem_mlp_grad_static": ([i, p, i, i, p, p, p, C.c_int64, p, p, p, p], i),
         "gem_mlp_launch_count": ([p], C.c_uint64),
+        "gem_cnn_param_count": ([p], C.c_int64),
+        "gem_cnn_create": ([p, p, i, p], i),
+        "gem_cnn_set_data": ([p, p, p, C.c_int64], i),
+        "gem_cnn_grad": ([p, p, i, p, p, p, p], i),
+        "gem_cnn_run": ([p, p, i, p, p, p], i),
+        "gem_cnn_status": ([p], i),
+        "gem_cnn_launch_count": ([p], C.c_uint64),
+        "gem_cnn_destroy": ([p], None),
         "gem_synth_theta0": ([C.c_uint64, sz, p, p], i),
         "gem_synth_grad_heavytail": ([C.c_uint64, C.c_uint64, i, sz, sz, p, p], i),
         "gem_synth_grad_loguniform": ([C.c_uint64, C.c_uint64, sz, p, p, p], i),
         "gem_synth_data": ([C.c_uint64, i, i, i, p, p, p], i),
         "gem_synth_xavier": ([C.c_uint64, p, i, p, p], i),
+        "gem_synth_cnn_theta0": ([C.c_uint64, p, p, p], i),
+        "gem_synth_dropout": ([C.c_uint64, C.c_uint64, i, i, i, C.c_float, p, p], i),
     }
     for name, (args, res) in sig.items():
         fn = getattr(L, name)

@@ -1,0 +1,563 @@
+// The MNIST convolutional network of Appendix A as the workers' model (include/gem_cnn.h).
+//
+// A segment of G distinct workers is processed together, each worker's layers reading
+// its snapshot s_w:
+//   conv1_pool_kernel      conv1 + bias, 2 x 2 max-pool, ReLU    (conv1 outputs kept)
+//   conv2_pool_kernel      conv2 + bias, dropout scale, max-pool, ReLU -> the head's input
+//   dense head             fc1 -> fc2 -> fc3, softmax cross-entropy and the backward pass
+//                          of the MLP engine, which also returns the gradient with respect
+//                          to the features
+//   pool2_back_kernel      ReLU mask, route to the window's first maximum, dropout scale
+//   conv2_back_kernel      gradient with respect to conv1's pooled output, ReLU mask,
+//                          route through pool1
+//   conv2_wpart_kernel,    per-sample partial sums of the convolution weight and bias
+//   conv1_wpart_kernel     gradients
+//   conv_finish_kernel     sums of the partials over the minibatch, in sample order
+// Every value is summed in a fixed order, so the gradients do not depend on timing.
+#include <cstdint>
+#include <cstring>
+#include <new>
+#include <vector>
+
+#include "../../include/gem_cnn.h"
+#include "../../include/gem_sim.h"
+#include "gem_internal.h"
+#include "mlp_internal.h"
+
+struct gem_cnn;
+
+namespace {
+
+using gem::mlp::kMaxGroups;
+
+constexpr int kK = 5;  // kernel side
+constexpr int kThreads = 256;
+
+struct Shape {
+  int H, c1, c2, f1, f2, C;
+  int H1, P1, H2, P2, F;
+  long long w1, b1, w2, b2, head, P;
+};
+
+bool make_shape(const int32_t* s, Shape& n) {
+  if (!s) return false;
+  n.H = s[0];
+  n.c1 = s[1];
+  n.c2 = s[2];
+  n.f1 = s[3];
+  n.f2 = s[4];
+  n.C = s[5];
+  if (n.H < kK || n.H > 1024 || n.c1 < 1 || n.c2 < 1 || n.f1 < 1 || n.f2 < 1 || n.C < 2 ||
+      n.C > gem::mlp::kMaxClasses || n.c1 > 256 || n.c2 > 256)
+    return false;
+  n.H1 = n.H - (kK - 1);
+  if (n.H1 % 2) return false;
+  n.P1 = n.H1 / 2;
+  n.H2 = n.P1 - (kK - 1);
+  if (n.H2 < 2 || n.H2 % 2) return false;
+  n.P2 = n.H2 / 2;
+  n.F = n.c2 * n.P2 * n.P2;
+  n.w1 = 0;
+  n.b1 = n.w1 + (long long)n.c1 * kK * kK;
+  n.w2 = n.b1 + n.c1;
+  n.b2 = n.w2 + (long long)n.c2 * n.c1 * kK * kK;
+  n.head = n.b2 + n.c2;
+  n.P = n.head + (long long)n.f1 * n.F + n.f1 + (long long)n.f2 * n.f1 + n.f2 +
+        (long long)n.C * n.f2 + n.C;
+  return true;
+}
+
+long long round32(long long x) { return (x + 31) / 32 * 32; }
+
+int cuda_rc(cudaError_t e) { return e == cudaSuccess ? GEM_OK : GEM_ECUDA; }
+
+struct ConvArgs {
+  int H, c1, c2, H1, P1, H2, P2, F, b, G;
+  const float* X;              // [rows][H * H]
+  const int32_t* rows;         // [G][b] minibatch rows
+  const float* snap;           // GEM snapshots s, [n][snap_stride]
+  long long snap_stride;
+  long long w1, b1, w2, b2;    // parameter offsets
+  const float* drop;           // [G][b][c2] dropout scales
+  float* scr;                  // conv scratch, slot g at scr + g * S
+  long long S;
+  long long o_z1, o_a1, o_z2, o_dz2, o_dz1, o_p1, o_p2;
+  float* head;                 // dense head scratch, slot g at head + g * head_S
+  long long head_S, head_x, head_dx;   // offsets of its input rows and input gradient
+  float* grads;                // gradient of group g at grads + g * grad_stride
+  long long grad_stride;
+  int workers[kMaxGroups];
+};
+
+__device__ __forceinline__ int first_max4(const float* v) {
+  int best = 0;
+#pragma unroll
+  for (int q = 1; q < 4; ++q)
+    if (v[q] > v[best]) best = q;
+  return best;
+}
+
+// One thread per pooled output (g, i, co, py, px) of conv1.
+__global__ void __launch_bounds__(kThreads) conv1_pool_kernel(const __grid_constant__ ConvArgs a) {
+  const long long total = (long long)a.G * a.b * a.c1 * a.P1 * a.P1;
+  const long long q = blockIdx.x * (long long)kThreads + threadIdx.x;
+  if (q >= total) return;
+  const int px = int(q % a.P1), py = int(q / a.P1 % a.P1);
+  const int co = int(q / ((long long)a.P1 * a.P1) % a.c1);
+  const long long gi = q / ((long long)a.P1 * a.P1 * a.c1);   // g * b + i
+  const int g = int(gi / a.b), i = int(gi % a.b);
+  const float* x = a.X + (long long)a.rows[gi] * a.H * a.H;
+  const float* th = a.snap + (long long)a.workers[g] * a.snap_stride;
+  const float* w = th + a.w1 + co * kK * kK;
+  float wr[kK * kK];
+#pragma unroll
+  for (int k = 0; k < kK * kK; ++k) wr[k] = w[k];
+  const float bias = th[a.b1 + co];
+  float* z1 = a.scr + g * a.S + a.o_z1 + ((long long)i * a.c1 + co) * a.H1 * a.H1;
+  float v[4];
+#pragma unroll
+  for (int d = 0; d < 4; ++d) {
+    const int y = 2 * py + (d >> 1), xx = 2 * px + (d & 1);
+    float acc = bias;
+#pragma unroll
+    for (int ky = 0; ky < kK; ++ky)
+#pragma unroll
+      for (int kx = 0; kx < kK; ++kx) acc = fmaf(wr[ky * kK + kx], x[(y + ky) * a.H + xx + kx], acc);
+    v[d] = acc;
+    z1[y * a.H1 + xx] = acc;
+  }
+  const float m = v[first_max4(v)];
+  a.scr[g * a.S + a.o_a1 + (((long long)i * a.c1 + co) * a.P1 + py) * a.P1 + px] = m > 0.f ? m : 0.f;
+}
+
+// One thread per pooled output (g, i, co, py, px) of conv2; writes the head's features.
+__global__ void __launch_bounds__(kThreads) conv2_pool_kernel(const __grid_constant__ ConvArgs a) {
+  const long long total = (long long)a.G * a.b * a.c2 * a.P2 * a.P2;
+  const long long q = blockIdx.x * (long long)kThreads + threadIdx.x;
+  if (q >= total) return;
+  const int px = int(q % a.P2), py = int(q / a.P2 % a.P2);
+  const int co = int(q / ((long long)a.P2 * a.P2) % a.c2);
+  const long long gi = q / ((long long)a.P2 * a.P2 * a.c2);
+  const int g = int(gi / a.b), i = int(gi % a.b);
+  const float* th = a.snap + (long long)a.workers[g] * a.snap_stride;
+  const float* w = th + a.w2 + (long long)co * a.c1 * kK * kK;
+  const float* a1 = a.scr + g * a.S + a.o_a1 + (long long)i * a.c1 * a.P1 * a.P1;
+  const float s = a.drop[gi * a.c2 + co];
+  float v[4];
+#pragma unroll
+  for (int d = 0; d < 4; ++d) v[d] = th[a.b2 + co];
+  for (int ci = 0; ci < a.c1; ++ci) {
+    const float* in = a1 + (long long)ci * a.P1 * a.P1;
+    const float* wc = w + ci * kK * kK;
+#pragma unroll
+    for (int ky = 0; ky < kK; ++ky)
+#pragma unroll
+      for (int kx = 0; kx < kK; ++kx) {
+        const float wv = wc[ky * kK + kx];
+#pragma unroll
+        for (int d = 0; d < 4; ++d) {
+          const int y = 2 * py + (d >> 1), xx = 2 * px + (d & 1);
+          v[d] = fmaf(wv, in[(y + ky) * a.P1 + xx + kx], v[d]);
+        }
+      }
+  }
+  float* z2 = a.scr + g * a.S + a.o_z2 + ((long long)i * a.c2 + co) * a.H2 * a.H2;
+#pragma unroll
+  for (int d = 0; d < 4; ++d) {
+    v[d] = v[d] * s;   // dropout: the channel's scale
+    z2[(2 * py + (d >> 1)) * a.H2 + 2 * px + (d & 1)] = v[d];
+  }
+  const float m = v[first_max4(v)];
+  a.head[g * a.head_S + a.head_x + (long long)i * a.F + (co * a.P2 + py) * a.P2 + px] = m > 0.f ? m : 0.f;
+}
+
+// Gradient into conv2's (pre-dropout) output: the feature gradient through the ReLU, to
+// the window's first maximum, times the channel's dropout scale; zeros elsewhere.
+__global__ void __launch_bounds__(kThreads) pool2_back_kernel(const __grid_constant__ ConvArgs a) {
+  const long long total = (long long)a.G * a.b * a.c2 * a.P2 * a.P2;
+  const long long q = blockIdx.x * (long long)kThreads + threadIdx.x;
+  if (q >= total) return;
+  const int px = int(q % a.P2), py = int(q / a.P2 % a.P2);
+  const int co = int(q / ((long long)a.P2 * a.P2) % a.c2);
+  const long long gi = q / ((long long)a.P2 * a.P2 * a.c2);
+  const int g = int(gi / a.b), i = int(gi % a.b);
+  const long long f = (long long)i * a.F + (co * a.P2 + py) * a.P2 + px;
+  const float feat = a.head[g * a.head_S + a.head_x + f];
+  const float dfeat = a.head[g * a.head_S + a.head_dx + f];
+  const float s = a.drop[gi * a.c2 + co];
+  const long long base = g * a.S + ((long long)i * a.c2 + co) * a.H2 * a.H2;
+  const float* z2 = a.scr + a.o_z2 + base;
+  float* dz2 = a.scr + a.o_dz2 + base;
+  float v[4];
+#pragma unroll
+  for (int d = 0; d < 4; ++d) v[d] = z2[(2 * py + (d >> 1)) * a.H2 + 2 * px + (d & 1)];
+  const int am = first_max4(v);
+  const float gval = feat > 0.f ? dfeat * s : 0.f;
+#pragma unroll
+  for (int d = 0; d < 4; ++d) dz2[(2 * py + (d >> 1)) * a.H2 + 2 * px + (d & 1)] = d == am ? gval : 0.f;
+}
+
+// One thread per pooled output (g, i, ci, py, px) of conv1: the gradient with respect to
+// it (sum over conv2's outputs that read it, channels then kernel rows then columns), the
+// ReLU mask, and the route through pool1 into conv1's output gradient.
+__global__ void __launch_bounds__(kThreads) conv2_back_kernel(const __grid_constant__ ConvArgs a) {
+  const long long total = (long long)a.G * a.b * a.c1 * a.P1 * a.P1;
+  const long long q = blockIdx.x * (long long)kThreads + threadIdx.x;
+  if (q >= total) return;
+  const int px = int(q % a.P1), py = int(q / a.P1 % a.P1);
+  const int ci = int(q / ((long long)a.P1 * a.P1) % a.c1);
+  const long long gi = q / ((long long)a.P1 * a.P1 * a.c1);
+  const int g = int(gi / a.b), i = int(gi % a.b);
+  const float a1v = a.scr[g * a.S + a.o_a1 + (((long long)i * a.c1 + ci) * a.P1 + py) * a.P1 + px];
+  float dv = 0.f;
+  if (a1v > 0.f) {
+    const float* th = a.snap + (long long)a.workers[g] * a.snap_stride;
+    const float* dz2 = a.scr + g * a.S + a.o_dz2 + (long long)i * a.c2 * a.H2 * a.H2;
+    for (int co = 0; co < a.c2; ++co) {
+      const float* wc = th + a.w2 + ((long long)co * a.c1 + ci) * kK * kK;
+      const float* dc = dz2 + (long long)co * a.H2 * a.H2;
+#pragma unroll
+      for (int ky = 0; ky < kK; ++ky) {
+        const int y = py - ky;
+        if (y < 0 || y >= a.H2) continue;
+#pragma unroll
+        for (int kx = 0; kx < kK; ++kx) {
+          const int xx = px - kx;
+          if (xx < 0 || xx >= a.H2) continue;
+          dv = fmaf(dc[y * a.H2 + xx], wc[ky * kK + kx], dv);
+        }
+      }
+    }
+  }
+  const long long base = g * a.S + ((long long)i * a.c1 + ci) * a.H1 * a.H1;
+  const float* z1 = a.scr + a.o_z1 + base;
+  float* dz1 = a.scr + a.o_dz1 + base;
+  float v[4];
+#pragma unroll
+  for (int d = 0; d < 4; ++d) v[d] = z1[(2 * py + (d >> 1)) * a.H1 + 2 * px + (d & 1)];
+  const int am = first_max4(v);
+#pragma unroll
+  for (int d = 0; d < 4; ++d) dz1[(2 * py + (d >> 1)) * a.H1 + 2 * px + (d & 1)] = d == am ? dv : 0.f;
+}
+
+// Per-sample partial sums of conv2's weight and bias gradients: thread (g, i, co, k), k <
+// c1 * 25 a weight (ci, ky, kx), k = c1 * 25 the bias; rows then columns of the output.
+__global__ void __launch_bounds__(kThreads) conv2_wpart_kernel(const __grid_constant__ ConvArgs a) {
+  const int per = a.c1 * kK * kK + 1;
+  const long long total = (long long)a.G * a.b * a.c2 * per;
+  const long long q = blockIdx.x * (long long)kThreads + threadIdx.x;
+  if (q >= total) return;
+  const int k = int(q % per);
+  const int co = int(q / per % a.c2);
+  const long long gi = q / ((long long)per * a.c2);
+  const int g = int(gi / a.b), i = int(gi % a.b);
+  const float* dz2 = a.scr + g * a.S + a.o_dz2 + ((long long)i * a.c2 + co) * a.H2 * a.H2;
+  float acc = 0.f;
+  if (k == per - 1) {
+    for (int p = 0; p < a.H2 * a.H2; ++p) acc += dz2[p];
+  } else {
+    const int ci = k / (kK * kK), ky = k % (kK * kK) / kK, kx = k % kK;
+    const float* a1 = a.scr + g * a.S + a.o_a1 + ((long long)i * a.c1 + ci) * a.P1 * a.P1;
+    for (int y = 0; y < a.H2; ++y)
+      for (int xx = 0; xx < a.H2; ++xx) acc = fmaf(dz2[y * a.H2 + xx], a1[(y + ky) * a.P1 + xx + kx], acc);
+  }
+  a.scr[g * a.S + a.o_p2 + ((long long)i * a.c2 + co) * per + k] = acc;
+}
+
+// Per-sample partial sums of conv1's weight and bias gradients: thread (g, i, co, k), k < 25
+// a weight (ky, kx), k = 25 the bias.
+__global__ void __launch_bounds__(kThreads) conv1_wpart_kernel(const __grid_constant__ ConvArgs a) {
+  constexpr int per = kK * kK + 1;
+  const long long total = (long long)a.G * a.b * a.c1 * per;
+  const long long q = blockIdx.x * (long long)kThreads + threadIdx.x;
+  if (q >= total) return;
+  const int k = int(q % per);
+  const int co = int(q / per % a.c1);
+  const long long gi = q / ((long long)per * a.c1);
+  const int g = int(gi / a.b), i = int(gi % a.b);
+  const float* dz1 = a.scr + g * a.S + a.o_dz1 + ((long long)i * a.c1 + co) * a.H1 * a.H1;
+  float acc = 0.f;
+  if (k == per - 1) {
+    for (int p = 0; p < a.H1 * a.H1; ++p) acc += dz1[p];
+  } else {
+    const int ky = k / kK, kx = k % kK;
+    const float* x = a.X + (long long)a.rows[gi] * a.H * a.H;
+    for (int y = 0; y < a.H1; ++y)
+      for (int xx = 0; xx < a.H1; ++xx) acc = fmaf(dz1[y * a.H1 + xx], x[(y + ky) * a.H + xx + kx], acc);
+  }
+  a.scr[g * a.S + a.o_p1 + ((long long)i * a.c1 + co) * per + k] = acc;
+}
+
+// Convolution gradients: the partials summed over the minibatch in sample order.
+__global__ void __launch_bounds__(kThreads) conv_finish_kernel(const __grid_constant__ ConvArgs a) {
+  const int per1 = kK * kK + 1, per2 = a.c1 * kK * kK + 1;
+  const long long n1 = (long long)a.c1 * per1, n2 = (long long)a.c2 * per2;
+  const long long total = (long long)a.G * (n1 + n2);
+  const long long q = blockIdx.x * (long long)kThreads + threadIdx.x;
+  if (q >= total) return;
+  const int g = int(q / (n1 + n2));
+  const long long e = q % (n1 + n2);
+  float* grad = a.grads + g * a.grad_stride;
+  const float* slot = a.scr + g * a.S;
+  float acc = 0.f;
+  if (e < n1) {
+    const int co = int(e / per1), k = int(e % per1);
+    for (int i = 0; i < a.b; ++i) acc += slot[a.o_p1 + ((long long)i * a.c1 + co) * per1 + k];
+    grad[k < per1 - 1 ? a.w1 + co * (per1 - 1) + k : a.b1 + co] = acc;
+  } else {
+    const long long e2 = e - n1;
+    const int co = int(e2 / per2), k = int(e2 % per2);
+    for (int i = 0; i < a.b; ++i) acc += slot[a.o_p2 + ((long long)i * a.c2 + co) * per2 + k];
+    grad[k < per2 - 1 ? a.w2 + (long long)co * (per2 - 1) + k : a.b2 + co] = acc;
+  }
+}
+
+unsigned blocks_for(long long n) { return unsigned((n + kThreads - 1) / kThreads); }
+
+}  // namespace
+
+struct gem_cnn {
+  gem_t* gem = nullptr;
+  Shape sh{};
+  int batch = 0;
+  gem_mlp* head = nullptr;   // fc1 -> fc2 -> fc3 and the loss, external input
+  const float* X = nullptr;
+  const int32_t* labels = nullptr;
+  int64_t rows = 0;
+  long long o_z1 = 0, o_a1 = 0, o_z2 = 0, o_dz2 = 0, o_dz1 = 0, o_p1 = 0, o_p2 = 0;
+  long long slot_stride = 0;
+  int slots = 0;
+  float* scratch = nullptr;
+  float* grads = nullptr;        // [n][gem stride]
+  int32_t* rows_dev = nullptr;   // minibatch rows uploaded from the host
+  size_t rows_cap = 0;
+  uint64_t launches = 0;
+};
+
+namespace {
+
+// Forward and backward of groups [0, G) of one chunk (workers, rows [G][b] and dropout
+// scales [G][b][c2] on the device), gradient of group g at grads + g * grad_stride.
+int cnn_chunk(gem_cnn* N, const int32_t* workers, int G, const int32_t* rows_dev,
+              const float* drop, float* grads, long long grad_stride, float* losses) {
+  gem_t* h = N->gem;
+  cudaStream_t st = h->stream;
+  const Shape& s = N->sh;
+  ConvArgs a;
+  std::memset(&a, 0, sizeof(a));
+  a.H = s.H; a.c1 = s.c1; a.c2 = s.c2; a.H1 = s.H1; a.P1 = s.P1; a.H2 = s.H2; a.P2 = s.P2;
+  a.F = s.F; a.b = N->batch; a.G = G;
+  a.X = N->X;
+  a.rows = rows_dev;
+  a.snap = h->s;
+  a.snap_stride = (long long)h->stride;
+  a.w1 = s.w1; a.b1 = s.b1; a.w2 = s.w2; a.b2 = s.b2;
+  a.drop = drop;
+  a.scr = N->scratch;
+  a.S = N->slot_stride;
+  a.o_z1 = N->o_z1; a.o_a1 = N->o_a1; a.o_z2 = N->o_z2; a.o_dz2 = N->o_dz2; a.o_dz1 = N->o_dz1;
+  a.o_p1 = N->o_p1; a.o_p2 = N->o_p2;
+  a.head = N->head->scratch;
+  a.head_S = N->head->slot_stride;
+  a.head_x = N->head->off_x;
+  a.head_dx = N->head->off_delta[0];
+  a.grads = grads;
+  a.grad_stride = grad_stride;
+  for (int g = 0; g < G; ++g) a.workers[g] = workers[g];
+  const long long b = N->batch;
+  const long long n_pool1 = G * b * s.c1 * s.P1 * s.P1, n_pool2 = G * b * s.c2 * s.P2 * s.P2;
+  int rc;
+  conv1_pool_kernel<<<blocks_for(n_pool1), kThreads, 0, st>>>(a);
+  conv2_pool_kernel<<<blocks_for(n_pool2), kThreads, 0, st>>>(a);
+  if ((rc = cuda_rc(cudaGetLastError()))) return rc;
+  N->launches += 2;
+  // the dense head: forward, loss, backward, and the feature gradient
+  if ((rc = gem::mlp::mlp_chunk(N->head, workers, G, rows_dev, grads, grad_stride, losses))) return rc;
+  pool2_back_kernel<<<blocks_for(n_pool2), kThreads, 0, st>>>(a);
+  conv2_back_kernel<<<blocks_for(n_pool1), kThreads, 0, st>>>(a);
+  conv2_wpart_kernel<<<blocks_for(G * b * s.c2 * (s.c1 * kK * kK + 1)), kThreads, 0, st>>>(a);
+  conv1_wpart_kernel<<<blocks_for(G * b * s.c1 * (kK * kK + 1)), kThreads, 0, st>>>(a);
+  conv_finish_kernel<<<blocks_for(G * ((long long)s.c1 * (kK * kK + 1) +
+                                       (long long)s.c2 * (s.c1 * kK * kK + 1))),
+                       kThreads, 0, st>>>(a);
+  if ((rc = cuda_rc(cudaGetLastError()))) return rc;
+  N->launches += 5;
+  return GEM_OK;
+}
+
+// Check minibatch rows on the host and copy them to the device (stream-ordered).
+int upload_rows(gem_cnn* N, const int32_t* rows_host, long long count) {
+  for (long long i = 0; i < count; ++i)
+    if (rows_host[i] < 0 || rows_host[i] >= N->rows) return GEM_EINVAL;
+  if ((size_t)count > N->rows_cap) {
+    cudaFree(N->rows_dev);   // synchronises with work still reading the old buffer
+    N->rows_dev = nullptr;
+    N->rows_cap = 0;
+    if (cudaMalloc(&N->rows_dev, sizeof(int32_t) * size_t(count)) != cudaSuccess) {
+      cudaGetLastError();
+      return GEM_ENOMEM;
+    }
+    N->rows_cap = size_t(count);
+  }
+  return cuda_rc(cudaMemcpyAsync(N->rows_dev, rows_host, sizeof(int32_t) * size_t(count),
+                                 cudaMemcpyHostToDevice, N->gem->stream));
+}
+
+}  // namespace
+
+extern "C" {
+
+int64_t gem_cnn_param_count(const int32_t* shape) {
+  Shape s;
+  return make_shape(shape, s) ? s.P : -1;
+}
+
+int gem_cnn_create(gem_t* g, const int32_t* shape, int batch, gem_cnn_t** out) {
+  if (!out) return GEM_EINVAL;
+  *out = nullptr;
+  Shape s;
+  if (!g || !make_shape(shape, s) || batch < 1 || batch > gem::mlp::kMaxBatch) return GEM_EINVAL;
+  if (g->broken) return GEM_ESTATE;
+  if ((size_t)s.P != g->P) return GEM_EINVAL;
+  gem_cnn* N = new (std::nothrow) gem_cnn();
+  if (!N) return GEM_ENOMEM;
+  N->gem = g;
+  N->sh = s;
+  N->batch = batch;
+  const int32_t dims[4] = {s.F, s.f1, s.f2, s.C};
+  int rc = gem::mlp::mlp_build(g, 3, dims, batch, GEM_MLP_FP32, s.head, true, true, false, &N->head);
+  if (rc) {
+    delete N;
+    return rc;
+  }
+  const long long b = batch;
+  long long off = 0;
+  auto take = [&](long long n) {
+    const long long o = off;
+    off += round32(n);
+    return o;
+  };
+  N->o_z1 = take(b * s.c1 * s.H1 * s.H1);
+  N->o_a1 = take(b * s.c1 * s.P1 * s.P1);
+  N->o_z2 = take(b * s.c2 * s.H2 * s.H2);
+  N->o_dz2 = take(b * s.c2 * s.H2 * s.H2);
+  N->o_dz1 = take(b * s.c1 * s.H1 * s.H1);
+  N->o_p1 = take(b * s.c1 * (kK * kK + 1));
+  N->o_p2 = take(b * s.c2 * (s.c1 * kK * kK + 1));
+  N->slot_stride = off;
+  N->slots = N->head->slots;
+  int dev_prev = 0;
+  cudaGetDevice(&dev_prev);
+  cudaSetDevice(g->device);
+  cudaError_t e = cudaMalloc(&N->scratch, sizeof(float) * size_t(N->slot_stride) * N->slots);
+  if (e == cudaSuccess) e = cudaMalloc(&N->grads, sizeof(float) * g->stride * size_t(g->n));
+  cudaSetDevice(dev_prev);
+  if (e != cudaSuccess) {
+    cudaGetLastError();
+    cudaFree(N->scratch);
+    cudaFree(N->grads);
+    gem::mlp::mlp_free(N->head);
+    delete N;
+    return GEM_ENOMEM;
+  }
+  *out = N;
+  return GEM_OK;
+}
+
+void gem_cnn_destroy(gem_cnn_t* N) {
+  if (!N) return;
+  int dev_prev = 0;
+  cudaGetDevice(&dev_prev);
+  cudaSetDevice(N->gem->device);
+  cudaStreamSynchronize(N->gem->stream);
+  cudaFree(N->scratch);
+  cudaFree(N->grads);
+  cudaFree(N->rows_dev);
+  cudaGetLastError();
+  cudaSetDevice(dev_prev);
+  gem::mlp::mlp_free(N->head);
+  delete N;
+}
+
+int gem_cnn_set_data(gem_cnn_t* N, const float* X, const int32_t* labels, int64_t rows) {
+  if (!N || !X || !labels || rows < 1) return GEM_EINVAL;
+  N->X = X;
+  N->labels = labels;
+  N->rows = rows;
+  N->head->labels = labels;
+  N->head->rows = rows;
+  return GEM_OK;
+}
+
+int gem_cnn_status(gem_cnn_t* N) {
+  if (!N) return GEM_EINVAL;
+  return gem_sync(N->gem);
+}
+
+uint64_t gem_cnn_launch_count(const gem_cnn_t* N) {
+  return N ? N->launches + N->head->launches : 0;
+}
+
+int gem_cnn_grad(gem_cnn_t* N, const int32_t* workers, int L, const int32_t* batch_rows,
+                 const float* drop, float* const* grads, float* losses) {
+  if (!N || L < 0 || (L > 0 && (!workers || !batch_rows || !grads || !drop))) return GEM_EINVAL;
+  if (!N->X) return GEM_EINVAL;
+  gem_t* h = N->gem;
+  if (h->broken) return GEM_ESTATE;
+  for (int i = 0; i < L; ++i) {
+    if (workers[i] < 0 || workers[i] >= h->n || !grads[i]) return GEM_EINVAL;
+    if ((reinterpret_cast<uintptr_t>(grads[i]) & 15u) != 0) return GEM_EINVAL;
+  }
+  int dev_prev = 0;
+  cudaGetDevice(&dev_prev);
+  cudaSetDevice(h->device);
+  int rc = upload_rows(N, batch_rows, (long long)L * N->batch);
+  const long long db = (long long)N->batch * N->sh.c2;
+  for (int c0 = 0; c0 < L && rc == GEM_OK; c0 += N->slots) {
+    const int G = (L - c0) < N->slots ? (L - c0) : N->slots;
+    rc = cnn_chunk(N, workers + c0, G, N->rows_dev + (long long)c0 * N->batch, drop + c0 * db,
+                   N->grads, (long long)h->stride, losses ? losses + c0 : nullptr);
+    for (int g = 0; g < G && rc == GEM_OK; ++g)
+      rc = cuda_rc(cudaMemcpyAsync(grads[c0 + g], N->grads + (long long)g * h->stride,
+                                   h->P * sizeof(float), cudaMemcpyDeviceToDevice, h->stream));
+  }
+  if (rc == GEM_ECUDA) h->broken = true;
+  cudaSetDevice(dev_prev);
+  return rc;
+}
+
+int gem_cnn_run(gem_cnn_t* N, const int32_t* order, int T, const int32_t* batch_rows,
+                const float* drop, float* losses) {
+  if (!N || T < 0 || (T > 0 && (!order || !batch_rows || !drop))) return GEM_EINVAL;
+  if (!N->X) return GEM_EINVAL;
+  gem_t* h = N->gem;
+  if (h->broken) return GEM_ESTATE;
+  if (T == 0) return GEM_OK;
+  std::vector<int32_t> seg(size_t(T) + 1);
+  const int S = gem_plan_segments(order, T, h->n, seg.data());
+  if (S < 0) return GEM_EINVAL;
+  int dev_prev = 0;
+  cudaGetDevice(&dev_prev);
+  cudaSetDevice(h->device);
+  int rc = upload_rows(N, batch_rows, (long long)T * N->batch);
+  std::vector<const float*> gptr(static_cast<size_t>(T));
+  const long long db = (long long)N->batch * N->sh.c2;
+  for (int i = 0; i < S && rc == GEM_OK; ++i) {
+    const int a = seg[i], e = seg[i + 1];
+    for (int c0 = a; c0 < e && rc == GEM_OK; c0 += N->slots) {
+      const int G = (e - c0) < N->slots ? (e - c0) : N->slots;
+      rc = cnn_chunk(N, order + c0, G, N->rows_dev + (long long)c0 * N->batch, drop + c0 * db,
+                     N->grads + (long long)(c0 - a) * h->stride, (long long)h->stride,
+                     losses ? losses + c0 : nullptr);
+    }
+    if (rc == GEM_OK) {
+      for (int k = a; k < e; ++k) gptr[size_t(k)] = N->grads + (long long)(k - a) * h->stride;
+      rc = cuda_rc(gem::commit_ordered(h, order + a, gptr.data() + a, e - a));
+    }
+  }
+  if (rc == GEM_ECUDA) h->broken = true;
+  cudaSetDevice(dev_prev);
+  return rc;
+}
+
+}  // extern "C"

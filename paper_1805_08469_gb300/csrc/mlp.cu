@@ -27,14 +27,11 @@
 
 #include "../../include/gem_sim.h"
 #include "gem_internal.h"
+#include "mlp_internal.h"
 
 namespace gem {
 namespace mlp {
 
-constexpr int kMaxLayers = 8;
-constexpr int kMaxGroups = 128;
-constexpr int kMaxClasses = 32;
-constexpr int kMaxBatch = 1024;
 
 // SIMT tile: 128 (or 64) x 64 outputs per block of 256 (or 128) threads, 8 x 4 per thread,
 // k-steps of 16 (also the split-K granularity).
@@ -884,35 +881,8 @@ cudaError_t launch_gemm(const GemmArgs& a_in, int groups, bool tf32, cudaStream_
 
 using namespace gem::mlp;
 
-struct gem_mlp {
-  gem_t* gem = nullptr;
-  int L = 0;
-  int dims[kMaxLayers + 1] = {};
-  long long w_off[kMaxLayers] = {}, b_off[kMaxLayers] = {};
-  int batch = 0;
-  int precision = 0;
-  const float* X = nullptr;
-  const int32_t* labels = nullptr;
-  int64_t rows = 0;
-  // per-slot scratch: X_s [b x d0], A_l [b x d_l] (l = 1..L-1), logits [b x C],
-  // D_l [b x d_l] (l = 1..L)
-  long long off_x = 0, off_act[kMaxLayers + 1] = {}, off_logits = 0, off_delta[kMaxLayers + 1] = {};
-  long long slot_stride = 0;
-  int slots = 0;
-  float* scratch = nullptr;
-  float* grads = nullptr;  // [n][gem stride]
-  float* ws = nullptr;     // split-K partial sums
-  float* pi_rows = nullptr;  // [n][gem stride] scaling factors of a segment's commits
-  long long ws_floats = 0;
-  // second stream for the weight-gradient products, which nothing waits for until the
-  // commit; ev_delta[l] marks D_l ready on the main stream, ev_side the side stream's end
-  cudaStream_t side = nullptr;
-  cudaEvent_t ev_delta[kMaxLayers + 1] = {};
-  cudaEvent_t ev_side = nullptr;
-  int32_t* rows_dev = nullptr;  // minibatch rows uploaded from the host
-  size_t rows_cap = 0;
-  uint64_t launches = 0;
-};
+
+
 
 namespace {
 
@@ -920,8 +890,11 @@ long long round32(long long x) { return (x + 31) / 32 * 32; }
 
 int cuda_rc(cudaError_t e) { return e == cudaSuccess ? GEM_OK : GEM_ECUDA; }
 
-// Forward and backward for groups [0, G) of one chunk: workers[g], minibatch rows
-// batch_rows[g][0..b), gradient of group g written at grads + g * grad_stride.
+}  // namespace
+
+namespace gem {
+namespace mlp {
+
 int mlp_chunk(gem_mlp* M, const int32_t* workers, int G, const int32_t* batch_rows,
               float* grads, long long grad_stride, float* losses) {
   gem_t* h = M->gem;
@@ -932,11 +905,13 @@ int mlp_chunk(gem_mlp* M, const int32_t* workers, int G, const int32_t* batch_ro
   float* scr = M->scratch;
   auto act = [&](int l) -> float* { return l == 0 ? scr + M->off_x : scr + M->off_act[l]; };
 
-  gather_rows_kernel<<<dim3(b, G), 256, 0, st>>>(M->X, M->dims[0], batch_rows, b,
-                                                 scr + M->off_x, S);
-  int rc = cuda_rc(cudaGetLastError());
-  if (rc) return rc;
-  M->launches++;
+  int rc = GEM_OK;
+  if (!M->external_input) {
+    gather_rows_kernel<<<dim3(b, G), 256, 0, st>>>(M->X, M->dims[0], batch_rows, b,
+                                                   scr + M->off_x, S);
+    if ((rc = cuda_rc(cudaGetLastError()))) return rc;
+    M->launches++;
+  }
 
   GemmArgs a;
   std::memset(&a, 0, sizeof(a));
@@ -995,7 +970,19 @@ int mlp_chunk(gem_mlp* M, const int32_t* workers, int G, const int32_t* batch_ro
     if (two_streams) w.ws = nullptr;
     if ((rc = cuda_rc(launch_gemm<false, false, kStore>(w, G, tf32, wst)))) return rc;
     M->launches++;
-    if (l == 0) break;
+    if (l == 0) {
+      if (!M->input_grad) break;
+      // D_0 = D_1 W_0, the gradient with respect to the input rows (no activation here)
+      a.M = b; a.N = din; a.K = dout;
+      a.A = Operand{scr + M->off_delta[1], S, dout, 0};
+      a.B = Operand{h->s + M->w_off[0], wstride, din, 1};
+      a.C = scr + M->off_delta[0];
+      a.c_group_stride = S;
+      a.ldc = din;
+      if ((rc = cuda_rc(launch_gemm<true, false, kStore>(a, G, tf32, st)))) return rc;
+      M->launches++;
+      break;
+    }
     // D_l = (D_{l+1} W_l) * [A_l > 0]: (m = r, k = o) from D, (k = o, n = j) from W_l [dout x din]
     a.M = b; a.N = din; a.K = dout;
     a.A = Operand{scr + M->off_delta[l + 1], S, dout, 0};
@@ -1031,6 +1018,93 @@ int mlp_chunk(gem_mlp* M, const int32_t* workers, int G, const int32_t* batch_ro
   return GEM_OK;
 }
 
+int mlp_build(gem_t* g, int n_layers, const int32_t* dims, int batch, int precision,
+              long long param_base, bool external_input, bool input_grad, bool own_grads,
+              gem_mlp** out) {
+  *out = nullptr;
+  gem_mlp* M = new (std::nothrow) gem_mlp();
+  if (!M) return GEM_ENOMEM;
+  M->gem = g;
+  M->L = n_layers;
+  M->batch = batch;
+  M->precision = precision;
+  M->param_base = param_base;
+  M->external_input = external_input;
+  M->input_grad = input_grad;
+  long long P = param_base;
+  for (int l = 0; l <= n_layers; ++l) M->dims[l] = dims[l];
+  for (int l = 0; l < n_layers; ++l) {
+    M->w_off[l] = P;
+    M->b_off[l] = P + (long long)dims[l + 1] * dims[l];
+    P = M->b_off[l] + dims[l + 1];
+  }
+  long long off = 0;
+  M->off_x = off;
+  off += round32((long long)batch * dims[0]);
+  for (int l = 1; l < n_layers; ++l) {
+    M->off_act[l] = off;
+    off += round32((long long)batch * dims[l]);
+  }
+  M->off_logits = off;
+  off += round32((long long)batch * dims[n_layers]);
+  for (int l = input_grad ? 0 : 1; l <= n_layers; ++l) {
+    M->off_delta[l] = off;
+    off += round32((long long)batch * dims[l]);
+  }
+  M->slot_stride = off;
+  M->slots = g->n < kMaxGroups ? g->n : kMaxGroups;
+  int dev_prev = 0;
+  cudaGetDevice(&dev_prev);
+  cudaSetDevice(g->device);
+  cudaError_t e = cudaMalloc(&M->scratch, sizeof(float) * size_t(M->slot_stride) * M->slots);
+  if (e == cudaSuccess && own_grads) e = cudaMalloc(&M->grads, sizeof(float) * g->stride * size_t(g->n));
+  if (e == cudaSuccess && batch <= 128) {
+    // split-K workspace: kMaxSplit partial products of at most batch x widest layer per slot
+    int widest = 0;
+    for (int l = input_grad ? 0 : 1; l <= n_layers; ++l) widest = dims[l] > widest ? dims[l] : widest;
+    M->ws_floats = (long long)kMaxSplit * 128 * widest * M->slots;
+    e = cudaMalloc(&M->ws, sizeof(float) * size_t(M->ws_floats));
+  }
+  if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&M->side, cudaStreamNonBlocking);
+  for (int l = 0; l <= n_layers && e == cudaSuccess; ++l)
+    e = cudaEventCreateWithFlags(&M->ev_delta[l], cudaEventDisableTiming);
+  if (e == cudaSuccess) e = cudaEventCreateWithFlags(&M->ev_side, cudaEventDisableTiming);
+  cudaSetDevice(dev_prev);
+  if (e != cudaSuccess) {
+    cudaGetLastError();
+    mlp_free(M);
+    return GEM_ENOMEM;
+  }
+  *out = M;
+  return GEM_OK;
+}
+
+void mlp_free(gem_mlp* M) {
+  if (!M) return;
+  int dev_prev = 0;
+  cudaGetDevice(&dev_prev);
+  cudaSetDevice(M->gem->device);
+  cudaStreamSynchronize(M->gem->stream);
+  if (M->side) cudaStreamSynchronize(M->side);
+  for (int l = 0; l <= kMaxLayers; ++l)
+    if (M->ev_delta[l]) cudaEventDestroy(M->ev_delta[l]);
+  if (M->ev_side) cudaEventDestroy(M->ev_side);
+  if (M->side) cudaStreamDestroy(M->side);
+  cudaFree(M->scratch);
+  cudaFree(M->grads);
+  cudaFree(M->ws);
+  cudaFree(M->pi_rows);
+  cudaFree(M->rows_dev);
+  cudaGetLastError();
+  cudaSetDevice(dev_prev);
+  delete M;
+}
+
+}  // namespace mlp
+}  // namespace gem
+
+namespace {
+
 // Check minibatch rows on the host and copy them to the device (stream-ordered).
 int upload_rows(gem_mlp* M, const int32_t* rows_host, long long count) {
   for (long long i = 0; i < count; ++i)
@@ -1065,90 +1139,12 @@ int gem_mlp_create(gem_t* g, int n_layers, const int32_t* dims, int batch, int p
   for (int l = 0; l <= n_layers; ++l)
     if (dims[l] < 1) return GEM_EINVAL;
   if (dims[n_layers] > kMaxClasses) return GEM_EINVAL;
-  gem_mlp* M = new (std::nothrow) gem_mlp();
-  if (!M) return GEM_ENOMEM;
-  M->gem = g;
-  M->L = n_layers;
-  M->batch = batch;
-  M->precision = precision;
-  for (int l = 0; l <= n_layers; ++l) M->dims[l] = dims[l];
-  for (int l = 0; l < n_layers; ++l) {
-    M->w_off[l] = P;
-    M->b_off[l] = P + (long long)dims[l + 1] * dims[l];
-    P = M->b_off[l] + dims[l + 1];
-  }
-  if ((size_t)P != g->P) {
-    delete M;
-    return GEM_EINVAL;
-  }
-  long long off = 0;
-  M->off_x = off;
-  off += round32((long long)batch * dims[0]);
-  for (int l = 1; l < n_layers; ++l) {
-    M->off_act[l] = off;
-    off += round32((long long)batch * dims[l]);
-  }
-  M->off_logits = off;
-  off += round32((long long)batch * dims[n_layers]);
-  for (int l = 1; l <= n_layers; ++l) {
-    M->off_delta[l] = off;
-    off += round32((long long)batch * dims[l]);
-  }
-  M->slot_stride = off;
-  M->slots = g->n < kMaxGroups ? g->n : kMaxGroups;
-  int dev_prev = 0;
-  cudaGetDevice(&dev_prev);
-  cudaSetDevice(g->device);
-  cudaError_t e = cudaMalloc(&M->scratch, sizeof(float) * size_t(M->slot_stride) * M->slots);
-  if (e == cudaSuccess) e = cudaMalloc(&M->grads, sizeof(float) * g->stride * size_t(g->n));
-  if (e == cudaSuccess && batch <= 128) {
-    // split-K workspace: kMaxSplit partial products of at most batch x widest layer per slot
-    int widest = 0;
-    for (int l = 1; l <= n_layers; ++l) widest = dims[l] > widest ? dims[l] : widest;
-    M->ws_floats = (long long)kMaxSplit * 128 * widest * M->slots;
-    e = cudaMalloc(&M->ws, sizeof(float) * size_t(M->ws_floats));
-  }
-  if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&M->side, cudaStreamNonBlocking);
-  for (int l = 0; l <= n_layers && e == cudaSuccess; ++l)
-    e = cudaEventCreateWithFlags(&M->ev_delta[l], cudaEventDisableTiming);
-  if (e == cudaSuccess) e = cudaEventCreateWithFlags(&M->ev_side, cudaEventDisableTiming);
-  cudaSetDevice(dev_prev);
-  if (e != cudaSuccess) {
-    cudaGetLastError();
-    cudaFree(M->scratch);
-    cudaFree(M->grads);
-    cudaFree(M->ws);
-    for (int l = 0; l <= kMaxLayers; ++l)
-      if (M->ev_delta[l]) cudaEventDestroy(M->ev_delta[l]);
-    if (M->ev_side) cudaEventDestroy(M->ev_side);
-    if (M->side) cudaStreamDestroy(M->side);
-    delete M;
-    return GEM_ENOMEM;
-  }
-  *out = M;
-  return GEM_OK;
+  for (int l = 0; l < n_layers; ++l) P += (long long)dims[l + 1] * dims[l] + dims[l + 1];
+  if ((size_t)P != g->P) return GEM_EINVAL;
+  return mlp_build(g, n_layers, dims, batch, precision, 0, false, false, true, out);
 }
 
-void gem_mlp_destroy(gem_mlp_t* M) {
-  if (!M) return;
-  int dev_prev = 0;
-  cudaGetDevice(&dev_prev);
-  cudaSetDevice(M->gem->device);
-  cudaStreamSynchronize(M->gem->stream);
-  if (M->side) cudaStreamSynchronize(M->side);
-  for (int l = 0; l <= kMaxLayers; ++l)
-    if (M->ev_delta[l]) cudaEventDestroy(M->ev_delta[l]);
-  if (M->ev_side) cudaEventDestroy(M->ev_side);
-  if (M->side) cudaStreamDestroy(M->side);
-  cudaFree(M->scratch);
-  cudaFree(M->grads);
-  cudaFree(M->ws);
-  cudaFree(M->pi_rows);
-  cudaFree(M->rows_dev);
-  cudaGetLastError();
-  cudaSetDevice(dev_prev);
-  delete M;
-}
+void gem_mlp_destroy(gem_mlp_t* M) { mlp_free(M); }
 
 int gem_mlp_set_data(gem_mlp_t* M, const float* X, const int32_t* labels, int64_t rows) {
   if (!M || !X || !labels || rows < 1) return GEM_EINVAL;

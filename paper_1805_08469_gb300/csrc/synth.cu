@@ -12,7 +12,8 @@ namespace {
 
 constexpr uint64_t kGamma = 0x9E3779B97F4A7C15ull;
 constexpr uint64_t kStreamTheta0 = 1, kStreamGradZ = 2, kStreamGradT = 3, kStreamMask = 4,
-                   kStreamDataX = 6, kStreamTeacher = 7, kStreamXavier = 8;
+                   kStreamDataX = 6, kStreamTeacher = 7, kStreamXavier = 8, kStreamDropout = 10,
+                   kStreamCnnInit = 11;
 constexpr uint64_t kHeavyThresholdU24 = 1677722;  // ceil(0.1 * 2^24)
 
 __host__ __device__ __forceinline__ uint64_t mix64(uint64_t z) {
@@ -113,6 +114,17 @@ __global__ void xavier_kernel(uint64_t key, size_t count, int fan_in, float a, f
   }
 }
 
+// Channel dropout scales: 0 where the 24-bit uniform of counter first + q is below p,
+// else keep.
+__global__ void dropout_kernel(uint64_t key, uint64_t first, size_t count, float p, float keep,
+                               float* out) {
+  for (size_t q = blockIdx.x * size_t(blockDim.x) + threadIdx.x; q < count;
+       q += size_t(gridDim.x) * blockDim.x) {
+    const float u = __fmul_rn(__uint2float_rn(unsigned(draw(key, first + q) >> 40)), 0x1p-24f);
+    out[q] = u < p ? 0.0f : keep;
+  }
+}
+
 int launched() { return cudaGetLastError() == cudaSuccess ? 0 : -3; }
 
 }  // namespace
@@ -172,6 +184,40 @@ int gem_synth_xavier(uint64_t seed, const int32_t* dims, int n_layers, float* th
       return -3;
     off += count + size_t(fo);
   }
+  return launched();
+}
+
+int gem_synth_cnn_theta0(uint64_t seed, const int32_t* shape, float* theta, void* stream) {
+  if (!shape || !theta) return -1;
+  const int H = shape[0], c1 = shape[1], c2 = shape[2], f1 = shape[3], f2 = shape[4],
+            C = shape[5];
+  if (H < 5 || c1 < 1 || c2 < 1 || f1 < 1 || f2 < 1 || C < 2 || (H - 4) % 2) return -1;
+  const int h2 = (H - 4) / 2 - 4;
+  if (h2 < 2 || h2 % 2) return -1;
+  const long long feat = (long long)c2 * (h2 / 2) * (h2 / 2);
+  const long long count[10] = {c1 * 25LL, c1, (long long)c2 * c1 * 25, c2, f1 * feat, f1,
+                               (long long)f2 * f1, f2, (long long)C * f2, C};
+  const long long fan_in[10] = {25, 25, c1 * 25LL, c1 * 25LL, feat, feat, f1, f1, f2, f2};
+  size_t off = 0;
+  for (int t = 0; t < 10; ++t) {
+    const float bound = float(1.0 / sqrt(double(fan_in[t])));
+    xavier_kernel<<<grid_for(size_t(count[t]), 256), 256, 0, cudaStream_t(stream)>>>(
+        stream_key(seed, kStreamCnnInit + 256ull * uint64_t(t)), size_t(count[t]), 0, bound,
+        theta + off);
+    off += size_t(count[t]);
+  }
+  return launched();
+}
+
+int gem_synth_dropout(uint64_t seed, uint64_t t0, int T, int b, int channels, float p,
+                      float* out, void* stream) {
+  if (!out || T < 0 || b < 1 || channels < 1 || !(p >= 0.0f && p < 1.0f)) return -1;
+  const size_t count = size_t(T) * size_t(b) * size_t(channels);
+  if (count == 0) return 0;
+  const float keep = float(1.0 / (1.0 - double(p)));
+  dropout_kernel<<<grid_for(count, 256), 256, 0, cudaStream_t(stream)>>>(
+      stream_key(seed, kStreamDropout), t0 * uint64_t(b) * uint64_t(channels), count, p, keep,
+      out);
   return launched();
 }
 

@@ -44,6 +44,8 @@ STREAM_DATA_X = 6
 STREAM_TEACHER = 7
 STREAM_XAVIER = 8  # + 256 * layer
 STREAM_BATCH = 9
+STREAM_DROPOUT = 10
+STREAM_CNN_INIT = 11  # + 256 * tensor
 
 # workload constants
 THETA0_SCALE = np.float32(0.05)
@@ -244,3 +246,58 @@ def schedule_batches(seed: int, order, b: int, n_rows: int = DATA_ROWS) -> np.nd
         seen[w] = k + 1
         out[t] = batch_indices(seed, w, k, b, n_rows)
     return out
+
+
+# ------------------------------------------------------------- the MNIST network
+
+# The convolutional network of the MNIST experiments (Appendix A): 28 x 28 inputs, conv 5x5
+# to 10 channels, conv 5x5 to 20 channels, fully connected 320 -> 128 -> 64 -> 10.
+CNN_MNIST = (28, 10, 20, 128, 64, 10)
+
+
+def cnn_layout(shape):
+    """[(name, offset, count, fan_in)] of the flat parameter vector: conv1.W, conv1.b,
+    conv2.W, conv2.b, fc1.W, fc1.b, fc2.W, fc2.b, fc3.W, fc3.b."""
+    H, c1, c2, f1, f2, C = shape
+    p2 = ((H - 4) // 2 - 4) // 2
+    feat = c2 * p2 * p2
+    tensors = [("conv1.W", c1 * 25, 25), ("conv1.b", c1, 25),
+               ("conv2.W", c2 * c1 * 25, c1 * 25), ("conv2.b", c2, c1 * 25),
+               ("fc1.W", f1 * feat, feat), ("fc1.b", f1, feat),
+               ("fc2.W", f2 * f1, f1), ("fc2.b", f2, f1),
+               ("fc3.W", C * f2, f2), ("fc3.b", C, f2)]
+    out, off = [], 0
+    for name, count, fan_in in tensors:
+        out.append((name, off, count, fan_in))
+        off += count
+    return out
+
+
+def cnn_param_count(shape) -> int:
+    name, off, count, _f = cnn_layout(shape)[-1]
+    return off + count
+
+
+def cnn_init_bound(fan_in: int) -> np.float32:
+    return np.float32(1.0 / np.sqrt(float(fan_in)))
+
+
+def cnn_theta0(seed: int, shape) -> np.ndarray:
+    """PyTorch's default initialisation of the network: every weight and bias uniform in
+    [-1/sqrt(fan_in), 1/sqrt(fan_in)), as bound * (2u - 1) with a 24-bit u, fp32."""
+    theta = np.empty(cnn_param_count(shape), dtype=np.float32)
+    for t, (_name, off, count, fan_in) in enumerate(cnn_layout(shape)):
+        u = u24(draw(key(seed, STREAM_CNN_INIT + 256 * t), np.arange(count, dtype=np.uint64)))
+        theta[off:off + count] = cnn_init_bound(fan_in) * (np.float32(2.0) * u - np.float32(1.0))
+    return theta
+
+
+def dropout_scales(seed: int, t0: int, T: int, b: int, channels: int, p: float = 0.5) -> np.ndarray:
+    """Channel dropout of commits t0 .. t0 + T - 1: scale [T, b, channels] is 0 where the
+    24-bit uniform of counter ((t b + i) channels + c) is below p, else 1 / (1 - p) (fp32)."""
+    c = ((np.arange(t0, t0 + T, dtype=np.uint64)[:, None, None] * _U64(b)
+          + np.arange(b, dtype=np.uint64)[None, :, None]) * _U64(channels)
+         + np.arange(channels, dtype=np.uint64)[None, None, :])
+    u = u24(draw(key(seed, STREAM_DROPOUT), c))
+    keep = np.float32(1.0 / (1.0 - p))
+    return np.where(u < np.float32(p), np.float32(0.0), keep).astype(np.float32)

@@ -53,3 +53,18 @@ def xavier(seed: int, dims, theta, stream=None):
     _check(lib().gem_synth_xavier(seed, d, len(dims) - 1, C.c_void_p(theta.data_ptr()),
                                   _stream(stream)), "gem_synth_xavier")
     return theta
+
+
+def cnn_theta0(seed: int, shape, theta, stream=None):
+    sh = (C.c_int32 * 6)(*shape)
+    _check(lib().gem_synth_cnn_theta0(seed, sh, C.c_void_p(theta.data_ptr()), _stream(stream)),
+           "gem_synth_cnn_theta0")
+    return theta
+
+
+def dropout(seed: int, t0: int, out, p: float = 0.5, stream=None):
+    """out: float32 CUDA tensor [T, b, channels]."""
+    T, b, ch = out.shape
+    _check(lib().gem_synth_dropout(seed, t0, T, b, ch, p, C.c_void_p(out.data_ptr()),
+                                   _stream(stream)), "gem_synth_dropout")
+    return out
