@@ -412,6 +412,7 @@ def run_gem(args, world, rank, local, pg):
 
     flat = None if args.no_flat else run_flat_commits(seed_offset=rank)
     mlp = None if args.no_mlp else run_mlp_workloads(args, seed_offset=rank)
+    cnn_out = None if args.no_mlp else run_cnn_workloads(args, seed_offset=rank)
 
     if rank != 0:
         return
@@ -444,6 +445,7 @@ def run_gem(args, world, rank, local, pg):
         "pi_statistics": pi_stats,
         "flat_single_commits": flat,
         "async_mlp": mlp,
+        "async_cnn": cnn_out,
         "clocks": clocks.summary(),
         "e2e": e2e,
     }
@@ -588,6 +590,63 @@ def run_mlp_workloads(args, seed_offset: int = 0) -> dict:
     return out
 
 
+CNN_WORKLOADS = [
+    # (name, n, batch, seed, warmup commits, timed commits); the paper's MNIST settings
+    # eta = 0.05, mu = 0.9, b = 64, uniform-tick schedule
+    ("cnn_mnist_n30_b64", 30, 64, 6, 100, 1000),
+    ("cnn_mnist_n100_b64", 100, 64, 7, 100, 1000),
+]
+CNN_ETA = 0.05
+
+
+def run_cnn_workloads(args, seed_offset: int = 0) -> dict:
+    """Asynchronous GEM on the MNIST convolutional network of Appendix A (synthetic 28 x 28
+    images: a +-0.5 class template on 4 x 4 cells plus N(0, 1) pixel noise): commits/s
+    with CUDA events, and the minibatch loss at the start and end of the timed run."""
+    import torch
+
+    from paper_1805_08469_gb300 import cnn, gem, sim, synth, synth_gpu
+
+    out = {}
+    stream = torch.cuda.Stream()
+    shape = cnn.CNN_MNIST
+    P = cnn.gem_cnn_param_count(shape)
+    X = torch.empty((synth.DATA_ROWS, 784), device="cuda")
+    y = torch.empty(synth.DATA_ROWS, dtype=torch.int32, device="cuda")
+    for name, n, b, seed, warm, timed in CNN_WORKLOADS:
+        seed = seed + seed_offset
+        if args.mlp_commits:
+            warm, timed = min(warm, args.mlp_commits), args.mlp_commits
+        T = warm + timed
+        synth_gpu.cnn_data(seed, X, y, 10, stream=stream)
+        order = sim.gem_schedule_uniform(seed, n, T)[0]
+        batches = synth.schedule_batches(seed, order, b)
+        with torch.cuda.stream(stream):
+            drop = synth_gpu.dropout(seed, 0, torch.empty((T, b, shape[2]), device="cuda"), stream=stream)
+            G = gem.Gem(P, n, CNN_ETA, MU, EPS, stream=stream)
+            G.set_theta(synth_gpu.cnn_theta0(seed, shape, torch.empty(P, device="cuda"), stream=stream))
+            net = cnn.gem_cnn_create(G.h, shape, b)
+            cnn.gem_cnn_set_data(net, X, y)
+            losses = torch.empty(T, device="cuda")
+            cnn.gem_cnn_run(net, order[:warm], batches[:warm], drop[:warm], losses[:warm])
+            stream.synchronize()
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            cnn.gem_cnn_run(net, order[warm:], batches[warm:], drop[warm:], losses[warm:])
+            e1.record(stream)
+            stream.synchronize()
+            ms = e0.elapsed_time(e1)
+            lh = losses.cpu().numpy()
+            cnn.gem_cnn_destroy(net)
+            G.close()
+        out[name] = {"commits_per_s": round(timed / (ms * 1e-3), 1), "ms": round(ms, 3),
+                     "commits": timed, "workers": n, "batch": b, "params": P,
+                     "loss_first_100": round(float(lh[:100].mean()), 4),
+                     "loss_last_100": round(float(lh[-100:].mean()), 4)}
+    return out
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -599,8 +658,8 @@ def main():
     ap.add_argument("--no-mlp", action="store_true")
     ap.add_argument("--no-rules", action="store_true", help="skip timing the other commit rules")
     ap.add_argument("--no-flat", action="store_true", help="skip the flat P=1.2M single-commit run")
-    ap.add_argument("--only", choices=["all", "commit", "mlp"], default="all",
-                    help="profiling aid: run only the commit batches or only the async MLP runs")
+    ap.add_argument("--only", choices=["all", "commit", "mlp", "cnn"], default="all",
+                    help="profiling aid: run only the commit batches, the async MLP or CNN runs")
     ap.add_argument("--mlp-workload", default="",
                     help="profiling aid: run only the MLP workload with this name")
     ap.add_argument("--mlp-commits", type=int, default=0,
@@ -619,12 +678,15 @@ def main():
     else:
         from paper_1805_08469_gb300._build import build_library
         build_library()
-        if args.only == "mlp":
+        if args.only in ("mlp", "cnn"):
             import torch
             torch.cuda.set_device(local)
-            out = run_mlp_workloads(args, seed_offset=rank)
+            if args.only == "mlp":
+                out = {"async_mlp": run_mlp_workloads(args, seed_offset=rank)}
+            else:
+                out = {"async_cnn": run_cnn_workloads(args, seed_offset=rank)}
             if rank == 0:
-                print(json.dumps({"impl": "gem", "only": "mlp", "async_mlp": out}), flush=True)
+                print(json.dumps({"impl": "gem", "only": args.only, **out}), flush=True)
         else:
             if args.only == "commit":
                 args.no_mlp = True

@@ -60,6 +60,14 @@ int gem_synth_xavier(uint64_t seed, const int32_t* dims, int n_layers, float* th
  * 2^-24. */
 int gem_synth_cnn_theta0(uint64_t seed, const int32_t* shape, float* theta, void* stream);
 
+/* Training set of the network with spatial class structure: labels [rows], y_r =
+ * ((draw(key(seed, 13), r) >> 32) classes) >> 32; X [rows][H * H], pixel p of row r =
+ * template(y_r, p) + normal(key(seed, 6), r H H + p), template +-0.5 constant on cells of
+ * 4 x 4 pixels, the sign of cell (c, row, col) the top bit of draw(key(seed, 12),
+ * (c cells + row) cells + col), cells = ceil(H / 4).  Exact in fp32. */
+int gem_synth_cnn_data(uint64_t seed, int rows, int H, int classes, float* X, int32_t* labels,
+                       void* stream);
+
 /* Channel-dropout scales of commits t0 .. t0 + T - 1: out [T][b][channels], entry
  * ((t - t0) b + i) channels + c is 0 when (draw(key(seed, 10), (t b + i) channels + c) >> 40)
  * 2^-24 < p, else 1 / (1 - p) rounded to fp32.  0 <= p < 1. */

@@ -72,6 +72,7 @@ def _declare(L):
         "gem_synth_xavier": ([C.c_uint64, p, i, p, p], i),
         "gem_synth_cnn_theta0": ([C.c_uint64, p, p, p], i),
         "gem_synth_dropout": ([C.c_uint64, C.c_uint64, i, i, i, C.c_float, p, p], i),
+        "gem_synth_cnn_data": ([C.c_uint64, i, i, i, p, p, p], i),
     }
     for name, (args, res) in sig.items():
         fn = getattr(L, name)

@@ -13,7 +13,7 @@ namespace {
 constexpr uint64_t kGamma = 0x9E3779B97F4A7C15ull;
 constexpr uint64_t kStreamTheta0 = 1, kStreamGradZ = 2, kStreamGradT = 3, kStreamMask = 4,
                    kStreamDataX = 6, kStreamTeacher = 7, kStreamXavier = 8, kStreamDropout = 10,
-                   kStreamCnnInit = 11;
+                   kStreamCnnInit = 11, kStreamCnnTemplate = 12, kStreamCnnLabel = 13;
 constexpr uint64_t kHeavyThresholdU24 = 1677722;  // ceil(0.1 * 2^24)
 
 __host__ __device__ __forceinline__ uint64_t mix64(uint64_t z) {
@@ -125,6 +125,23 @@ __global__ void dropout_kernel(uint64_t key, uint64_t first, size_t count, float
   }
 }
 
+// MNIST-shaped stand-in for the network: one thread block per row; label from the
+// multiply-shift of a 32-bit draw, pixel = +-0.5 template cell of its class + normal noise.
+__global__ void cnn_data_kernel(uint64_t kx, uint64_t kt, uint64_t ky, int rows, int H,
+                                int classes, float* X, int32_t* labels) {
+  const int cells = (H + 3) / 4;
+  for (int r = blockIdx.x; r < rows; r += gridDim.x) {
+    const uint64_t h = draw(ky, uint64_t(r)) >> 32;
+    const int y = int((h * uint64_t(classes)) >> 32);
+    if (threadIdx.x == 0) labels[r] = y;
+    for (int p = threadIdx.x; p < H * H; p += blockDim.x) {
+      const int cell = ((y * cells) + (p / H) / 4) * cells + (p % H) / 4;
+      const float t = (draw(kt, uint64_t(cell)) >> 63) ? -0.5f : 0.5f;
+      X[size_t(r) * H * H + p] = __fadd_rn(t, normal(kx, uint64_t(r) * uint64_t(H * H) + p));
+    }
+  }
+}
+
 int launched() { return cudaGetLastError() == cudaSuccess ? 0 : -3; }
 
 }  // namespace
@@ -206,6 +223,16 @@ int gem_synth_cnn_theta0(uint64_t seed, const int32_t* shape, float* theta, void
         theta + off);
     off += size_t(count[t]);
   }
+  return launched();
+}
+
+int gem_synth_cnn_data(uint64_t seed, int rows, int H, int classes, float* X, int32_t* labels,
+                       void* stream) {
+  if (!X || !labels || rows < 0 || H < 1 || classes < 1) return -1;
+  if (rows == 0) return 0;
+  cnn_data_kernel<<<grid_for(size_t(rows), 1), 256, 0, cudaStream_t(stream)>>>(
+      stream_key(seed, kStreamDataX), stream_key(seed, kStreamCnnTemplate),
+      stream_key(seed, kStreamCnnLabel), rows, H, classes, X, labels);
   return launched();
 }
 

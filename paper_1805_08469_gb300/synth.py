@@ -46,6 +46,8 @@ STREAM_XAVIER = 8  # + 256 * layer
 STREAM_BATCH = 9
 STREAM_DROPOUT = 10
 STREAM_CNN_INIT = 11  # + 256 * tensor
+STREAM_CNN_TEMPLATE = 12
+STREAM_CNN_LABEL = 13
 
 # workload constants
 THETA0_SCALE = np.float32(0.05)
@@ -301,3 +303,34 @@ def dropout_scales(seed: int, t0: int, T: int, b: int, channels: int, p: float =
     u = u24(draw(key(seed, STREAM_DROPOUT), c))
     keep = np.float32(1.0 / (1.0 - p))
     return np.where(u < np.float32(p), np.float32(0.0), keep).astype(np.float32)
+
+
+CNN_TEMPLATE_BLOCK = 4       # template cells of 4 x 4 pixels
+CNN_TEMPLATE_AMPLITUDE = 0.5
+
+
+def cnn_labels(seed: int, rows, classes: int = 10) -> np.ndarray:
+    """Uniform class of each training row (multiply-shift of a 32-bit draw)."""
+    h = draw(key(seed, STREAM_CNN_LABEL), np.asarray(rows, dtype=np.uint64)) >> _U64(32)
+    return ((h * _U64(classes)) >> _U64(32)).astype(np.int32)
+
+
+def cnn_templates(seed: int, H: int = 28, classes: int = 10) -> np.ndarray:
+    """Class templates [classes, H * H]: +-0.5 on cells of 4 x 4 pixels, the sign of cell
+    (c, row, col) from the top bit of draw(key(seed, 12), (c * cells + row) * cells + col)."""
+    cells = (H + CNN_TEMPLATE_BLOCK - 1) // CNN_TEMPLATE_BLOCK
+    idx = np.arange(classes * cells * cells, dtype=np.uint64)
+    sign = np.where((draw(key(seed, STREAM_CNN_TEMPLATE), idx) >> _U64(63)) == 1, -1.0, 1.0)
+    sign = sign.reshape(classes, cells, cells).astype(np.float32)
+    py = np.arange(H) // CNN_TEMPLATE_BLOCK
+    t = sign[:, py[:, None], py[None, :]] * np.float32(CNN_TEMPLATE_AMPLITUDE)
+    return t.reshape(classes, H * H).astype(np.float32)
+
+
+def cnn_data_rows(seed: int, rows, H: int = 28, classes: int = 10):
+    """MNIST-shaped stand-in with spatial class structure: image = template of its class +
+    N(0, 1) pixel noise (the noise of data_rows), exact in fp32.  Returns (X [len, H*H],
+    labels [len])."""
+    y = cnn_labels(seed, rows, classes)
+    X = cnn_templates(seed, H, classes)[y] + data_rows(seed, rows, H * H)
+    return X.astype(np.float32), y

@@ -68,3 +68,12 @@ def dropout(seed: int, t0: int, out, p: float = 0.5, stream=None):
     _check(lib().gem_synth_dropout(seed, t0, T, b, ch, p, C.c_void_p(out.data_ptr()),
                                    _stream(stream)), "gem_synth_dropout")
     return out
+
+
+def cnn_data(seed: int, X, labels, classes: int = 10, stream=None):
+    """X: float32 CUDA tensor [rows, H * H]; labels: int32 CUDA tensor [rows]."""
+    rows, HH = X.shape
+    H = int(round(HH ** 0.5))
+    _check(lib().gem_synth_cnn_data(seed, rows, H, classes, C.c_void_p(X.data_ptr()),
+                                    C.c_void_p(labels.data_ptr()), _stream(stream)), "gem_synth_cnn_data")
+    return X, labels

@@ -2,9 +2,20 @@
 
 The network's gradient at a worker's snapshot is fp32 on the GPU and double in the oracle
 (rounded once to fp32), so the bar is the MLP's: 1e-5 relative L2 per parameter tensor.
-The asynchronous runs are compared as the MLP's are: in windows resumed from the oracle's
-state, and free-running over a horizon.  The dropout scales and initial parameters come
-from the seeded generators, whose device and host twins must agree bit for bit.
+The asynchronous runs are compared commit by commit, each resumed from the oracle's
+state, and free-running over a horizon.
+
+One tensor gets a wider bar.  Max-pooling and ReLU take discrete decisions; where two
+values of a pooling window (or a ReLU input and zero) are within fp32 rounding of each
+other, the GPU's fp32 sums and the oracle's double sums can decide differently, and both
+are correct at fp32 accuracy.  The first layer has about 92,000 such decisions per
+gradient (64 samples x 10 channels x 144 windows); a flipped one moves one sample's
+contribution to conv1.W's gradient onto the neighbouring input patch, up to about 1% of
+that tensor (measured: 5.1e-3 on one of ten commits), while conv1.b, which sums the same
+routed values, stays within 1e-6.  conv1.W's gradient is therefore compared at 1e-2.  The
+same flips separate free-running trajectories (see the run test).  The dropout
+scales and initial parameters come from the seeded generators, whose device and host twins
+must agree bit for bit.
 """
 import numpy as np
 import pytest
@@ -15,7 +26,7 @@ from paper_1805_08469_gb300 import cnn, gem, synth, synth_gpu
 from paper_1805_08469_gb300._build import build_library
 from paper_1805_08469_gb300._lib import GemError
 
-from test_gpu_mlp import device_data, host_rows, rel_l2
+from test_gpu_mlp import rel_l2
 
 pytestmark = pytest.mark.gpu
 
@@ -38,6 +49,33 @@ def test_device_generators_match_host_generators():
     host = synth.dropout_scales(4, 17, 5, 64, 20)
     assert np.array_equal(dev.cpu().numpy(), host)
     assert 0.4 < (host == 0).mean() < 0.6 and set(np.unique(host)) == {0.0, 2.0}
+    for H in (28, 16):
+        X = torch.empty((2000, H * H), device="cuda")
+        y = torch.empty(2000, dtype=torch.int32, device="cuda")
+        synth_gpu.cnn_data(5, X, y)
+        hx, hy = synth.cnn_data_rows(5, np.arange(2000), H)
+        assert np.array_equal(X.cpu().numpy(), hx) and np.array_equal(y.cpu().numpy(), hy)
+    assert np.bincount(hy, minlength=10).min() > 150          # every class present
+
+
+_cnn_data_cache = {}
+
+
+def cnn_device_data(seed):
+    if seed not in _cnn_data_cache:
+        X = torch.empty((synth.DATA_ROWS, 784), device="cuda")
+        y = torch.empty(synth.DATA_ROWS, dtype=torch.int32, device="cuda")
+        synth_gpu.cnn_data(seed, X, y)
+        torch.cuda.synchronize()
+        _cnn_data_cache[seed] = (X, y)
+    return _cnn_data_cache[seed]
+
+
+def cnn_host_rows(seed, batch_rows):
+    """Rows that the oracle needs (host twin), with batch_rows remapped to them."""
+    rows, inv = np.unique(batch_rows, return_inverse=True)
+    X, y = synth.cnn_data_rows(seed, rows)
+    return X, y, inv.reshape(batch_rows.shape).astype(np.int32)
 
 
 def _blocks(shape):
@@ -54,8 +92,9 @@ def test_gradients_match_the_oracle(shape, b, G):
     P = synth.cnn_param_count(shape)
     H = shape[0]
     rows_total = 300
-    X = torch.from_numpy(synth.data_rows(seed, np.arange(rows_total), H * H)).cuda()
-    y = torch.from_numpy(synth.teacher_labels(seed, np.arange(rows_total), H * H, shape[5])).cuda()
+    Xh, yh = synth.cnn_data_rows(seed, np.arange(rows_total), H, shape[5])
+    X = torch.from_numpy(Xh).cuda()
+    y = torch.from_numpy(yh).cuda()
     theta0 = synth.cnn_theta0(seed, shape)
     rng = np.random.default_rng(3)
     snaps = np.stack([theta0 + (0.02 * rng.standard_normal(P)).astype(np.float32) for _ in range(G)])
@@ -76,8 +115,6 @@ def test_gradients_match_the_oracle(shape, b, G):
             got_loss = losses.cpu().numpy()
         finally:
             cnn.gem_cnn_destroy(net)
-    Xh = synth.data_rows(seed, np.arange(rows_total), H * H)
-    yh = synth.teacher_labels(seed, np.arange(rows_total), H * H, shape[5])
     blocks, _names = _blocks(shape)
     for g in range(G):
         loss, ref = oracle.cnn_loss_grad(shape, snaps[g].astype(np.float64), Xh[rows[g]], yh[rows[g]],
@@ -85,7 +122,7 @@ def test_gradients_match_the_oracle(shape, b, G):
         assert abs(got_loss[g] - loss) <= 1e-5 * abs(loss), (g, got_loss[g], loss)
         for nm, off, cnt in blocks:
             err = rel_l2(got[g, off:off + cnt], ref[off:off + cnt])
-            assert err < 1e-5, (g, nm, err)
+            assert err < (1e-2 if nm == "conv1.W" else 1e-5), (g, nm, err)
 
 
 def _cnn_inputs(shape, n, b, T, seed):
@@ -95,52 +132,57 @@ def _cnn_inputs(shape, n, b, T, seed):
     return order, tau, batches, drop
 
 
-def test_windows_and_free_run_match_the_oracle():
-    """The paper's network, n = 4 workers, b = 64, 60 uniform-tick commits (seed 1):
-    windows of 10 commits resumed from the oracle's state at commits 0, 20 and 40 within
-    1e-4, and the free-running first 30 commits within 1e-4."""
-    shape, n, b, seed, W = cnn.CNN_MNIST, 4, 64, 1, 10
-    starts = [0, 20, 40]
-    T = starts[-1] + W
+def test_every_commit_and_the_free_run_match_the_oracle():
+    """The paper's network, n = 4 workers, b = 64, 60 uniform-tick commits (seed 1).
+
+    Every commit, resumed from the oracle's state before it: each tensor of theta within
+    1e-5 after the commit (conv1.W within 1e-4: a flipped pooling decision changes its
+    gradient by up to ~1%, which a single commit scales by eta; measured 6e-6).
+
+    Free-running from theta_0 for 30 commits: the trajectories separate through those
+    flips, not through sensitivity to rounding (the oracle moves by 2e-8 at commit 30 for a
+    50-ulp change of theta_0): each flip adds ~1e-4 and the perturbed states meet more
+    near-ties (measured total relative L2 2.3e-4 at commit 10, 4.1e-3 at 30).  The bar is
+    1e-2 at commit 30, and the minibatch losses within 1%."""
+    shape, n, b, seed, T = cnn.CNN_MNIST, 4, 64, 1, 60
     P = synth.cnn_param_count(shape)
     order, _tau, batches, drop_host = _cnn_inputs(shape, n, b, T, seed)
     theta0 = synth.cnn_theta0(seed, shape)
-    Xh, yh, local = host_rows(seed, batches)
-    # oracle states at the window boundaries
+    Xh, yh, local = cnn_host_rows(seed, batches)
     th, m, s = theta0.copy(), np.zeros((n, P), np.float32), np.tile(theta0, (n, 1))
-    states, ref_losses, t = {}, np.empty(T), 0
-    for c in sorted(set(starts + [c + W for c in starts])):
-        if c > t:
-            _r, ls = oracle.cnn_sim_run(shape, th, m, s, order[t:c], Xh, yh, local[t:c], drop_host[t:c],
-                                        eta=ETA, mu=MU, eps=EPS, want_losses=True)
-            ref_losses[t:c] = ls
-        states[c] = (th.copy(), m.copy(), s.copy())
-        t = c
-    X, y = device_data(seed)
+    states, ref_losses = [(th.copy(), m.copy(), s.copy())], np.empty(T)
+    for t in range(T):
+        _r, ls = oracle.cnn_sim_run(shape, th, m, s, order[t:t + 1], Xh, yh, local[t:t + 1],
+                                    drop_host[t:t + 1], eta=ETA, mu=MU, eps=EPS, want_losses=True)
+        ref_losses[t] = ls[0]
+        states.append((th.copy(), m.copy(), s.copy()))
+    X, y = cnn_device_data(seed)
     drop = torch.from_numpy(drop_host).cuda()
     with gem.Gem(P, n, ETA, MU, EPS) as G:
         net = cnn.gem_cnn_create(G.h, shape, b)
         try:
             cnn.gem_cnn_set_data(net, X, y)
-            losses = torch.empty(W, device="cuda")
-            for c in starts:
-                gem.gem_load_state(G.h, *states[c])
-                cnn.gem_cnn_run(net, order[c:c + W], batches[c:c + W], drop[c:c + W], losses)
+            loss = torch.empty(1, device="cuda")
+            for t in range(T):
+                gem.gem_load_state(G.h, *states[t])
+                cnn.gem_cnn_run(net, order[t:t + 1], batches[t:t + 1], drop[t:t + 1], loss)
                 G.sync()
-                err = rel_l2(G.theta().cpu().numpy(), states[c + W][0])
-                assert err < 1e-4, (c, err)
-                np.testing.assert_allclose(losses.cpu().numpy(), ref_losses[c:c + W], rtol=1e-4)
+                got = G.theta().cpu().numpy()
+                for nm, off, cnt, _f in synth.cnn_layout(shape):
+                    err = rel_l2(got[off:off + cnt], states[t + 1][0][off:off + cnt])
+                    assert err < (1e-4 if nm == "conv1.W" else 1e-5), (t, nm, err)
+                assert abs(float(loss) - ref_losses[t]) <= 1e-5 * ref_losses[t], t
             # free-running from theta_0
             G.set_theta(torch.from_numpy(theta0).cuda())
-            cnn.gem_cnn_run(net, order[:30], batches[:30], drop[:30])
+            losses = torch.empty(30, device="cuda")
+            cnn.gem_cnn_run(net, order[:30], batches[:30], drop[:30], losses)
             G.sync()
             free = G.theta().cpu().numpy()
+            free_losses = losses.cpu().numpy()
         finally:
             cnn.gem_cnn_destroy(net)
-    th, m, s = theta0.copy(), np.zeros((n, P), np.float32), np.tile(theta0, (n, 1))
-    oracle.cnn_sim_run(shape, th, m, s, order[:30], Xh, yh, local[:30], drop_host[:30], eta=ETA, mu=MU,
-                       eps=EPS)
-    assert rel_l2(free, th) < 1e-4, rel_l2(free, th)
+    assert rel_l2(free, states[30][0]) < 1e-2, rel_l2(free, states[30][0])
+    np.testing.assert_allclose(free_losses, ref_losses[:30], rtol=1e-2)
 
 
 def test_argument_checks():
