@@ -617,7 +617,8 @@ def run_cnn_workloads(args, seed_offset: int = 0) -> dict:
         seed = seed + seed_offset
         if args.mlp_commits:
             warm, timed = min(warm, args.mlp_commits), args.mlp_commits
-        T = warm + timed
+        pi_commits = min(timed, 500)      # then per-tensor factor medians on further commits
+        T = warm + timed + pi_commits
         synth_gpu.cnn_data(seed, X, y, 10, stream=stream)
         order = sim.gem_schedule_uniform(seed, n, T)[0]
         batches = synth.schedule_batches(seed, order, b)
@@ -633,17 +634,30 @@ def run_cnn_workloads(args, seed_offset: int = 0) -> dict:
             e0 = torch.cuda.Event(enable_timing=True)
             e1 = torch.cuda.Event(enable_timing=True)
             e0.record(stream)
-            cnn.gem_cnn_run(net, order[warm:], batches[warm:], drop[warm:], losses[warm:])
+            w1 = warm + timed
+            cnn.gem_cnn_run(net, order[warm:w1], batches[warm:w1], drop[warm:w1], losses[warm:w1])
             e1.record(stream)
             stream.synchronize()
             ms = e0.elapsed_time(e1)
-            lh = losses.cpu().numpy()
+            lh = losses[:w1].cpu().numpy()
+            pi_lo = torch.empty((pi_commits, 10), device="cuda")
+            pi_hi = torch.empty((pi_commits, 10), device="cuda")
+            cnn.gem_cnn_run_pi(net, order[w1:w1 + 1], batches[w1:w1 + 1], drop[w1:w1 + 1], pi_lo[:1], pi_hi[:1])
+            e0.record(stream)   # the first call allocated the factor rows and select scratch
+            cnn.gem_cnn_run_pi(net, order[w1 + 1:], batches[w1 + 1:], drop[w1 + 1:], pi_lo[1:], pi_hi[1:])
+            e1.record(stream)
+            stream.synchronize()
+            ms_pi = e0.elapsed_time(e1)
+            med = pi_lo.cpu().numpy()[-100:].mean(axis=0)
             cnn.gem_cnn_destroy(net)
             G.close()
         out[name] = {"commits_per_s": round(timed / (ms * 1e-3), 1), "ms": round(ms, 3),
                      "commits": timed, "workers": n, "batch": b, "params": P,
                      "loss_first_100": round(float(lh[:100].mean()), 4),
-                     "loss_last_100": round(float(lh[-100:].mean()), 4)}
+                     "loss_last_100": round(float(lh[-100:].mean()), 4),
+                     "with_pi_medians": {"commits_per_s": round((pi_commits - 1) / (ms_pi * 1e-3), 1),
+                                         "commits": pi_commits - 1,
+                                         "median_pi_per_tensor_last_100": [round(float(v), 5) for v in med]}}
     return out
 
 

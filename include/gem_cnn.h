@@ -66,6 +66,15 @@ int gem_cnn_grad(gem_cnn_t* cnn, const int32_t* workers, int L, const int32_t* b
 int gem_cnn_run(gem_cnn_t* cnn, const int32_t* order, int T, const int32_t* batch_rows,
                 const float* drop, float* losses);
 
+/* gem_cnn_run that also follows the scaling factors, as the experiments section does for
+ * this network: for each commit t, the lower and upper medians (gem_pi_median) of the
+ * factors pi that the commit applied to each of the 10 tensors of the flat layout are
+ * written to pi_lo[t][10] and pi_hi[t][10] (device arrays of 10 T floats, tensors in
+ * layout order).  The commits are the same, bit for bit.  The first call allocates a
+ * factor buffer of n rows of the handle's stride and the select scratch. */
+int gem_cnn_run_pi(gem_cnn_t* cnn, const int32_t* order, int T, const int32_t* batch_rows,
+                   const float* drop, float* losses, float* pi_lo, float* pi_hi);
+
 /* Wait for the network's work; GEM_ECUDA if device work failed. */
 int gem_cnn_status(gem_cnn_t* cnn);
 

@@ -62,6 +62,7 @@ def _declare(L):
         "gem_cnn_set_data": ([p, p, p, C.c_int64], i),
         "gem_cnn_grad": ([p, p, i, p, p, p, p], i),
         "gem_cnn_run": ([p, p, i, p, p, p], i),
+        "gem_cnn_run_pi": ([p, p, i, p, p, p, p, p], i),
         "gem_cnn_status": ([p], i),
         "gem_cnn_launch_count": ([p], C.c_uint64),
         "gem_cnn_destroy": ([p], None),

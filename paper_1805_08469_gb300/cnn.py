@@ -64,6 +64,17 @@ def gem_cnn_run(net: int, order, batch_rows, drop, losses=None) -> None:
                             _opt_ptr(losses)), "gem_cnn_run")
 
 
+def gem_cnn_run_pi(net: int, order, batch_rows, drop, pi_lo, pi_hi, losses=None) -> None:
+    """gem_cnn_run with each commit's per-tensor factor medians in pi_lo, pi_hi (float32
+    CUDA tensors [T, 10])."""
+    o = np.ascontiguousarray(order, dtype=np.int32)
+    r = np.ascontiguousarray(batch_rows, dtype=np.int32)
+    if r.shape[0] != o.shape[0]:
+        raise ValueError("batch_rows must have one row per commit")
+    check(lib().gem_cnn_run_pi(C.c_void_p(net), _p(o), len(o), _p(r), C.c_void_p(drop.data_ptr()),
+                               _opt_ptr(losses), _opt_ptr(pi_lo), _opt_ptr(pi_hi)), "gem_cnn_run_pi")
+
+
 def gem_cnn_status(net: int) -> None:
     check(lib().gem_cnn_status(C.c_void_p(net)), "gem_cnn_status")
 

@@ -331,6 +331,7 @@ struct gem_cnn {
   float* grads = nullptr;        // [n][gem stride]
   int32_t* rows_dev = nullptr;   // minibatch rows uploaded from the host
   size_t rows_cap = 0;
+  float* pi_rows = nullptr;      // [n][gem stride] scaling factors of a segment's commits
   uint64_t launches = 0;
 };
 
@@ -473,6 +474,7 @@ void gem_cnn_destroy(gem_cnn_t* N) {
   cudaFree(N->scratch);
   cudaFree(N->grads);
   cudaFree(N->rows_dev);
+  cudaFree(N->pi_rows);
   cudaGetLastError();
   cudaSetDevice(dev_prev);
   gem::mlp::mlp_free(N->head);
@@ -526,13 +528,32 @@ int gem_cnn_grad(gem_cnn_t* N, const int32_t* workers, int L, const int32_t* bat
   return rc;
 }
 
-int gem_cnn_run(gem_cnn_t* N, const int32_t* order, int T, const int32_t* batch_rows,
-                const float* drop, float* losses) {
+}  // extern "C"
+
+namespace {
+
+// gem_cnn_run, with per-tensor factor medians when pi_lo is not null.
+int cnn_run(gem_cnn_t* N, const int32_t* order, int T, const int32_t* batch_rows,
+            const float* drop, float* losses, float* pi_lo, float* pi_hi) {
   if (!N || T < 0 || (T > 0 && (!order || !batch_rows || !drop))) return GEM_EINVAL;
   if (!N->X) return GEM_EINVAL;
   gem_t* h = N->gem;
   if (h->broken) return GEM_ESTATE;
   if (T == 0) return GEM_OK;
+  const bool want_pi = pi_lo != nullptr;
+  if (want_pi && !pi_hi) return GEM_EINVAL;
+  constexpr int kTensors = 10;
+  int64_t tensors[kTensors + 1];
+  {
+    const Shape& sh = N->sh;
+    const int64_t head = sh.head;
+    const int64_t t[kTensors + 1] = {0, sh.b1, sh.w2, sh.b2, head, head + (int64_t)sh.f1 * sh.F,
+                                     head + (int64_t)sh.f1 * sh.F + sh.f1,
+                                     head + (int64_t)sh.f1 * sh.F + sh.f1 + (int64_t)sh.f2 * sh.f1,
+                                     head + (int64_t)sh.f1 * sh.F + sh.f1 + (int64_t)sh.f2 * sh.f1 + sh.f2,
+                                     sh.P - sh.C, sh.P};
+    for (int i = 0; i <= kTensors; ++i) tensors[i] = t[i];
+  }
   std::vector<int32_t> seg(size_t(T) + 1);
   const int S = gem_plan_segments(order, T, h->n, seg.data());
   if (S < 0) return GEM_EINVAL;
@@ -540,7 +561,15 @@ int gem_cnn_run(gem_cnn_t* N, const int32_t* order, int T, const int32_t* batch_
   cudaGetDevice(&dev_prev);
   cudaSetDevice(h->device);
   int rc = upload_rows(N, batch_rows, (long long)T * N->batch);
+  if (rc == GEM_OK && want_pi && !N->pi_rows) {
+    if (cudaMalloc(&N->pi_rows, sizeof(float) * h->stride * size_t(h->n)) != cudaSuccess) {
+      cudaGetLastError();
+      N->pi_rows = nullptr;
+      rc = GEM_ENOMEM;
+    }
+  }
   std::vector<const float*> gptr(static_cast<size_t>(T));
+  std::vector<float*> pptr(want_pi ? static_cast<size_t>(T) : 1, nullptr);
   const long long db = (long long)N->batch * N->sh.c2;
   for (int i = 0; i < S && rc == GEM_OK; ++i) {
     const int a = seg[i], e = seg[i + 1];
@@ -551,13 +580,38 @@ int gem_cnn_run(gem_cnn_t* N, const int32_t* order, int T, const int32_t* batch_
                      losses ? losses + c0 : nullptr);
     }
     if (rc == GEM_OK) {
-      for (int k = a; k < e; ++k) gptr[size_t(k)] = N->grads + (long long)(k - a) * h->stride;
-      rc = cuda_rc(gem::commit_ordered(h, order + a, gptr.data() + a, e - a));
+      for (int k = a; k < e; ++k) {
+        gptr[size_t(k)] = N->grads + (long long)(k - a) * h->stride;
+        if (want_pi) pptr[size_t(k)] = N->pi_rows + (long long)(k - a) * h->stride;
+      }
+      rc = cuda_rc(gem::commit_ordered(h, order + a, gptr.data() + a, e - a,
+                                       want_pi ? pptr.data() + a : nullptr));
+    }
+    if (rc == GEM_OK && want_pi) {
+      const cudaError_t ce = gem::pi_median_ordered(h, pptr.data() + a, e - a, tensors, kTensors,
+                                                     pi_lo + (long long)a * kTensors,
+                                                     pi_hi + (long long)a * kTensors);
+      rc = ce == cudaErrorMemoryAllocation ? GEM_ENOMEM : cuda_rc(ce);
     }
   }
   if (rc == GEM_ECUDA) h->broken = true;
   cudaSetDevice(dev_prev);
   return rc;
+}
+
+}  // namespace
+
+extern "C" {
+
+int gem_cnn_run(gem_cnn_t* N, const int32_t* order, int T, const int32_t* batch_rows,
+                const float* drop, float* losses) {
+  return cnn_run(N, order, T, batch_rows, drop, losses, nullptr, nullptr);
+}
+
+int gem_cnn_run_pi(gem_cnn_t* N, const int32_t* order, int T, const int32_t* batch_rows,
+                   const float* drop, float* losses, float* pi_lo, float* pi_hi) {
+  if (!pi_lo || !pi_hi) return GEM_EINVAL;
+  return cnn_run(N, order, T, batch_rows, drop, losses, pi_lo, pi_hi);
 }
 
 }  // extern "C"

@@ -209,3 +209,53 @@ def test_argument_checks():
             assert cnn.gem_cnn_launch_count(net) > 0
         finally:
             cnn.gem_cnn_destroy(net)
+
+
+def test_run_pi_equals_the_flat_calls_bitwise():
+    """gem_cnn_run_pi against the same segments replayed through gem_cnn_grad,
+    gem_commit_batch_pi and gem_pi_median over the 10 tensors: identical medians and
+    theta, bit for bit."""
+    from paper_1805_08469_gb300 import sim
+    shape, n, b, seed, T = cnn.CNN_MNIST, 6, 64, 2, 24
+    P = synth.cnn_param_count(shape)
+    order, _tau, batches, drop_host = _cnn_inputs(shape, n, b, T, seed)
+    theta0 = synth.cnn_theta0(seed, shape)
+    X, y = cnn_device_data(seed)
+    drop = torch.from_numpy(drop_host).cuda()
+    tensors = [off for _nm, off, _c, _f in synth.cnn_layout(shape)] + [P]
+    lo_a = torch.empty((T, 10), device="cuda")
+    hi_a = torch.empty((T, 10), device="cuda")
+    with gem.Gem(P, n, ETA, MU, EPS) as A:
+        A.set_theta(torch.from_numpy(theta0).cuda())
+        net = cnn.gem_cnn_create(A.h, shape, b)
+        try:
+            cnn.gem_cnn_set_data(net, X, y)
+            cnn.gem_cnn_run_pi(net, order, batches, drop, lo_a, hi_a)
+            A.sync()
+            theta_a = A.theta().clone()
+        finally:
+            cnn.gem_cnn_destroy(net)
+    segs = sim.gem_plan_segments(order, n)
+    lo_b = torch.empty((T, 10), device="cuda")
+    hi_b = torch.empty((T, 10), device="cuda")
+    ld = (P + 3) // 4 * 4
+    grads = torch.empty((n, ld), device="cuda")
+    pis = torch.empty((n, ld), device="cuda")
+    with gem.Gem(P, n, ETA, MU, EPS) as B:
+        B.set_theta(torch.from_numpy(theta0).cuda())
+        net = cnn.gem_cnn_create(B.h, shape, b)
+        try:
+            cnn.gem_cnn_set_data(net, X, y)
+            for a, e in zip(segs[:-1], segs[1:]):
+                k = e - a
+                cnn.gem_cnn_grad(net, order[a:e], batches[a:e], drop[a:e], [grads[i, :P] for i in range(k)])
+                B.commit_batch_pi(order[a:e].tolist(), [grads[i, :P] for i in range(k)],
+                                  [pis[i, :P] for i in range(k)])
+                B.pi_median([pis[i, :P] for i in range(k)], tensors, lo_b[a:e], hi_b[a:e])
+            B.sync()
+            theta_b = B.theta().clone()
+        finally:
+            cnn.gem_cnn_destroy(net)
+    assert torch.equal(theta_a, theta_b)
+    assert torch.equal(lo_a, lo_b) and torch.equal(hi_a, hi_b)
+    assert float(lo_a.max()) > 0
