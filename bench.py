@@ -48,8 +48,8 @@ FALLBACK_HBM_GBS = 6800.0
 # DRAM traffic of one launch of the batched commit kernel, from an ncu capture of the
 # same workload (see profiles/commit_batch_p25m_n100.md).  Valid only for the kernel
 # source it was taken on; reported as null once that source changes.
-NCU_TRAFFIC_BYTES_PER_LAUNCH = 44_737_829_120   # mean of two full-size launches
-NCU_TRAFFIC_SOURCE_SHA = "afc2bd2d841409cd"
+NCU_TRAFFIC_BYTES_PER_LAUNCH = 40_834_115_456   # mean of two full-size launches
+NCU_TRAFFIC_SOURCE_SHA = "12a1f2beda7488bc"
 
 
 def kernel_source_sha() -> str:

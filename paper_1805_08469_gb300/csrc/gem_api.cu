@@ -127,6 +127,7 @@ cudaError_t commit_ordered(gem_ctx* h, const int* order, const float* const* gra
       // adaptive staleness: pi = 1 / (tau + 1) in fp32 (IEEE division); DOWNPOUR: pi = 1
       a.pi[k] = h->mode == GEM_MODE_ADAPTIVE ? 1.0f / (static_cast<float>(tau) + 1.0f) : 1.0f;
     }
+    plan_slots(a);
     const cudaError_t e = launch_commit_batch(a, h->sm_count, h->stream);
     if (e != cudaSuccess) return e;
     h->launches += 1;

@@ -35,6 +35,10 @@
 #ifndef GEM_COMMIT_STREAM_STATE
 #define GEM_COMMIT_STREAM_STATE 0
 #endif
+// Resident blocks per SM used to size the grid, at most (0: as many as fit).
+#ifndef GEM_COMMIT_MAX_BLOCKS_PER_SM
+#define GEM_COMMIT_MAX_BLOCKS_PER_SM 0
+#endif
 
 namespace gem {
 namespace {
@@ -112,13 +116,23 @@ __device__ __forceinline__ void commit_vec_fixed(float4& th, float4& s, const fl
 // 40 registers for three blocks and spills, which costs about 4% of its bandwidth.
 // REC: the commits whose pi_out[k] is set also store their scaling factors there (4 more
 // bytes per coordinate).
+// A worker that commits again later in the launch can keep its m_w, s_w lanes on chip:
+// each thread owns lanes slot_mem[(2 slot + {0: m, 1: s}) L kThreads + l kThreads + tid]
+// of dynamic shared memory, so no synchronisation is needed.
 template <int L, int RULE, bool REC>
 __global__ void __launch_bounds__(kThreads, RULE == kRuleScaled ? 2 : GEM_COMMIT_MIN_BLOCKS)
 commit_batch_kernel(const __grid_constant__ BatchArgs a) {
+  extern __shared__ float4 slot_mem[];
   const size_t nvec = a.P >> 2;
   const size_t nthreads = size_t(gridDim.x) * kThreads;
   const size_t tid = size_t(blockIdx.x) * kThreads + threadIdx.x;
   float4* theta4 = reinterpret_cast<float4*>(a.theta);
+  auto slot_m = [&](int slot, int l) -> float4& {
+    return slot_mem[(2 * slot) * L * kThreads + l * kThreads + threadIdx.x];
+  };
+  auto slot_s = [&](int slot, int l) -> float4& {
+    return slot_mem[(2 * slot + 1) * L * kThreads + l * kThreads + threadIdx.x];
+  };
 
   for (size_t base = tid; base < nvec; base += nthreads * L) {
     float4 th[L];
@@ -132,6 +146,7 @@ commit_batch_kernel(const __grid_constant__ BatchArgs a) {
       const size_t row = size_t(a.worker[k]) * a.stride;
       float4* m4 = reinterpret_cast<float4*>(a.m + row);
       float4* s4 = reinterpret_cast<float4*>(a.s + row);
+      const int sin = a.slot_in[k], sout = a.slot_out[k];
       float4 g[L], m[L], s[L];
 #pragma unroll
       for (int l = 0; l < L; ++l) {
@@ -139,8 +154,13 @@ commit_batch_kernel(const __grid_constant__ BatchArgs a) {
         if (i < nvec) {
           g[l] = __ldcs(g4 + i);
           if (RULE != kRuleFixed) {
-            m[l] = load_state(m4 + i);
-            s[l] = load_state(s4 + i);
+            if (sin >= 0) {
+              m[l] = slot_m(sin, l);
+              s[l] = slot_s(sin, l);
+            } else {
+              m[l] = load_state(m4 + i);
+              s[l] = load_state(s4 + i);
+            }
           }
         }
       }
@@ -152,11 +172,17 @@ commit_batch_kernel(const __grid_constant__ BatchArgs a) {
           if (RULE == kRuleFixed) {
             commit_vec_fixed(th[l], s[l], g[l], a.eta, a.pi[k]);
             pi = make_float4(a.pi[k], a.pi[k], a.pi[k], a.pi[k]);
+            if (a.keep_s[k]) store_state(s4 + i, s[l]);
           } else {
             pi = commit_vec<RULE>(th[l], m[l], s[l], g[l], a.eta, a.mu, a.eps, a.energy_scale);
-            store_state(m4 + i, m[l]);
+            if (sout >= 0) {
+              slot_m(sout, l) = m[l];
+              slot_s(sout, l) = s[l];
+            } else {
+              store_state(m4 + i, m[l]);
+              store_state(s4 + i, s[l]);
+            }
           }
-          store_state(s4 + i, s[l]);
           if (REC && a.pi_out[k]) reinterpret_cast<float4*>(a.pi_out[k])[i] = pi;
         }
       }
@@ -197,11 +223,19 @@ constexpr int kLanes = GEM_COMMIT_LANES;
 
 template <int RULE, bool REC>
 cudaError_t launch_rule(const BatchArgs& a, int sm_count, cudaStream_t stream) {
+  constexpr int smem = RULE == kRuleFixed ? 0 : kCommitSlots * 2 * kLanes * kThreads * 16;
   static int blocks_per_sm = 0;
   if (blocks_per_sm == 0) {
+    if (smem > 48 * 1024) {
+      cudaError_t e = cudaFuncSetAttribute(commit_batch_kernel<kLanes, RULE, REC>,
+                                           cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+      if (e != cudaSuccess) return e;
+    }
     cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(
-        &blocks_per_sm, commit_batch_kernel<kLanes, RULE, REC>, kThreads, 0);
+        &blocks_per_sm, commit_batch_kernel<kLanes, RULE, REC>, kThreads, smem);
     if (e != cudaSuccess) return e;
+    if (GEM_COMMIT_MAX_BLOCKS_PER_SM > 0 && blocks_per_sm > GEM_COMMIT_MAX_BLOCKS_PER_SM)
+      blocks_per_sm = GEM_COMMIT_MAX_BLOCKS_PER_SM;
     if (blocks_per_sm < 1) blocks_per_sm = 1;
   }
   const size_t nvec = a.P >> 2;
@@ -215,11 +249,64 @@ cudaError_t launch_rule(const BatchArgs& a, int sm_count, cudaStream_t stream) {
     grid = (nvec + rounds * per_block - 1) / (rounds * per_block);
   }
   if (grid < 1) grid = 1;
-  commit_batch_kernel<kLanes, RULE, REC><<<unsigned(grid), kThreads, 0, stream>>>(a);
+  commit_batch_kernel<kLanes, RULE, REC><<<unsigned(grid), kThreads, smem, stream>>>(a);
   return cudaGetLastError();
 }
 
 }  // namespace
+
+void plan_slots(BatchArgs& a) {
+  // next occurrence of each commit's worker within the launch
+  int next[kMaxBatchPerLaunch];
+  {
+    int last_seen[kMaxBatchPerLaunch];   // commit index per distinct worker, via search
+    int seen_worker[kMaxBatchPerLaunch];
+    int n_seen = 0;
+    for (int k = a.K - 1; k >= 0; --k) {
+      next[k] = -1;
+      for (int q = 0; q < n_seen; ++q)
+        if (seen_worker[q] == a.worker[k]) {
+          next[k] = last_seen[q];
+          last_seen[q] = k;
+          goto found;
+        }
+      seen_worker[n_seen] = a.worker[k];
+      last_seen[n_seen] = k;
+      ++n_seen;
+    found:;
+    }
+  }
+  for (int k = 0; k < a.K; ++k) {
+    a.slot_in[k] = -1;
+    a.slot_out[k] = -1;
+    a.keep_s[k] = next[k] < 0 ? 1 : 0;
+  }
+  if (a.rule == kRuleFixed || kCommitSlots == 0) return;
+  // Choose repeat intervals (k, next[k]) longer than kSlotMinDistance, at most kCommitSlots
+  // open at a time, as many as possible: by increasing end, each into the free slot that
+  // became free last (greedy, optimal for interval graphs).
+  int order[kMaxBatchPerLaunch], cnt = 0;
+  for (int k = 0; k < a.K; ++k)
+    if (next[k] >= 0 && next[k] - k > kSlotMinDistance) order[cnt++] = k;
+  for (int x = 1; x < cnt; ++x)   // insertion sort by end point
+    for (int y = x; y > 0 && next[order[y - 1]] > next[order[y]]; --y) {
+      const int t = order[y];
+      order[y] = order[y - 1];
+      order[y - 1] = t;
+    }
+  int free_at[kCommitSlots > 0 ? kCommitSlots : 1];
+  for (int q = 0; q < kCommitSlots; ++q) free_at[q] = -1;
+  for (int x = 0; x < cnt; ++x) {
+    const int k = order[x], e = next[k];
+    int best = -1;
+    for (int q = 0; q < kCommitSlots; ++q)
+      if (free_at[q] <= k && (best < 0 || free_at[q] > free_at[best])) best = q;
+    if (best < 0) continue;
+    free_at[best] = e;
+    a.slot_out[k] = int8_t(best);
+    a.slot_in[e] = int8_t(best);
+  }
+}
 
 cudaError_t launch_commit_batch(const BatchArgs& a, int sm_count, cudaStream_t stream) {
   if (a.record_pi) {

@@ -44,7 +44,29 @@ struct BatchArgs {
   float pi[kMaxBatchPerLaunch];            // kRuleFixed: scaling factor of commit k
   int record_pi;                           // 1: pi_out[k] (when not null) receives pi
   float* pi_out[kMaxBatchPerLaunch];       // scaling factors of commit k, P floats, or null
+  // On-chip reuse of a worker that commits again later in the launch (energy rules):
+  // commit k keeps its m_w, s_w lanes in shared-memory slot slot_out[k] instead of writing
+  // them to global memory, and the worker's next commit reads them from slot_in[k];
+  // -1 means global memory.  Fixed-factor rules: keep_s[k] = 0 skips the store of s_w
+  // when the worker commits again in the launch (nothing reads it before that).
+  int8_t slot_in[kMaxBatchPerLaunch];
+  int8_t slot_out[kMaxBatchPerLaunch];
+  uint8_t keep_s[kMaxBatchPerLaunch];
 };
+
+// Shared-memory slots of the commit kernel (m_w and s_w lanes of one worker per slot), and
+// the shortest repeat distance (in commits) given a slot: shorter repeats are served by L2.
+#ifndef GEM_COMMIT_SLOTS
+#define GEM_COMMIT_SLOTS 6
+#endif
+#ifndef GEM_COMMIT_SLOT_MIN_DISTANCE
+#define GEM_COMMIT_SLOT_MIN_DISTANCE 4
+#endif
+constexpr int kCommitSlots = GEM_COMMIT_SLOTS;
+constexpr int kSlotMinDistance = GEM_COMMIT_SLOT_MIN_DISTANCE;
+
+// Fill slot_in, slot_out and keep_s of a launch from its a.K workers.
+void plan_slots(BatchArgs& a);
 
 // Launch the fused commit kernel for a.K commits on `stream`.
 cudaError_t launch_commit_batch(const BatchArgs& a, int sm_count, cudaStream_t stream);
