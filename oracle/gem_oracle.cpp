@@ -34,6 +34,7 @@ enum Mode : int {
   MODE_ADAPTIVE = 2,       // commit dtheta / (tau + 1)
   MODE_KAPPA_SQRT = 3,     // App. B, Eq. pi_with_kappa: sqrt(kappa) |m|
   MODE_KAPPA_LINEAR = 4,   // App. B, the modified form used in that study: kappa |m|
+  MODE_MOMENTUM = 5,       // the proxy itself, Eq. momentum_update: theta += (m <- mu m + dtheta)
 };
 
 // One worker's commit on one coordinate (Algorithm 1, procedures Worker and Psi_GEM,
@@ -48,6 +49,14 @@ inline T commit_coordinate(T& theta, T& m, T& s, T g, T eta, T mu, T eps, int mo
   // theta <- Pull(): the value of the central variable the commit is applied to.
   const T theta_pulled = theta;
   T pi;
+  if (mode == MODE_MOMENTUM) {
+    // The target dynamics of the proxy (sequential momentum SGD with the worker's moment):
+    // the commit adds the moment itself; no scaling factor is formed (NaN is recorded).
+    m = mu * m + dtheta;
+    theta = theta_pulled + m;
+    s = precommit_snapshot ? theta_pulled : theta;
+    return T(NAN);
+  }
   if (mode == MODE_DOWNPOUR) {
     pi = T(1);
   } else if (mode == MODE_ADAPTIVE) {

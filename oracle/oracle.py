@@ -12,6 +12,7 @@ MODE_DOWNPOUR = 1
 MODE_ADAPTIVE = 2
 MODE_KAPPA_SQRT = 3
 MODE_KAPPA_LINEAR = 4
+MODE_MOMENTUM = 5
 
 _lib = None
 

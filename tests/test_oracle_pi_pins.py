@@ -157,3 +157,33 @@ def test_mlp_simulator_records_the_factors_of_its_commits():
                          record_pi=True)
     assert np.array_equal(pi[0], ref[0])
     assert pi.shape == (4, P) and np.all(pi >= 0)
+
+
+def test_momentum_proxy_rule_closed_form_and_identities():
+    """The proxy rule (Eq. momentum_update committed as is): with one worker and a constant
+    gradient g, theta_t = theta_0 - eta g sum_{k=1..t} (1 - mu^k) / (1 - mu); with mu = 0 it
+    is DOWNPOUR bit for bit; with one worker it is the textbook recursion v <- mu v - eta g,
+    theta <- theta + v."""
+    P, T, eta, mu = 50, 25, 0.05, 0.9
+    rng = np.random.default_rng(2)
+    theta0 = rng.standard_normal(P)
+    g = rng.standard_normal(P)
+    th, m, s = _fresh(theta0, 1)
+    oracle.gem_run(th, m, s, np.tile(g, (T, 1)), [0] * T, eta=eta, mu=mu, eps=1e-8,
+                   mode=oracle.MODE_MOMENTUM)
+    want = theta0 - eta * g * sum((1 - mu ** k) / (1 - mu) for k in range(1, T + 1))
+    np.testing.assert_allclose(th, want, rtol=1e-12, atol=1e-12)
+    theta0, grads, order, _tau = _rand(64, 3, 40, 4, np.float32)
+    a = _fresh(theta0, 3)
+    b = _fresh(theta0, 3)
+    oracle.gem_run(*a, grads, order, eta=0.01, mu=0.0, eps=1e-8, mode=oracle.MODE_MOMENTUM)
+    oracle.gem_run(*b, grads, order, eta=0.01, mu=0.0, eps=1e-8, mode=oracle.MODE_DOWNPOUR)
+    assert np.array_equal(a[0], b[0]) and np.array_equal(a[2], b[2])
+    theta0, grads, _o, _t = _rand(32, 1, 30, 6, np.float64)
+    th, m, s = _fresh(theta0, 1)
+    oracle.gem_run(th, m, s, grads, [0] * 30, eta=0.02, mu=0.8, eps=1e-8, mode=oracle.MODE_MOMENTUM)
+    v, ref = np.zeros(32), theta0.copy()
+    for t in range(30):
+        v = 0.8 * v - 0.02 * grads[t]
+        ref = ref + v
+    np.testing.assert_allclose(th, ref, rtol=1e-13, atol=1e-15)
