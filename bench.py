@@ -40,8 +40,9 @@ SEED = 5
 ETA, MU, EPS = 0.01, 0.9, 1e-8
 # the other commit rules (gem_mode values of include/gem.h) and kappa; bytes per parameter
 # and commit moved by each rule (theta adds 8 per batch for all)
-RULES = [("downpour", 1, 1.0), ("adaptive", 2, 1.0), ("kappa_sqrt_2", 3, 2.0), ("kappa_linear_2", 4, 2.0)]
-RULE_BYTES = {0: 20, 1: 8, 2: 8, 3: 20, 4: 20}
+RULES = [("downpour", 1, 1.0), ("adaptive", 2, 1.0), ("kappa_sqrt_2", 3, 2.0), ("kappa_linear_2", 4, 2.0),
+         ("momentum_proxy", 5, 1.0)]
+RULE_BYTES = {0: 20, 1: 8, 2: 8, 3: 20, 4: 20, 5: 16}
 BYTES_PER_BATCH = P_FULL * (20 * K_BATCH + 8)
 FALLBACK_HBM_GBS = 6800.0
 

@@ -143,13 +143,18 @@ int gem_shape(const gem_t* h, size_t* P, int* n, size_t* stride);
  *   GEM_MODE_KAPPA_SQRT    App. B, Eq. pi_with_kappa: as GEM with |m_w| replaced by
  *                          sqrt(kappa) * |m_w| (sqrt(kappa) rounded to fp32 first).
  *   GEM_MODE_KAPPA_LINEAR  App. B, the modified form used in its study: as GEM with |m_w|
- *                          replaced by kappa * |m_w|. */
+ *                          replaced by kappa * |m_w|.
+ *   GEM_MODE_MOMENTUM      the proxy itself, as a reference run (Eq. momentum_update):
+ *                          m_w = mu * m_w + dtheta, theta = theta + m_w, s_w = theta; no
+ *                          scaling factor is formed (gem_commit_batch_pi records NaN).  With
+ *                          one worker this is sequential momentum SGD. */
 enum gem_mode {
   GEM_MODE_GEM = 0,
   GEM_MODE_DOWNPOUR = 1,
   GEM_MODE_ADAPTIVE = 2,
   GEM_MODE_KAPPA_SQRT = 3,
-  GEM_MODE_KAPPA_LINEAR = 4
+  GEM_MODE_KAPPA_LINEAR = 4,
+  GEM_MODE_MOMENTUM = 5
 };
 
 /* Select the rule of every later commit.  kappa is the proxy's energy factor: required

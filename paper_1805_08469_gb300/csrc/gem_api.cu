@@ -104,6 +104,9 @@ cudaError_t commit_ordered(gem_ctx* h, const int* order, const float* const* gra
     case GEM_MODE_ADAPTIVE:
       a.rule = kRuleFixed;
       break;
+    case GEM_MODE_MOMENTUM:
+      a.rule = kRuleMomentum;
+      break;
     default:
       a.rule = kRuleGem;
       break;
@@ -250,7 +253,7 @@ int gem_set_theta(gem_t* h, const float* theta0) {
 int gem_set_mode(gem_t* h, int mode, float kappa) {
   int rc = check_handle(h);
   if (rc) return rc;
-  if (mode < GEM_MODE_GEM || mode > GEM_MODE_KAPPA_LINEAR) return GEM_EINVAL;
+  if (mode < GEM_MODE_GEM || mode > GEM_MODE_MOMENTUM) return GEM_EINVAL;
   if ((mode == GEM_MODE_KAPPA_SQRT || mode == GEM_MODE_KAPPA_LINEAR) &&
       !(kappa > 0.0f && kappa <= 3.0e38f))
     return GEM_EINVAL;

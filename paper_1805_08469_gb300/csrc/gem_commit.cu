@@ -90,6 +90,16 @@ __device__ __forceinline__ void store_state(float4* p, float4 v) {
 #endif
 }
 
+// The momentum-SGD proxy committed as is (Eq. momentum_update): m <- mu m + dtheta,
+// theta <- theta + m, s <- theta.
+__device__ __forceinline__ void commit_coord_momentum(float& theta, float& m, float& s, float g,
+                                                      float eta, float mu) {
+  const float dtheta = -__fmul_rn(eta, g);
+  m = __fadd_rn(__fmul_rn(mu, m), dtheta);
+  theta = __fadd_rn(theta, m);
+  s = theta;
+}
+
 template <int RULE>
 __device__ __forceinline__ float4 commit_vec(float4& th, float4& m, float4& s, const float4 g,
                                              float eta, float mu, float eps, float scale) {
@@ -153,7 +163,9 @@ commit_batch_kernel(const __grid_constant__ BatchArgs a) {
         const size_t i = base + size_t(l) * nthreads;
         if (i < nvec) {
           g[l] = __ldcs(g4 + i);
-          if (RULE != kRuleFixed) {
+          if (RULE == kRuleMomentum) {
+            m[l] = sin >= 0 ? slot_m(sin, l) : load_state(m4 + i);
+          } else if (RULE != kRuleFixed) {
             if (sin >= 0) {
               m[l] = slot_m(sin, l);
               s[l] = slot_s(sin, l);
@@ -172,6 +184,16 @@ commit_batch_kernel(const __grid_constant__ BatchArgs a) {
           if (RULE == kRuleFixed) {
             commit_vec_fixed(th[l], s[l], g[l], a.eta, a.pi[k]);
             pi = make_float4(a.pi[k], a.pi[k], a.pi[k], a.pi[k]);
+            if (a.keep_s[k]) store_state(s4 + i, s[l]);
+          } else if (RULE == kRuleMomentum) {
+            commit_coord_momentum(th[l].x, m[l].x, s[l].x, g[l].x, a.eta, a.mu);
+            commit_coord_momentum(th[l].y, m[l].y, s[l].y, g[l].y, a.eta, a.mu);
+            commit_coord_momentum(th[l].z, m[l].z, s[l].z, g[l].z, a.eta, a.mu);
+            commit_coord_momentum(th[l].w, m[l].w, s[l].w, g[l].w, a.eta, a.mu);
+            const float nan = __int_as_float(0x7fc00000);
+            pi = make_float4(nan, nan, nan, nan);
+            if (sout >= 0) slot_m(sout, l) = m[l];
+            else store_state(m4 + i, m[l]);
             if (a.keep_s[k]) store_state(s4 + i, s[l]);
           } else {
             pi = commit_vec<RULE>(th[l], m[l], s[l], g[l], a.eta, a.mu, a.eps, a.energy_scale);
@@ -206,6 +228,11 @@ commit_batch_kernel(const __grid_constant__ BatchArgs a) {
       if (RULE == kRuleFixed) {
         commit_coord_fixed(th, s, a.grad[k][j], a.eta, a.pi[k]);
         pi = a.pi[k];
+      } else if (RULE == kRuleMomentum) {
+        float m = a.m[row + j];
+        commit_coord_momentum(th, m, s, a.grad[k][j], a.eta, a.mu);
+        a.m[row + j] = m;
+        pi = __int_as_float(0x7fc00000);
       } else {
         float m = a.m[row + j];
         s = a.s[row + j];
@@ -314,6 +341,7 @@ cudaError_t launch_commit_batch(const BatchArgs& a, int sm_count, cudaStream_t s
       case kRuleGem: return launch_rule<kRuleGem, true>(a, sm_count, stream);
       case kRuleScaled: return launch_rule<kRuleScaled, true>(a, sm_count, stream);
       case kRuleFixed: return launch_rule<kRuleFixed, true>(a, sm_count, stream);
+      case kRuleMomentum: return launch_rule<kRuleMomentum, true>(a, sm_count, stream);
       default: return cudaErrorInvalidValue;
     }
   }
@@ -321,6 +349,7 @@ cudaError_t launch_commit_batch(const BatchArgs& a, int sm_count, cudaStream_t s
     case kRuleGem: return launch_rule<kRuleGem, false>(a, sm_count, stream);
     case kRuleScaled: return launch_rule<kRuleScaled, false>(a, sm_count, stream);
     case kRuleFixed: return launch_rule<kRuleFixed, false>(a, sm_count, stream);
+    case kRuleMomentum: return launch_rule<kRuleMomentum, false>(a, sm_count, stream);
     default: return cudaErrorInvalidValue;
   }
 }

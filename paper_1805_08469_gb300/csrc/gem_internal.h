@@ -27,6 +27,7 @@ enum RuleKind : int {
   kRuleGem = 0,     // pi from energy matching with the proxy |m_w| (Algorithm 1)
   kRuleScaled = 1,  // the same with the proxy energy_scale |m_w| (App. B, high-energy proxies)
   kRuleFixed = 2,   // pi[k] given per commit; m_w untouched (DOWNPOUR, adaptive staleness)
+  kRuleMomentum = 3,  // the proxy itself: theta += (m_w <- mu m_w + dtheta); no factor
 };
 
 struct BatchArgs {

@@ -22,6 +22,7 @@ GEM_MODE_DOWNPOUR = 1
 GEM_MODE_ADAPTIVE = 2
 GEM_MODE_KAPPA_SQRT = 3
 GEM_MODE_KAPPA_LINEAR = 4
+GEM_MODE_MOMENTUM = 5
 
 
 def _dev_ptr(t, what: str) -> int:

@@ -1,8 +1,9 @@
 """GPU parity of the other commit rules against the oracle, through the C ABI.
 
 Besides Algorithm 1 the library applies the comparison rules of the paper's experiments
-(DOWNPOUR: pi = 1; adaptive staleness: the update divided by tau + 1) and the high-energy
-proxies of Appendix B (sqrt(kappa) |m| and kappa |m|).  Each is one IEEE fp32 operation per
+(DOWNPOUR: pi = 1; adaptive staleness: the update divided by tau + 1), the high-energy
+proxies of Appendix B (sqrt(kappa) |m| and kappa |m|), and the momentum proxy itself
+(Eq. momentum_update) as a reference run.  Each is one IEEE fp32 operation per
 step on both sides, so the bar is bit-for-bit equality, as for the GEM rule.  The staleness
 of the adaptive rule comes from the library's own commit clock; the oracle takes the tau
 that its schedule generator computes, so the two are counted independently.
@@ -30,6 +31,7 @@ RULES = [
     (gem.GEM_MODE_KAPPA_SQRT, oracle.MODE_KAPPA_SQRT, 4.0),
     (gem.GEM_MODE_KAPPA_LINEAR, oracle.MODE_KAPPA_LINEAR, 1.5),
     (gem.GEM_MODE_KAPPA_LINEAR, oracle.MODE_KAPPA_LINEAR, 0.3),
+    (gem.GEM_MODE_MOMENTUM, oracle.MODE_MOMENTUM, 1.0),
 ]
 
 
@@ -175,7 +177,7 @@ def test_clock_checkpoint_resume():
 
 def test_mode_and_clock_argument_checks():
     with gem.Gem(100, 3, ETA, MU, EPS) as G:
-        for mode, kappa in [(-1, 1.0), (5, 1.0), (gem.GEM_MODE_KAPPA_SQRT, 0.0),
+        for mode, kappa in [(-1, 1.0), (6, 1.0), (gem.GEM_MODE_KAPPA_SQRT, 0.0),
                             (gem.GEM_MODE_KAPPA_LINEAR, -2.0), (gem.GEM_MODE_KAPPA_LINEAR, float("nan")),
                             (gem.GEM_MODE_KAPPA_SQRT, float("inf"))]:
             with pytest.raises(GemError) as e:
