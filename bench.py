@@ -49,8 +49,8 @@ FALLBACK_HBM_GBS = 6800.0
 # DRAM traffic of one launch of the batched commit kernel, from an ncu capture of the
 # same workload (see profiles/commit_batch_p25m_n100.md).  Valid only for the kernel
 # source it was taken on; reported as null once that source changes.
-NCU_TRAFFIC_BYTES_PER_LAUNCH = 40_834_115_456   # mean of two full-size launches
-NCU_TRAFFIC_SOURCE_SHA = "12a1f2beda7488bc"
+NCU_TRAFFIC_BYTES_PER_LAUNCH = 40_834_628_608   # mean of two full-size launches
+NCU_TRAFFIC_SOURCE_SHA = "0797a90967922f98"
 
 
 def kernel_source_sha() -> str:
