@@ -13,7 +13,9 @@
 //   conv2_wpart_kernel,    per-sample partial sums of the convolution weight and bias
 //   conv1_wpart_kernel     gradients
 //   conv_finish_kernel     sums of the partials over the minibatch, in sample order
-// Every value is summed in a fixed order, so the gradients do not depend on timing.
+// Every value is summed in a fixed order, so the gradients do not depend on timing.  The
+// per-sample kernels stage a sample's maps and the worker's weights in shared memory; a
+// shape whose staging exceeds 160 KB is refused.
 #include <cstdint>
 #include <cstring>
 #include <new>
@@ -32,6 +34,7 @@ using gem::mlp::kMaxGroups;
 
 constexpr int kK = 5;  // kernel side
 constexpr int kThreads = 256;
+constexpr long long kMaxSampleSmem = 160 * 1024;   // per-sample staging, bytes
 
 struct Shape {
   int H, c1, c2, f1, f2, C;
@@ -97,78 +100,95 @@ __device__ __forceinline__ int first_max4(const float* v) {
   return best;
 }
 
-// One thread per pooled output (g, i, co, py, px) of conv1.
-__global__ void __launch_bounds__(kThreads) conv1_pool_kernel(const __grid_constant__ ConvArgs a) {
-  const long long total = (long long)a.G * a.b * a.c1 * a.P1 * a.P1;
-  const long long q = blockIdx.x * (long long)kThreads + threadIdx.x;
-  if (q >= total) return;
-  const int px = int(q % a.P1), py = int(q / a.P1 % a.P1);
-  const int co = int(q / ((long long)a.P1 * a.P1) % a.c1);
-  const long long gi = q / ((long long)a.P1 * a.P1 * a.c1);   // g * b + i
-  const int g = int(gi / a.b), i = int(gi % a.b);
-  const float* x = a.X + (long long)a.rows[gi] * a.H * a.H;
-  const float* th = a.snap + (long long)a.workers[g] * a.snap_stride;
-  const float* w = th + a.w1 + co * kK * kK;
-  float wr[kK * kK];
-#pragma unroll
-  for (int k = 0; k < kK * kK; ++k) wr[k] = w[k];
-  const float bias = th[a.b1 + co];
-  float* z1 = a.scr + g * a.S + a.o_z1 + ((long long)i * a.c1 + co) * a.H1 * a.H1;
-  float v[4];
-#pragma unroll
-  for (int d = 0; d < 4; ++d) {
-    const int y = 2 * py + (d >> 1), xx = 2 * px + (d & 1);
-    float acc = bias;
-#pragma unroll
-    for (int ky = 0; ky < kK; ++ky)
-#pragma unroll
-      for (int kx = 0; kx < kK; ++kx) acc = fmaf(wr[ky * kK + kx], x[(y + ky) * a.H + xx + kx], acc);
-    v[d] = acc;
-    z1[y * a.H1 + xx] = acc;
-  }
-  const float m = v[first_max4(v)];
-  a.scr[g * a.S + a.o_a1 + (((long long)i * a.c1 + co) * a.P1 + py) * a.P1 + px] = m > 0.f ? m : 0.f;
+// The forward and weight-gradient kernels below run one block per (slot g, sample i)
+// (blockIdx.x = g b + i): the block first copies that sample's maps and the worker's
+// weights into shared memory (coalesced), then its threads compute the sample's outputs
+// from there.  Each output is summed in the same order as in the oracle's loops.
+__device__ __forceinline__ void stage(float* dst, const float* src, int n) {
+  for (int q = threadIdx.x; q < n; q += blockDim.x) dst[q] = src[q];
 }
 
-// One thread per pooled output (g, i, co, py, px) of conv2; writes the head's features.
-__global__ void __launch_bounds__(kThreads) conv2_pool_kernel(const __grid_constant__ ConvArgs a) {
-  const long long total = (long long)a.G * a.b * a.c2 * a.P2 * a.P2;
-  const long long q = blockIdx.x * (long long)kThreads + threadIdx.x;
-  if (q >= total) return;
-  const int px = int(q % a.P2), py = int(q / a.P2 % a.P2);
-  const int co = int(q / ((long long)a.P2 * a.P2) % a.c2);
-  const long long gi = q / ((long long)a.P2 * a.P2 * a.c2);
+// conv1 + bias, 2 x 2 max-pool, ReLU: thread per pooled output (co, py, px).
+__global__ void __launch_bounds__(kThreads) conv1_pool_kernel(const __grid_constant__ ConvArgs a) {
+  extern __shared__ float sm[];
+  const long long gi = blockIdx.x;
   const int g = int(gi / a.b), i = int(gi % a.b);
   const float* th = a.snap + (long long)a.workers[g] * a.snap_stride;
-  const float* w = th + a.w2 + (long long)co * a.c1 * kK * kK;
-  const float* a1 = a.scr + g * a.S + a.o_a1 + (long long)i * a.c1 * a.P1 * a.P1;
-  const float s = a.drop[gi * a.c2 + co];
-  float v[4];
+  float* xs = sm;                                   // [H * H]
+  float* ws = xs + a.H * a.H;                       // [c1][25]
+  float* bs = ws + a.c1 * kK * kK;                  // [c1]
+  stage(xs, a.X + (long long)a.rows[gi] * a.H * a.H, a.H * a.H);
+  stage(ws, th + a.w1, a.c1 * kK * kK);
+  stage(bs, th + a.b1, a.c1);
+  __syncthreads();
+  float* z1s = a.scr + g * a.S + a.o_z1 + (long long)i * a.c1 * a.H1 * a.H1;
+  float* a1s = a.scr + g * a.S + a.o_a1 + (long long)i * a.c1 * a.P1 * a.P1;
+  for (int q = threadIdx.x; q < a.c1 * a.P1 * a.P1; q += blockDim.x) {
+    const int px = q % a.P1, py = q / a.P1 % a.P1, co = q / (a.P1 * a.P1);
+    const float* w = ws + co * kK * kK;
+    float v[4];
 #pragma unroll
-  for (int d = 0; d < 4; ++d) v[d] = th[a.b2 + co];
-  for (int ci = 0; ci < a.c1; ++ci) {
-    const float* in = a1 + (long long)ci * a.P1 * a.P1;
-    const float* wc = w + ci * kK * kK;
+    for (int d = 0; d < 4; ++d) {
+      const int y = 2 * py + (d >> 1), xx = 2 * px + (d & 1);
+      float acc = bs[co];
 #pragma unroll
-    for (int ky = 0; ky < kK; ++ky)
+      for (int ky = 0; ky < kK; ++ky)
 #pragma unroll
-      for (int kx = 0; kx < kK; ++kx) {
-        const float wv = wc[ky * kK + kx];
+        for (int kx = 0; kx < kK; ++kx) acc = fmaf(w[ky * kK + kx], xs[(y + ky) * a.H + xx + kx], acc);
+      v[d] = acc;
+      z1s[(co * a.H1 + y) * a.H1 + xx] = acc;
+    }
+    const float m = v[first_max4(v)];
+    a1s[q] = m > 0.f ? m : 0.f;
+  }
+}
+
+// conv2 + bias, dropout scale, 2 x 2 max-pool, ReLU -> the head's features: thread per
+// pooled output (co, py, px).
+__global__ void __launch_bounds__(kThreads) conv2_pool_kernel(const __grid_constant__ ConvArgs a) {
+  extern __shared__ float sm[];
+  const long long gi = blockIdx.x;
+  const int g = int(gi / a.b), i = int(gi % a.b);
+  const float* th = a.snap + (long long)a.workers[g] * a.snap_stride;
+  const int n_a1 = a.c1 * a.P1 * a.P1, n_w = a.c2 * a.c1 * kK * kK;
+  float* a1s = sm;                                  // [c1][P1][P1]
+  float* ws = a1s + n_a1;                           // [c2][c1][25]
+  float* bs = ws + n_w;                             // [c2]
+  stage(a1s, a.scr + g * a.S + a.o_a1 + (long long)i * n_a1, n_a1);
+  stage(ws, th + a.w2, n_w);
+  stage(bs, th + a.b2, a.c2);
+  __syncthreads();
+  for (int q = threadIdx.x; q < a.c2 * a.P2 * a.P2; q += blockDim.x) {
+    const int px = q % a.P2, py = q / a.P2 % a.P2, co = q / (a.P2 * a.P2);
+    const float* w = ws + co * a.c1 * kK * kK;
+    const float s = a.drop[gi * a.c2 + co];
+    float v[4];
 #pragma unroll
-        for (int d = 0; d < 4; ++d) {
-          const int y = 2 * py + (d >> 1), xx = 2 * px + (d & 1);
-          v[d] = fmaf(wv, in[(y + ky) * a.P1 + xx + kx], v[d]);
+    for (int d = 0; d < 4; ++d) v[d] = bs[co];
+    for (int ci = 0; ci < a.c1; ++ci) {
+      const float* in = a1s + ci * a.P1 * a.P1;
+      const float* wc = w + ci * kK * kK;
+#pragma unroll
+      for (int ky = 0; ky < kK; ++ky)
+#pragma unroll
+        for (int kx = 0; kx < kK; ++kx) {
+          const float wv = wc[ky * kK + kx];
+#pragma unroll
+          for (int d = 0; d < 4; ++d) {
+            const int y = 2 * py + (d >> 1), xx = 2 * px + (d & 1);
+            v[d] = fmaf(wv, in[(y + ky) * a.P1 + xx + kx], v[d]);
+          }
         }
-      }
-  }
-  float* z2 = a.scr + g * a.S + a.o_z2 + ((long long)i * a.c2 + co) * a.H2 * a.H2;
+    }
+    float* z2 = a.scr + g * a.S + a.o_z2 + ((long long)i * a.c2 + co) * a.H2 * a.H2;
 #pragma unroll
-  for (int d = 0; d < 4; ++d) {
-    v[d] = v[d] * s;   // dropout: the channel's scale
-    z2[(2 * py + (d >> 1)) * a.H2 + 2 * px + (d & 1)] = v[d];
+    for (int d = 0; d < 4; ++d) {
+      v[d] = v[d] * s;   // dropout: the channel's scale
+      z2[(2 * py + (d >> 1)) * a.H2 + 2 * px + (d & 1)] = v[d];
+    }
+    const float m = v[first_max4(v)];
+    a.head[g * a.head_S + a.head_x + (long long)i * a.F + q] = m > 0.f ? m : 0.f;
   }
-  const float m = v[first_max4(v)];
-  a.head[g * a.head_S + a.head_x + (long long)i * a.F + (co * a.P2 + py) * a.P2 + px] = m > 0.f ? m : 0.f;
 }
 
 // Gradient into conv2's (pre-dropout) output: the feature gradient through the ReLU, to
@@ -197,95 +217,112 @@ __global__ void __launch_bounds__(kThreads) pool2_back_kernel(const __grid_const
   for (int d = 0; d < 4; ++d) dz2[(2 * py + (d >> 1)) * a.H2 + 2 * px + (d & 1)] = d == am ? gval : 0.f;
 }
 
-// One thread per pooled output (g, i, ci, py, px) of conv1: the gradient with respect to
-// it (sum over conv2's outputs that read it, channels then kernel rows then columns), the
-// ReLU mask, and the route through pool1 into conv1's output gradient.
+// Gradient with respect to conv1's pooled outputs (sum over the conv2 outputs that read
+// each, channels then kernel rows then columns), the ReLU mask, and the route through
+// pool1 into conv1's output gradient: thread per pooled output (ci, py, px).
 __global__ void __launch_bounds__(kThreads) conv2_back_kernel(const __grid_constant__ ConvArgs a) {
-  const long long total = (long long)a.G * a.b * a.c1 * a.P1 * a.P1;
-  const long long q = blockIdx.x * (long long)kThreads + threadIdx.x;
-  if (q >= total) return;
-  const int px = int(q % a.P1), py = int(q / a.P1 % a.P1);
-  const int ci = int(q / ((long long)a.P1 * a.P1) % a.c1);
-  const long long gi = q / ((long long)a.P1 * a.P1 * a.c1);
+  extern __shared__ float sm[];
+  const long long gi = blockIdx.x;
   const int g = int(gi / a.b), i = int(gi % a.b);
-  const float a1v = a.scr[g * a.S + a.o_a1 + (((long long)i * a.c1 + ci) * a.P1 + py) * a.P1 + px];
-  float dv = 0.f;
-  if (a1v > 0.f) {
-    const float* th = a.snap + (long long)a.workers[g] * a.snap_stride;
-    const float* dz2 = a.scr + g * a.S + a.o_dz2 + (long long)i * a.c2 * a.H2 * a.H2;
-    for (int co = 0; co < a.c2; ++co) {
-      const float* wc = th + a.w2 + ((long long)co * a.c1 + ci) * kK * kK;
-      const float* dc = dz2 + (long long)co * a.H2 * a.H2;
+  const float* th = a.snap + (long long)a.workers[g] * a.snap_stride;
+  const int n_dz2 = a.c2 * a.H2 * a.H2, n_w = a.c2 * a.c1 * kK * kK, n_a1 = a.c1 * a.P1 * a.P1;
+  float* dzs = sm;                                  // [c2][H2][H2]
+  float* ws = dzs + n_dz2;                          // [c2][c1][25]
+  float* a1s = ws + n_w;                            // [c1][P1][P1]
+  stage(dzs, a.scr + g * a.S + a.o_dz2 + (long long)i * n_dz2, n_dz2);
+  stage(ws, th + a.w2, n_w);
+  stage(a1s, a.scr + g * a.S + a.o_a1 + (long long)i * n_a1, n_a1);
+  __syncthreads();
+  const float* z1s = a.scr + g * a.S + a.o_z1 + (long long)i * a.c1 * a.H1 * a.H1;
+  float* dz1s = a.scr + g * a.S + a.o_dz1 + (long long)i * a.c1 * a.H1 * a.H1;
+  for (int q = threadIdx.x; q < n_a1; q += blockDim.x) {
+    const int px = q % a.P1, py = q / a.P1 % a.P1, ci = q / (a.P1 * a.P1);
+    float dv = 0.f;
+    if (a1s[q] > 0.f) {
+      for (int co = 0; co < a.c2; ++co) {
+        const float* wc = ws + (co * a.c1 + ci) * kK * kK;
+        const float* dc = dzs + co * a.H2 * a.H2;
 #pragma unroll
-      for (int ky = 0; ky < kK; ++ky) {
-        const int y = py - ky;
-        if (y < 0 || y >= a.H2) continue;
+        for (int ky = 0; ky < kK; ++ky) {
+          const int y = py - ky;
+          if (y < 0 || y >= a.H2) continue;
 #pragma unroll
-        for (int kx = 0; kx < kK; ++kx) {
-          const int xx = px - kx;
-          if (xx < 0 || xx >= a.H2) continue;
-          dv = fmaf(dc[y * a.H2 + xx], wc[ky * kK + kx], dv);
+          for (int kx = 0; kx < kK; ++kx) {
+            const int xx = px - kx;
+            if (xx < 0 || xx >= a.H2) continue;
+            dv = fmaf(dc[y * a.H2 + xx], wc[ky * kK + kx], dv);
+          }
         }
       }
     }
+    const float* z1 = z1s + ci * a.H1 * a.H1;
+    float* dz1 = dz1s + ci * a.H1 * a.H1;
+    float v[4];
+#pragma unroll
+    for (int d = 0; d < 4; ++d) v[d] = z1[(2 * py + (d >> 1)) * a.H1 + 2 * px + (d & 1)];
+    const int am = first_max4(v);
+#pragma unroll
+    for (int d = 0; d < 4; ++d) dz1[(2 * py + (d >> 1)) * a.H1 + 2 * px + (d & 1)] = d == am ? dv : 0.f;
   }
-  const long long base = g * a.S + ((long long)i * a.c1 + ci) * a.H1 * a.H1;
-  const float* z1 = a.scr + a.o_z1 + base;
-  float* dz1 = a.scr + a.o_dz1 + base;
-  float v[4];
-#pragma unroll
-  for (int d = 0; d < 4; ++d) v[d] = z1[(2 * py + (d >> 1)) * a.H1 + 2 * px + (d & 1)];
-  const int am = first_max4(v);
-#pragma unroll
-  for (int d = 0; d < 4; ++d) dz1[(2 * py + (d >> 1)) * a.H1 + 2 * px + (d & 1)] = d == am ? dv : 0.f;
 }
 
-// Per-sample partial sums of conv2's weight and bias gradients: thread (g, i, co, k), k <
+// Per-sample partial sums of conv2's weight and bias gradients: thread per (co, k), k <
 // c1 * 25 a weight (ci, ky, kx), k = c1 * 25 the bias; rows then columns of the output.
 __global__ void __launch_bounds__(kThreads) conv2_wpart_kernel(const __grid_constant__ ConvArgs a) {
-  const int per = a.c1 * kK * kK + 1;
-  const long long total = (long long)a.G * a.b * a.c2 * per;
-  const long long q = blockIdx.x * (long long)kThreads + threadIdx.x;
-  if (q >= total) return;
-  const int k = int(q % per);
-  const int co = int(q / per % a.c2);
-  const long long gi = q / ((long long)per * a.c2);
+  extern __shared__ float sm[];
+  const long long gi = blockIdx.x;
   const int g = int(gi / a.b), i = int(gi % a.b);
-  const float* dz2 = a.scr + g * a.S + a.o_dz2 + ((long long)i * a.c2 + co) * a.H2 * a.H2;
-  float acc = 0.f;
-  if (k == per - 1) {
-    for (int p = 0; p < a.H2 * a.H2; ++p) acc += dz2[p];
-  } else {
-    const int ci = k / (kK * kK), ky = k % (kK * kK) / kK, kx = k % kK;
-    const float* a1 = a.scr + g * a.S + a.o_a1 + ((long long)i * a.c1 + ci) * a.P1 * a.P1;
-    for (int y = 0; y < a.H2; ++y)
-      for (int xx = 0; xx < a.H2; ++xx) acc = fmaf(dz2[y * a.H2 + xx], a1[(y + ky) * a.P1 + xx + kx], acc);
+  const int n_dz2 = a.c2 * a.H2 * a.H2, n_a1 = a.c1 * a.P1 * a.P1;
+  float* dzs = sm;                                  // [c2][H2][H2]
+  float* a1s = dzs + n_dz2;                         // [c1][P1][P1]
+  stage(dzs, a.scr + g * a.S + a.o_dz2 + (long long)i * n_dz2, n_dz2);
+  stage(a1s, a.scr + g * a.S + a.o_a1 + (long long)i * n_a1, n_a1);
+  __syncthreads();
+  const int per = a.c1 * kK * kK + 1;
+  float* part = a.scr + g * a.S + a.o_p2 + (long long)i * a.c2 * per;
+  for (int q = threadIdx.x; q < a.c2 * per; q += blockDim.x) {
+    const int k = q % per, co = q / per;
+    const float* dz2 = dzs + co * a.H2 * a.H2;
+    float acc = 0.f;
+    if (k == per - 1) {
+      for (int p = 0; p < a.H2 * a.H2; ++p) acc += dz2[p];
+    } else {
+      const int ci = k / (kK * kK), ky = k % (kK * kK) / kK, kx = k % kK;
+      const float* in = a1s + ci * a.P1 * a.P1;
+      for (int y = 0; y < a.H2; ++y)
+        for (int xx = 0; xx < a.H2; ++xx) acc = fmaf(dz2[y * a.H2 + xx], in[(y + ky) * a.P1 + xx + kx], acc);
+    }
+    part[q] = acc;
   }
-  a.scr[g * a.S + a.o_p2 + ((long long)i * a.c2 + co) * per + k] = acc;
 }
 
-// Per-sample partial sums of conv1's weight and bias gradients: thread (g, i, co, k), k < 25
+// Per-sample partial sums of conv1's weight and bias gradients: thread per (co, k), k < 25
 // a weight (ky, kx), k = 25 the bias.
 __global__ void __launch_bounds__(kThreads) conv1_wpart_kernel(const __grid_constant__ ConvArgs a) {
-  constexpr int per = kK * kK + 1;
-  const long long total = (long long)a.G * a.b * a.c1 * per;
-  const long long q = blockIdx.x * (long long)kThreads + threadIdx.x;
-  if (q >= total) return;
-  const int k = int(q % per);
-  const int co = int(q / per % a.c1);
-  const long long gi = q / ((long long)per * a.c1);
+  extern __shared__ float sm[];
+  const long long gi = blockIdx.x;
   const int g = int(gi / a.b), i = int(gi % a.b);
-  const float* dz1 = a.scr + g * a.S + a.o_dz1 + ((long long)i * a.c1 + co) * a.H1 * a.H1;
-  float acc = 0.f;
-  if (k == per - 1) {
-    for (int p = 0; p < a.H1 * a.H1; ++p) acc += dz1[p];
-  } else {
-    const int ky = k / kK, kx = k % kK;
-    const float* x = a.X + (long long)a.rows[gi] * a.H * a.H;
-    for (int y = 0; y < a.H1; ++y)
-      for (int xx = 0; xx < a.H1; ++xx) acc = fmaf(dz1[y * a.H1 + xx], x[(y + ky) * a.H + xx + kx], acc);
+  const int n_dz1 = a.c1 * a.H1 * a.H1;
+  float* dzs = sm;                                  // [c1][H1][H1]
+  float* xs = dzs + n_dz1;                          // [H][H]
+  stage(dzs, a.scr + g * a.S + a.o_dz1 + (long long)i * n_dz1, n_dz1);
+  stage(xs, a.X + (long long)a.rows[gi] * a.H * a.H, a.H * a.H);
+  __syncthreads();
+  constexpr int per = kK * kK + 1;
+  float* part = a.scr + g * a.S + a.o_p1 + (long long)i * a.c1 * per;
+  for (int q = threadIdx.x; q < a.c1 * per; q += blockDim.x) {
+    const int k = q % per, co = q / per;
+    const float* dz1 = dzs + co * a.H1 * a.H1;
+    float acc = 0.f;
+    if (k == per - 1) {
+      for (int p = 0; p < a.H1 * a.H1; ++p) acc += dz1[p];
+    } else {
+      const int ky = k / kK, kx = k % kK;
+      for (int y = 0; y < a.H1; ++y)
+        for (int xx = 0; xx < a.H1; ++xx) acc = fmaf(dz1[y * a.H1 + xx], xs[(y + ky) * a.H + xx + kx], acc);
+    }
+    part[q] = acc;
   }
-  a.scr[g * a.S + a.o_p1 + ((long long)i * a.c1 + co) * per + k] = acc;
 }
 
 // Convolution gradients: the partials summed over the minibatch in sample order.
@@ -332,6 +369,7 @@ struct gem_cnn {
   int32_t* rows_dev = nullptr;   // minibatch rows uploaded from the host
   size_t rows_cap = 0;
   float* pi_rows = nullptr;      // [n][gem stride] scaling factors of a segment's commits
+  int smem[5] = {};              // dynamic shared memory of the per-sample kernels (bytes)
   uint64_t launches = 0;
 };
 
@@ -366,18 +404,19 @@ int cnn_chunk(gem_cnn* N, const int32_t* workers, int G, const int32_t* rows_dev
   a.grad_stride = grad_stride;
   for (int g = 0; g < G; ++g) a.workers[g] = workers[g];
   const long long b = N->batch;
-  const long long n_pool1 = G * b * s.c1 * s.P1 * s.P1, n_pool2 = G * b * s.c2 * s.P2 * s.P2;
+  const long long n_pool2 = G * b * s.c2 * s.P2 * s.P2;
   int rc;
-  conv1_pool_kernel<<<blocks_for(n_pool1), kThreads, 0, st>>>(a);
-  conv2_pool_kernel<<<blocks_for(n_pool2), kThreads, 0, st>>>(a);
+  const unsigned samples = unsigned(G * b);
+  conv1_pool_kernel<<<samples, kThreads, N->smem[0], st>>>(a);
+  conv2_pool_kernel<<<samples, kThreads, N->smem[1], st>>>(a);
   if ((rc = cuda_rc(cudaGetLastError()))) return rc;
   N->launches += 2;
   // the dense head: forward, loss, backward, and the feature gradient
   if ((rc = gem::mlp::mlp_chunk(N->head, workers, G, rows_dev, grads, grad_stride, losses))) return rc;
   pool2_back_kernel<<<blocks_for(n_pool2), kThreads, 0, st>>>(a);
-  conv2_back_kernel<<<blocks_for(n_pool1), kThreads, 0, st>>>(a);
-  conv2_wpart_kernel<<<blocks_for(G * b * s.c2 * (s.c1 * kK * kK + 1)), kThreads, 0, st>>>(a);
-  conv1_wpart_kernel<<<blocks_for(G * b * s.c1 * (kK * kK + 1)), kThreads, 0, st>>>(a);
+  conv2_back_kernel<<<samples, kThreads, N->smem[2], st>>>(a);
+  conv2_wpart_kernel<<<samples, kThreads, N->smem[3], st>>>(a);
+  conv1_wpart_kernel<<<samples, kThreads, N->smem[4], st>>>(a);
   conv_finish_kernel<<<blocks_for(G * ((long long)s.c1 * (kK * kK + 1) +
                                        (long long)s.c2 * (s.c1 * kK * kK + 1))),
                        kThreads, 0, st>>>(a);
@@ -447,6 +486,34 @@ int gem_cnn_create(gem_t* g, const int32_t* shape, int batch, gem_cnn_t** out) {
   N->o_p2 = take(b * s.c2 * (s.c1 * kK * kK + 1));
   N->slot_stride = off;
   N->slots = N->head->slots;
+  {
+    const long long f = sizeof(float);
+    const long long need[5] = {
+        f * (s.H * s.H + s.c1 * kK * kK + s.c1),                                    // conv1_pool
+        f * (s.c1 * s.P1 * s.P1 + (long long)s.c2 * s.c1 * kK * kK + s.c2),        // conv2_pool
+        f * (s.c2 * s.H2 * s.H2 + (long long)s.c2 * s.c1 * kK * kK + s.c1 * s.P1 * s.P1),  // conv2_back
+        f * (s.c2 * s.H2 * s.H2 + s.c1 * s.P1 * s.P1),                              // conv2_wpart
+        f * (s.c1 * s.H1 * s.H1 + s.H * s.H)};                                      // conv1_wpart
+    const void* fn[5] = {(const void*)conv1_pool_kernel, (const void*)conv2_pool_kernel,
+                         (const void*)conv2_back_kernel, (const void*)conv2_wpart_kernel,
+                         (const void*)conv1_wpart_kernel};
+    for (int k = 0; k < 5; ++k) {
+      if (need[k] > kMaxSampleSmem) {   // a sample's maps and weights must fit on chip
+        gem::mlp::mlp_free(N->head);
+        delete N;
+        return GEM_EINVAL;
+      }
+      N->smem[k] = int(need[k]);
+      if (need[k] > 48 * 1024 &&
+          cudaFuncSetAttribute(fn[k], cudaFuncAttributeMaxDynamicSharedMemorySize, int(need[k])) !=
+              cudaSuccess) {
+        cudaGetLastError();
+        gem::mlp::mlp_free(N->head);
+        delete N;
+        return GEM_ECUDA;
+      }
+    }
+  }
   int dev_prev = 0;
   cudaGetDevice(&dev_prev);
   cudaSetDevice(g->device);
