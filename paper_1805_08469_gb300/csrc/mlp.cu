@@ -602,22 +602,51 @@ gemm_mma_pipe_kernel(const __grid_constant__ GemmArgs p) {
 
 // Sum of the split-K partials of every output in split order (deterministic), then the
 // epilogue of the product.
-template <int EPI>
-__global__ void splitk_reduce_kernel(const __grid_constant__ GemmArgs p, int groups) {
-  const long long MN = (long long)p.M * p.N;
-  const long long q = blockIdx.x * (long long)blockDim.x + threadIdx.x;
-  if (q >= MN * groups) return;
-  const int g = int(q / MN);
-  const long long r = q - g * MN;
-  const int m = int(r / p.N), n = int(r - (long long)m * p.N);
-  const float* W = p.ws + (long long)g * p.ksplit * MN + r;
-  float v = 0.f;
-  for (int s = 0; s < p.ksplit; ++s) v += W[s * MN];
-  if (EPI == kBias) v = v + p.bias[(long long)p.workers[g] * p.bias_group_stride + n];
-  if (EPI == kBiasRelu) v = fmaxf(v + p.bias[(long long)p.workers[g] * p.bias_group_stride + n], 0.f);
-  if (EPI == kMask)
-    v = p.mask[(long long)g * p.mask_group_stride + (long long)m * p.ldmask + n] > 0.f ? v : 0.f;
-  p.C[(long long)g * p.c_group_stride + (long long)m * p.ldc + n] = v;
+template <int EPI, int V>
+__global__ void __launch_bounds__(256) splitk_reduce_kernel(const __grid_constant__ GemmArgs p) {
+  // one output row (g, m) per blockIdx.y; thread t of blockIdx.x covers V consecutive columns
+  const int M = p.M, N = p.N;
+  const int g = blockIdx.y / M, m = blockIdx.y - g * M;
+  const int n0 = (blockIdx.x * blockDim.x + threadIdx.x) * V;
+  if (n0 >= N) return;
+  const long long MN = (long long)M * N;
+  const float* W = p.ws + (long long)g * p.ksplit * MN + (long long)m * N + n0;
+  const float* bias = (EPI == kBias || EPI == kBiasRelu)
+                          ? p.bias + (long long)p.workers[g] * p.bias_group_stride + n0 : nullptr;
+  const float* mask = EPI == kMask ? p.mask + (long long)g * p.mask_group_stride + (long long)m * p.ldmask + n0
+                                   : nullptr;
+  float* C = p.C + (long long)g * p.c_group_stride + (long long)m * p.ldc + n0;
+  if (V == 4) {
+    float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int s = 0; s < p.ksplit; ++s) {
+      const float4 w = *reinterpret_cast<const float4*>(W + s * MN);
+      v.x += w.x;
+      v.y += w.y;
+      v.z += w.z;
+      v.w += w.w;
+    }
+    float o[4] = {v.x, v.y, v.z, v.w};
+    if (EPI == kBias || EPI == kBiasRelu) {
+      const float4 b = *reinterpret_cast<const float4*>(bias);
+      const float bb[4] = {b.x, b.y, b.z, b.w};
+#pragma unroll
+      for (int j = 0; j < 4; ++j) o[j] = EPI == kBiasRelu ? fmaxf(o[j] + bb[j], 0.f) : o[j] + bb[j];
+    }
+    if (EPI == kMask) {
+      const float4 k = *reinterpret_cast<const float4*>(mask);
+      const float kk[4] = {k.x, k.y, k.z, k.w};
+#pragma unroll
+      for (int j = 0; j < 4; ++j) o[j] = kk[j] > 0.f ? o[j] : 0.f;
+    }
+    *reinterpret_cast<float4*>(C) = make_float4(o[0], o[1], o[2], o[3]);
+  } else {
+    float v = 0.f;
+    for (int s = 0; s < p.ksplit; ++s) v += W[s * MN];
+    if (EPI == kBias) v = v + bias[0];
+    if (EPI == kBiasRelu) v = fmaxf(v + bias[0], 0.f);
+    if (EPI == kMask) v = mask[0] > 0.f ? v : 0.f;
+    C[0] = v;
+  }
 }
 
 // Products with few outputs per row (N <= kMaxClasses), used for the logits:
@@ -844,19 +873,23 @@ cudaError_t launch_gemm(const GemmArgs& a_in, int groups, bool tf32, cudaStream_
   GemmArgs a = a_in;
   a.ksplit = 1;
   a.kchunk = a.K;
+  // Products with fewer than 32 rows or a K below 32 (the last layer's weight and input
+  // gradients) would leave a 128-row tensor-core tile mostly empty or its pipeline idle:
+  // they run on the CUDA cores, with the same TF32 operand rounding.
+  const bool tc = tf32 && a.M >= 32 && a.K >= 32;
   const long long mt = (a.M + 127) / 128, nt64 = (a.N + 63) / 64, nt128 = (a.N + 127) / 128;
-  const long long big = (tf32 ? nt128 : nt64) * mt * groups;
-  if (big >= (tf32 ? GEM_TF32_BIG_TILE_BLOCKS : 2) * kSmCountHint) {
-    if (tf32)
+  const long long big = (tc ? nt128 : nt64) * mt * groups;
+  if (big >= (tc ? GEM_TF32_BIG_TILE_BLOCKS : 2) * kSmCountHint) {
+    if (tc)
       launch_mma<128, AK, BK_, EPI>(a, groups, st);
     else
-      launch_tile<128, AK, BK_, EPI>(a, groups, false, st);
+      launch_tile<128, AK, BK_, EPI>(a, groups, tf32, st);
     return cudaGetLastError();
   }
-  const long long small = tf32 ? nt64 * mt * groups : nt64 * ((a.M + 63) / 64) * groups;
+  const long long small = tc ? nt64 * mt * groups : nt64 * ((a.M + 63) / 64) * groups;
   int split = 1;
   const long long mn = (long long)a.M * a.N * groups;
-  const int min_chunk = tf32 ? GEM_TF32_MIN_CHUNK : 128;   // the tensor cores get through K faster
+  const int min_chunk = tc ? GEM_TF32_MIN_CHUNK : 128;   // the tensor cores get through K faster
   if (a.ws && a.M <= 128)
     while (split < kMaxSplit && small * split < 4 * kSmCountHint && a.K / (2 * split) >= min_chunk &&
            mn * 2 * split <= a.ws_floats)
@@ -865,13 +898,24 @@ cudaError_t launch_gemm(const GemmArgs& a_in, int groups, bool tf32, cudaStream_
     a.ksplit = split;
     a.kchunk = ((a.K + split - 1) / split + BK - 1) / BK * BK;
   }
-  if (tf32)
+  if (tc)
     launch_mma<64, AK, BK_, EPI>(a, groups * split, st);
   else
-    launch_tile<64, AK, BK_, EPI>(a, groups * split, false, st);
+    launch_tile<64, AK, BK_, EPI>(a, groups * split, tf32, st);
   if (split > 1) {
-    const long long total = (long long)a.M * a.N * groups;
-    splitk_reduce_kernel<EPI><<<unsigned((total + 255) / 256), 256, 0, st>>>(a, groups);
+    // float4 columns when every row of every array starts on a 16-byte boundary
+    auto al = [](const void* ptr, long long stride) {
+      return (reinterpret_cast<uintptr_t>(ptr) & 15u) == 0 && stride % 4 == 0;
+    };
+    const bool vec = a.N % 4 == 0 && al(a.C, a.c_group_stride) && a.ldc % 4 == 0 &&
+                     (!(EPI == kBias || EPI == kBiasRelu) || al(a.bias, a.bias_group_stride)) &&
+                     (EPI != kMask || (al(a.mask, a.mask_group_stride) && a.ldmask % 4 == 0));
+    const int V = vec ? 4 : 1;
+    dim3 grid(unsigned((a.N + 256 * V - 1) / (256 * V)), unsigned(a.M * groups));
+    if (vec)
+      splitk_reduce_kernel<EPI, 4><<<grid, 256, 0, st>>>(a);
+    else
+      splitk_reduce_kernel<EPI, 1><<<grid, 256, 0, st>>>(a);
   }
   return cudaGetLastError();
 }
