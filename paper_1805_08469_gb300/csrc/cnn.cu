@@ -219,109 +219,182 @@ __global__ void __launch_bounds__(kThreads) pool2_back_kernel(const __grid_const
 
 // Gradient with respect to conv1's pooled outputs (sum over the conv2 outputs that read
 // each, channels then kernel rows then columns), the ReLU mask, and the route through
-// pool1 into conv1's output gradient: thread per pooled output (ci, py, px).
-__global__ void __launch_bounds__(kThreads) conv2_back_kernel(const __grid_constant__ ConvArgs a) {
+// pool1 into conv1's output gradient.  A thread takes kBackRow consecutive outputs of one
+// row (ci, py): the stretch of a dz2 row that a kernel row reads is loaded once into
+// registers and serves all of them.  dz2 is staged with a row pitch of H2 + 1 floats,
+// which spreads the rows that one warp reads over distinct banks.
+constexpr int kBackRow = 12;
+constexpr int kBackThreads = 128;
+__global__ void __launch_bounds__(kBackThreads) conv2_back_kernel(const __grid_constant__ ConvArgs a) {
   extern __shared__ float sm[];
   const long long gi = blockIdx.x;
   const int g = int(gi / a.b), i = int(gi % a.b);
   const float* th = a.snap + (long long)a.workers[g] * a.snap_stride;
+  const int H2 = a.H2, pitch = a.H2 + 1;
   const int n_dz2 = a.c2 * a.H2 * a.H2, n_w = a.c2 * a.c1 * kK * kK, n_a1 = a.c1 * a.P1 * a.P1;
-  float* dzs = sm;                                  // [c2][H2][H2]
-  float* ws = dzs + n_dz2;                          // [c2][c1][25]
+  float* dzs = sm;                                  // [c2][H2][pitch]
+  float* ws = dzs + a.c2 * H2 * pitch;              // [c2][c1][25]
   float* a1s = ws + n_w;                            // [c1][P1][P1]
-  stage(dzs, a.scr + g * a.S + a.o_dz2 + (long long)i * n_dz2, n_dz2);
+  const float* dz_src = a.scr + g * a.S + a.o_dz2 + (long long)i * n_dz2;
+  for (int q = threadIdx.x; q < n_dz2; q += blockDim.x) dzs[q / H2 * pitch + q % H2] = dz_src[q];
   stage(ws, th + a.w2, n_w);
   stage(a1s, a.scr + g * a.S + a.o_a1 + (long long)i * n_a1, n_a1);
   __syncthreads();
   const float* z1s = a.scr + g * a.S + a.o_z1 + (long long)i * a.c1 * a.H1 * a.H1;
   float* dz1s = a.scr + g * a.S + a.o_dz1 + (long long)i * a.c1 * a.H1 * a.H1;
-  for (int q = threadIdx.x; q < n_a1; q += blockDim.x) {
-    const int px = q % a.P1, py = q / a.P1 % a.P1, ci = q / (a.P1 * a.P1);
-    float dv = 0.f;
-    if (a1s[q] > 0.f) {
-      for (int co = 0; co < a.c2; ++co) {
-        const float* wc = ws + (co * a.c1 + ci) * kK * kK;
-        const float* dc = dzs + co * a.H2 * a.H2;
+  const int nxb = (a.P1 + kBackRow - 1) / kBackRow;
+  for (int q = threadIdx.x; q < a.c1 * a.P1 * nxb; q += blockDim.x) {
+    const int xb = q % nxb, py = q / nxb % a.P1, ci = q / (nxb * a.P1);
+    const int px0 = xb * kBackRow;
+    // column t of the register stretch is dz2 column px0 - 4 + t
+    bool col_ok[kBackRow + kK - 1];
 #pragma unroll
-        for (int ky = 0; ky < kK; ++ky) {
-          const int y = py - ky;
-          if (y < 0 || y >= a.H2) continue;
+    for (int t = 0; t < kBackRow + kK - 1; ++t) col_ok[t] = px0 - (kK - 1) + t >= 0 && px0 - (kK - 1) + t < H2;
+    float acc[kBackRow];
 #pragma unroll
-          for (int kx = 0; kx < kK; ++kx) {
-            const int xx = px - kx;
-            if (xx < 0 || xx >= a.H2) continue;
-            dv = fmaf(dc[y * a.H2 + xx], wc[ky * kK + kx], dv);
-          }
-        }
+    for (int j = 0; j < kBackRow; ++j) acc[j] = 0.f;
+    for (int co = 0; co < a.c2; ++co) {
+      const float* wc = ws + (co * a.c1 + ci) * kK * kK;
+      const float* dc = dzs + co * H2 * pitch;
+#pragma unroll
+      for (int ky = 0; ky < kK; ++ky) {
+        const int y = py - ky;
+        if (y < 0 || y >= H2) continue;
+        const float* drow = dc + y * pitch + px0 - (kK - 1);
+        float d[kBackRow + kK - 1];
+#pragma unroll
+        for (int t = 0; t < kBackRow + kK - 1; ++t) d[t] = col_ok[t] ? drow[t] : 0.f;
+        float w[kK];
+#pragma unroll
+        for (int kx = 0; kx < kK; ++kx) w[kx] = wc[ky * kK + kx];
+#pragma unroll
+        for (int j = 0; j < kBackRow; ++j)
+#pragma unroll
+          for (int kx = 0; kx < kK; ++kx)
+            if (col_ok[j - kx + kK - 1]) acc[j] = fmaf(d[j - kx + kK - 1], w[kx], acc[j]);
       }
     }
     const float* z1 = z1s + ci * a.H1 * a.H1;
     float* dz1 = dz1s + ci * a.H1 * a.H1;
-    float v[4];
 #pragma unroll
-    for (int d = 0; d < 4; ++d) v[d] = z1[(2 * py + (d >> 1)) * a.H1 + 2 * px + (d & 1)];
-    const int am = first_max4(v);
+    for (int j = 0; j < kBackRow; ++j) {
+      const int px = px0 + j;
+      if (px >= a.P1) break;
+      const float dv = a1s[(ci * a.P1 + py) * a.P1 + px] > 0.f ? acc[j] : 0.f;
+      float v[4];
 #pragma unroll
-    for (int d = 0; d < 4; ++d) dz1[(2 * py + (d >> 1)) * a.H1 + 2 * px + (d & 1)] = d == am ? dv : 0.f;
+      for (int d = 0; d < 4; ++d) v[d] = z1[(2 * py + (d >> 1)) * a.H1 + 2 * px + (d & 1)];
+      const int am = first_max4(v);
+#pragma unroll
+      for (int d = 0; d < 4; ++d) dz1[(2 * py + (d >> 1)) * a.H1 + 2 * px + (d & 1)] = d == am ? dv : 0.f;
+    }
   }
 }
 
-// Per-sample partial sums of conv2's weight and bias gradients: thread per (co, k), k <
-// c1 * 25 a weight (ci, ky, kx), k = c1 * 25 the bias; rows then columns of the output.
+// Per-sample partial sums of conv2's weight and bias gradients, each over the output rows
+// then columns.  A thread takes the kK weights (co, ci, ky, 0..kK-1) of one kernel row and
+// slides a window of kK input values along each input row (one new load per column); the
+// last c2 work items are the biases.
 __global__ void __launch_bounds__(kThreads) conv2_wpart_kernel(const __grid_constant__ ConvArgs a) {
   extern __shared__ float sm[];
   const long long gi = blockIdx.x;
   const int g = int(gi / a.b), i = int(gi % a.b);
-  const int n_dz2 = a.c2 * a.H2 * a.H2, n_a1 = a.c1 * a.P1 * a.P1;
+  const int H2 = a.H2, P1 = a.P1;
+  const int n_dz2 = a.c2 * H2 * H2, n_a1 = a.c1 * P1 * P1;
   float* dzs = sm;                                  // [c2][H2][H2]
   float* a1s = dzs + n_dz2;                         // [c1][P1][P1]
   stage(dzs, a.scr + g * a.S + a.o_dz2 + (long long)i * n_dz2, n_dz2);
   stage(a1s, a.scr + g * a.S + a.o_a1 + (long long)i * n_a1, n_a1);
   __syncthreads();
   const int per = a.c1 * kK * kK + 1;
+  const int n_rows = a.c2 * a.c1 * kK;
   float* part = a.scr + g * a.S + a.o_p2 + (long long)i * a.c2 * per;
-  for (int q = threadIdx.x; q < a.c2 * per; q += blockDim.x) {
-    const int k = q % per, co = q / per;
-    const float* dz2 = dzs + co * a.H2 * a.H2;
-    float acc = 0.f;
-    if (k == per - 1) {
-      for (int p = 0; p < a.H2 * a.H2; ++p) acc += dz2[p];
-    } else {
-      const int ci = k / (kK * kK), ky = k % (kK * kK) / kK, kx = k % kK;
-      const float* in = a1s + ci * a.P1 * a.P1;
-      for (int y = 0; y < a.H2; ++y)
-        for (int xx = 0; xx < a.H2; ++xx) acc = fmaf(dz2[y * a.H2 + xx], in[(y + ky) * a.P1 + xx + kx], acc);
+  for (int q = threadIdx.x; q < n_rows + a.c2; q += blockDim.x) {
+    if (q >= n_rows) {
+      const int co = q - n_rows;
+      const float* dz2 = dzs + co * H2 * H2;
+      float acc = 0.f;
+      for (int p = 0; p < H2 * H2; ++p) acc += dz2[p];
+      part[co * per + per - 1] = acc;
+      continue;
     }
-    part[q] = acc;
+    const int ky = q % kK, ci = q / kK % a.c1, co = q / (kK * a.c1);
+    const float* dz2 = dzs + co * H2 * H2;
+    const float* in = a1s + (ci * P1 + ky) * P1;
+    float acc[kK];
+#pragma unroll
+    for (int kx = 0; kx < kK; ++kx) acc[kx] = 0.f;
+    for (int y = 0; y < H2; ++y) {
+      const float* drow = dz2 + y * H2;
+      const float* irow = in + y * P1;
+      float win[kK];
+#pragma unroll
+      for (int kx = 0; kx < kK - 1; ++kx) win[kx] = irow[kx];
+#pragma unroll 4
+      for (int xx = 0; xx < H2; ++xx) {
+        win[kK - 1] = irow[xx + kK - 1];
+        const float dv = drow[xx];
+#pragma unroll
+        for (int kx = 0; kx < kK; ++kx) acc[kx] = fmaf(dv, win[kx], acc[kx]);
+#pragma unroll
+        for (int kx = 0; kx < kK - 1; ++kx) win[kx] = win[kx + 1];
+      }
+    }
+#pragma unroll
+    for (int kx = 0; kx < kK; ++kx) part[co * per + (ci * kK + ky) * kK + kx] = acc[kx];
   }
 }
 
-// Per-sample partial sums of conv1's weight and bias gradients: thread per (co, k), k < 25
-// a weight (ky, kx), k = 25 the bias.
-__global__ void __launch_bounds__(kThreads) conv1_wpart_kernel(const __grid_constant__ ConvArgs a) {
+// Per-sample partial sums of conv1's weight and bias gradients, over the output rows then
+// columns: a thread per kernel row (co, ky) with a sliding window as in conv2_wpart_kernel,
+// then the c1 biases.
+constexpr int kW1Threads = 64;
+__global__ void __launch_bounds__(kW1Threads) conv1_wpart_kernel(const __grid_constant__ ConvArgs a) {
   extern __shared__ float sm[];
   const long long gi = blockIdx.x;
   const int g = int(gi / a.b), i = int(gi % a.b);
-  const int n_dz1 = a.c1 * a.H1 * a.H1;
+  const int H1 = a.H1, H = a.H;
+  const int n_dz1 = a.c1 * H1 * H1;
   float* dzs = sm;                                  // [c1][H1][H1]
   float* xs = dzs + n_dz1;                          // [H][H]
   stage(dzs, a.scr + g * a.S + a.o_dz1 + (long long)i * n_dz1, n_dz1);
-  stage(xs, a.X + (long long)a.rows[gi] * a.H * a.H, a.H * a.H);
+  stage(xs, a.X + (long long)a.rows[gi] * H * H, H * H);
   __syncthreads();
   constexpr int per = kK * kK + 1;
+  const int n_rows = a.c1 * kK;
   float* part = a.scr + g * a.S + a.o_p1 + (long long)i * a.c1 * per;
-  for (int q = threadIdx.x; q < a.c1 * per; q += blockDim.x) {
-    const int k = q % per, co = q / per;
-    const float* dz1 = dzs + co * a.H1 * a.H1;
-    float acc = 0.f;
-    if (k == per - 1) {
-      for (int p = 0; p < a.H1 * a.H1; ++p) acc += dz1[p];
-    } else {
-      const int ky = k / kK, kx = k % kK;
-      for (int y = 0; y < a.H1; ++y)
-        for (int xx = 0; xx < a.H1; ++xx) acc = fmaf(dz1[y * a.H1 + xx], xs[(y + ky) * a.H + xx + kx], acc);
+  for (int q = threadIdx.x; q < n_rows + a.c1; q += blockDim.x) {
+    if (q >= n_rows) {
+      const int co = q - n_rows;
+      const float* dz1 = dzs + co * H1 * H1;
+      float acc = 0.f;
+      for (int p = 0; p < H1 * H1; ++p) acc += dz1[p];
+      part[co * per + per - 1] = acc;
+      continue;
     }
-    part[q] = acc;
+    const int ky = q % kK, co = q / kK;
+    const float* dz1 = dzs + co * H1 * H1;
+    float acc[kK];
+#pragma unroll
+    for (int kx = 0; kx < kK; ++kx) acc[kx] = 0.f;
+    for (int y = 0; y < H1; ++y) {
+      const float* drow = dz1 + y * H1;
+      const float* irow = xs + (y + ky) * H;
+      float win[kK];
+#pragma unroll
+      for (int kx = 0; kx < kK - 1; ++kx) win[kx] = irow[kx];
+#pragma unroll 4
+      for (int xx = 0; xx < H1; ++xx) {
+        win[kK - 1] = irow[xx + kK - 1];
+        const float dv = drow[xx];
+#pragma unroll
+        for (int kx = 0; kx < kK; ++kx) acc[kx] = fmaf(dv, win[kx], acc[kx]);
+#pragma unroll
+        for (int kx = 0; kx < kK - 1; ++kx) win[kx] = win[kx + 1];
+      }
+    }
+#pragma unroll
+    for (int kx = 0; kx < kK; ++kx) part[co * per + ky * kK + kx] = acc[kx];
   }
 }
 
@@ -414,9 +487,9 @@ int cnn_chunk(gem_cnn* N, const int32_t* workers, int G, const int32_t* rows_dev
   // the dense head: forward, loss, backward, and the feature gradient
   if ((rc = gem::mlp::mlp_chunk(N->head, workers, G, rows_dev, grads, grad_stride, losses))) return rc;
   pool2_back_kernel<<<blocks_for(n_pool2), kThreads, 0, st>>>(a);
-  conv2_back_kernel<<<samples, kThreads, N->smem[2], st>>>(a);
+  conv2_back_kernel<<<samples, kBackThreads, N->smem[2], st>>>(a);
   conv2_wpart_kernel<<<samples, kThreads, N->smem[3], st>>>(a);
-  conv1_wpart_kernel<<<samples, kThreads, N->smem[4], st>>>(a);
+  conv1_wpart_kernel<<<samples, kW1Threads, N->smem[4], st>>>(a);
   conv_finish_kernel<<<blocks_for(G * ((long long)s.c1 * (kK * kK + 1) +
                                        (long long)s.c2 * (s.c1 * kK * kK + 1))),
                        kThreads, 0, st>>>(a);
@@ -491,7 +564,7 @@ int gem_cnn_create(gem_t* g, const int32_t* shape, int batch, gem_cnn_t** out) {
     const long long need[5] = {
         f * (s.H * s.H + s.c1 * kK * kK + s.c1),                                    // conv1_pool
         f * (s.c1 * s.P1 * s.P1 + (long long)s.c2 * s.c1 * kK * kK + s.c2),        // conv2_pool
-        f * (s.c2 * s.H2 * s.H2 + (long long)s.c2 * s.c1 * kK * kK + s.c1 * s.P1 * s.P1),  // conv2_back
+        f * (s.c2 * s.H2 * (s.H2 + 1) + (long long)s.c2 * s.c1 * kK * kK + s.c1 * s.P1 * s.P1),  // conv2_back
         f * (s.c2 * s.H2 * s.H2 + s.c1 * s.P1 * s.P1),                              // conv2_wpart
         f * (s.c1 * s.H1 * s.H1 + s.H * s.H)};                                      // conv1_wpart
     const void* fn[5] = {(const void*)conv1_pool_kernel, (const void*)conv2_pool_kernel,

@@ -84,7 +84,9 @@ def _blocks(shape):
 
 
 @pytest.mark.parametrize("shape,b,G", [(cnn.CNN_MNIST, 64, 3), ((16, 3, 4, 5, 4, 3), 7, 2),
-                                       ((20, 2, 3, 7, 6, 4), 5, 3)])
+                                       ((20, 2, 3, 7, 6, 4), 5, 3),
+                                       # pooled conv1 rows of 16: two row blocks, the second ragged
+                                       ((36, 2, 3, 6, 5, 3), 3, 2)])
 def test_gradients_match_the_oracle(shape, b, G):
     """G workers with different snapshots, in one batched call; every parameter tensor of
     every worker's gradient within 1e-5 relative L2 of the oracle's double gradient."""
