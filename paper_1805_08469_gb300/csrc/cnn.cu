@@ -92,20 +92,51 @@ struct ConvArgs {
   int workers[kMaxGroups];
 };
 
-__device__ __forceinline__ int first_max4(const float* v) {
+// Index of the first maximum of a 2 x 2 window (row-major), and its value in *mx.
+__device__ __forceinline__ int first_max4(const float (&v)[4], float* mx) {
   int best = 0;
+  float bv = v[0];
 #pragma unroll
   for (int q = 1; q < 4; ++q)
-    if (v[q] > v[best]) best = q;
+    if (v[q] > bv) {
+      best = q;
+      bv = v[q];
+    }
+  *mx = bv;
   return best;
 }
 
-// The forward and weight-gradient kernels below run one block per (slot g, sample i)
-// (blockIdx.x = g b + i): the block first copies that sample's maps and the worker's
-// weights into shared memory (coalesced), then its threads compute the sample's outputs
-// from there.  Each output is summed in the same order as in the oracle's loops.
+// The per-sample kernels below run one block per (slot g, sample i) (blockIdx.x = g b + i):
+// the block first copies that sample's maps and the worker's weights into shared memory
+// with asynchronous copies (every thread's copies in flight at once, so the block waits
+// for about one memory latency rather than one per element), then its threads compute the
+// sample's outputs from there.  Each output is summed in the same order as in the
+// oracle's loops.
+__device__ __forceinline__ void cp_async4(float* dst, const float* src) {
+  const uint32_t d = static_cast<uint32_t>(__cvta_generic_to_shared(dst));
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(d), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async16(float* dst, const float* src) {
+  const uint32_t d = static_cast<uint32_t>(__cvta_generic_to_shared(dst));
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(d), "l"(src) : "memory");
+}
+
+// Start copying n floats from global src to shared dst: 16-byte copies when both ends are
+// 16-byte aligned, 4-byte copies for the rest.
 __device__ __forceinline__ void stage(float* dst, const float* src, int n) {
-  for (int q = threadIdx.x; q < n; q += blockDim.x) dst[q] = src[q];
+  int head = 0;
+  if (((reinterpret_cast<uintptr_t>(dst) | reinterpret_cast<uintptr_t>(src)) & 15u) == 0) {
+    const int n4 = n >> 2;
+    for (int q = threadIdx.x; q < n4; q += blockDim.x) cp_async16(dst + 4 * q, src + 4 * q);
+    head = n4 << 2;
+  }
+  for (int q = head + threadIdx.x; q < n; q += blockDim.x) cp_async4(dst + q, src + q);
+}
+
+// Wait for this thread's copies, then for the whole block's.
+__device__ __forceinline__ void stage_wait() {
+  asm volatile("cp.async.commit_group;\n\tcp.async.wait_group 0;" ::: "memory");
+  __syncthreads();
 }
 
 // conv1 + bias, 2 x 2 max-pool, ReLU: thread per pooled output (co, py, px).
@@ -120,7 +151,7 @@ __global__ void __launch_bounds__(kThreads) conv1_pool_kernel(const __grid_const
   stage(xs, a.X + (long long)a.rows[gi] * a.H * a.H, a.H * a.H);
   stage(ws, th + a.w1, a.c1 * kK * kK);
   stage(bs, th + a.b1, a.c1);
-  __syncthreads();
+  stage_wait();
   float* z1s = a.scr + g * a.S + a.o_z1 + (long long)i * a.c1 * a.H1 * a.H1;
   float* a1s = a.scr + g * a.S + a.o_a1 + (long long)i * a.c1 * a.P1 * a.P1;
   for (int q = threadIdx.x; q < a.c1 * a.P1 * a.P1; q += blockDim.x) {
@@ -138,7 +169,8 @@ __global__ void __launch_bounds__(kThreads) conv1_pool_kernel(const __grid_const
       v[d] = acc;
       z1s[(co * a.H1 + y) * a.H1 + xx] = acc;
     }
-    const float m = v[first_max4(v)];
+    float m;
+    first_max4(v, &m);
     a1s[q] = m > 0.f ? m : 0.f;
   }
 }
@@ -157,7 +189,7 @@ __global__ void __launch_bounds__(kThreads) conv2_pool_kernel(const __grid_const
   stage(a1s, a.scr + g * a.S + a.o_a1 + (long long)i * n_a1, n_a1);
   stage(ws, th + a.w2, n_w);
   stage(bs, th + a.b2, a.c2);
-  __syncthreads();
+  stage_wait();
   for (int q = threadIdx.x; q < a.c2 * a.P2 * a.P2; q += blockDim.x) {
     const int px = q % a.P2, py = q / a.P2 % a.P2, co = q / (a.P2 * a.P2);
     const float* w = ws + co * a.c1 * kK * kK;
@@ -186,7 +218,8 @@ __global__ void __launch_bounds__(kThreads) conv2_pool_kernel(const __grid_const
       v[d] = v[d] * s;   // dropout: the channel's scale
       z2[(2 * py + (d >> 1)) * a.H2 + 2 * px + (d & 1)] = v[d];
     }
-    const float m = v[first_max4(v)];
+    float m;
+    first_max4(v, &m);
     a.head[g * a.head_S + a.head_x + (long long)i * a.F + q] = m > 0.f ? m : 0.f;
   }
 }
@@ -211,7 +244,8 @@ __global__ void __launch_bounds__(kThreads) pool2_back_kernel(const __grid_const
   float v[4];
 #pragma unroll
   for (int d = 0; d < 4; ++d) v[d] = z2[(2 * py + (d >> 1)) * a.H2 + 2 * px + (d & 1)];
-  const int am = first_max4(v);
+  float vmax;
+  const int am = first_max4(v, &vmax);
   const float gval = feat > 0.f ? dfeat * s : 0.f;
 #pragma unroll
   for (int d = 0; d < 4; ++d) dz2[(2 * py + (d >> 1)) * a.H2 + 2 * px + (d & 1)] = d == am ? gval : 0.f;
@@ -236,10 +270,10 @@ __global__ void __launch_bounds__(kBackThreads) conv2_back_kernel(const __grid_c
   float* ws = dzs + a.c2 * H2 * pitch;              // [c2][c1][25]
   float* a1s = ws + n_w;                            // [c1][P1][P1]
   const float* dz_src = a.scr + g * a.S + a.o_dz2 + (long long)i * n_dz2;
-  for (int q = threadIdx.x; q < n_dz2; q += blockDim.x) dzs[q / H2 * pitch + q % H2] = dz_src[q];
+  for (int q = threadIdx.x; q < n_dz2; q += blockDim.x) cp_async4(dzs + q / H2 * pitch + q % H2, dz_src + q);
   stage(ws, th + a.w2, n_w);
   stage(a1s, a.scr + g * a.S + a.o_a1 + (long long)i * n_a1, n_a1);
-  __syncthreads();
+  stage_wait();
   const float* z1s = a.scr + g * a.S + a.o_z1 + (long long)i * a.c1 * a.H1 * a.H1;
   float* dz1s = a.scr + g * a.S + a.o_dz1 + (long long)i * a.c1 * a.H1 * a.H1;
   const int nxb = (a.P1 + kBackRow - 1) / kBackRow;
@@ -284,7 +318,8 @@ __global__ void __launch_bounds__(kBackThreads) conv2_back_kernel(const __grid_c
       float v[4];
 #pragma unroll
       for (int d = 0; d < 4; ++d) v[d] = z1[(2 * py + (d >> 1)) * a.H1 + 2 * px + (d & 1)];
-      const int am = first_max4(v);
+      float vmax;
+  const int am = first_max4(v, &vmax);
 #pragma unroll
       for (int d = 0; d < 4; ++d) dz1[(2 * py + (d >> 1)) * a.H1 + 2 * px + (d & 1)] = d == am ? dv : 0.f;
     }
@@ -305,7 +340,7 @@ __global__ void __launch_bounds__(kThreads) conv2_wpart_kernel(const __grid_cons
   float* a1s = dzs + n_dz2;                         // [c1][P1][P1]
   stage(dzs, a.scr + g * a.S + a.o_dz2 + (long long)i * n_dz2, n_dz2);
   stage(a1s, a.scr + g * a.S + a.o_a1 + (long long)i * n_a1, n_a1);
-  __syncthreads();
+  stage_wait();
   const int per = a.c1 * kK * kK + 1;
   const int n_rows = a.c2 * a.c1 * kK;
   float* part = a.scr + g * a.S + a.o_p2 + (long long)i * a.c2 * per;
@@ -359,7 +394,7 @@ __global__ void __launch_bounds__(kW1Threads) conv1_wpart_kernel(const __grid_co
   float* xs = dzs + n_dz1;                          // [H][H]
   stage(dzs, a.scr + g * a.S + a.o_dz1 + (long long)i * n_dz1, n_dz1);
   stage(xs, a.X + (long long)a.rows[gi] * H * H, H * H);
-  __syncthreads();
+  stage_wait();
   constexpr int per = kK * kK + 1;
   const int n_rows = a.c1 * kK;
   float* part = a.scr + g * a.S + a.o_p1 + (long long)i * a.c1 * per;
