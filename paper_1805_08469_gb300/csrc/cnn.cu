@@ -259,13 +259,19 @@ __global__ void __launch_bounds__(kThreads) pool2_back_kernel(const __grid_const
 // which spreads the rows that one warp reads over distinct banks.
 constexpr int kBackRow = 12;
 constexpr int kBackThreads = 128;
+// H2C, P1C: conv2's output side and conv1's pooled side when known at compile time (the
+// paper's network: 8 and 12), which folds the column bounds; 0 reads them from the
+// arguments.  Threads take channels fastest, so the lanes of a warp share a few output
+// rows: they read the same dz2 row stretch (a shared-memory broadcast) and skip the same
+// kernel rows.
+template <int H2C, int P1C>
 __global__ void __launch_bounds__(kBackThreads) conv2_back_kernel(const __grid_constant__ ConvArgs a) {
   extern __shared__ float sm[];
   const long long gi = blockIdx.x;
   const int g = int(gi / a.b), i = int(gi % a.b);
   const float* th = a.snap + (long long)a.workers[g] * a.snap_stride;
-  const int H2 = a.H2, pitch = a.H2 + 1;
-  const int n_dz2 = a.c2 * a.H2 * a.H2, n_w = a.c2 * a.c1 * kK * kK, n_a1 = a.c1 * a.P1 * a.P1;
+  const int H2 = H2C ? H2C : a.H2, P1 = P1C ? P1C : a.P1, pitch = H2 + 1;
+  const int n_dz2 = a.c2 * H2 * H2, n_w = a.c2 * a.c1 * kK * kK, n_a1 = a.c1 * P1 * P1;
   float* dzs = sm;                                  // [c2][H2][pitch]
   float* ws = dzs + a.c2 * H2 * pitch;              // [c2][c1][25]
   float* a1s = ws + n_w;                            // [c1][P1][P1]
@@ -274,11 +280,13 @@ __global__ void __launch_bounds__(kBackThreads) conv2_back_kernel(const __grid_c
   stage(ws, th + a.w2, n_w);
   stage(a1s, a.scr + g * a.S + a.o_a1 + (long long)i * n_a1, n_a1);
   stage_wait();
-  const float* z1s = a.scr + g * a.S + a.o_z1 + (long long)i * a.c1 * a.H1 * a.H1;
-  float* dz1s = a.scr + g * a.S + a.o_dz1 + (long long)i * a.c1 * a.H1 * a.H1;
-  const int nxb = (a.P1 + kBackRow - 1) / kBackRow;
-  for (int q = threadIdx.x; q < a.c1 * a.P1 * nxb; q += blockDim.x) {
-    const int xb = q % nxb, py = q / nxb % a.P1, ci = q / (nxb * a.P1);
+  const int H1 = 2 * P1;
+  const float* z1s = a.scr + g * a.S + a.o_z1 + (long long)i * a.c1 * H1 * H1;
+  float* dz1s = a.scr + g * a.S + a.o_dz1 + (long long)i * a.c1 * H1 * H1;
+  const int nxb = (P1 + kBackRow - 1) / kBackRow;
+  for (int q = threadIdx.x; q < a.c1 * P1 * nxb; q += blockDim.x) {
+    const int ci = q % a.c1, rest = q / a.c1;
+    const int xb = rest % nxb, py = rest / nxb;
     const int px0 = xb * kBackRow;
     // column t of the register stretch is dz2 column px0 - 4 + t
     bool col_ok[kBackRow + kK - 1];
@@ -308,20 +316,20 @@ __global__ void __launch_bounds__(kBackThreads) conv2_back_kernel(const __grid_c
             if (col_ok[j - kx + kK - 1]) acc[j] = fmaf(d[j - kx + kK - 1], w[kx], acc[j]);
       }
     }
-    const float* z1 = z1s + ci * a.H1 * a.H1;
-    float* dz1 = dz1s + ci * a.H1 * a.H1;
+    const float* z1 = z1s + ci * H1 * H1;
+    float* dz1 = dz1s + ci * H1 * H1;
 #pragma unroll
     for (int j = 0; j < kBackRow; ++j) {
       const int px = px0 + j;
-      if (px >= a.P1) break;
-      const float dv = a1s[(ci * a.P1 + py) * a.P1 + px] > 0.f ? acc[j] : 0.f;
+      if (px >= P1) break;
+      const float dv = a1s[(ci * P1 + py) * P1 + px] > 0.f ? acc[j] : 0.f;
       float v[4];
 #pragma unroll
-      for (int d = 0; d < 4; ++d) v[d] = z1[(2 * py + (d >> 1)) * a.H1 + 2 * px + (d & 1)];
+      for (int d = 0; d < 4; ++d) v[d] = z1[(2 * py + (d >> 1)) * H1 + 2 * px + (d & 1)];
       float vmax;
-  const int am = first_max4(v, &vmax);
+      const int am = first_max4(v, &vmax);
 #pragma unroll
-      for (int d = 0; d < 4; ++d) dz1[(2 * py + (d >> 1)) * a.H1 + 2 * px + (d & 1)] = d == am ? dv : 0.f;
+      for (int d = 0; d < 4; ++d) dz1[(2 * py + (d >> 1)) * H1 + 2 * px + (d & 1)] = d == am ? dv : 0.f;
     }
   }
 }
@@ -330,11 +338,13 @@ __global__ void __launch_bounds__(kBackThreads) conv2_back_kernel(const __grid_c
 // then columns.  A thread takes the kK weights (co, ci, ky, 0..kK-1) of one kernel row and
 // slides a window of kK input values along each input row (one new load per column); the
 // last c2 work items are the biases.
+// H2C, P1C as in conv2_back_kernel.
+template <int H2C, int P1C>
 __global__ void __launch_bounds__(kThreads) conv2_wpart_kernel(const __grid_constant__ ConvArgs a) {
   extern __shared__ float sm[];
   const long long gi = blockIdx.x;
   const int g = int(gi / a.b), i = int(gi % a.b);
-  const int H2 = a.H2, P1 = a.P1;
+  const int H2 = H2C ? H2C : a.H2, P1 = P1C ? P1C : a.P1;
   const int n_dz2 = a.c2 * H2 * H2, n_a1 = a.c1 * P1 * P1;
   float* dzs = sm;                                  // [c2][H2][H2]
   float* a1s = dzs + n_dz2;                         // [c1][P1][P1]
@@ -383,12 +393,15 @@ __global__ void __launch_bounds__(kThreads) conv2_wpart_kernel(const __grid_cons
 // Per-sample partial sums of conv1's weight and bias gradients, over the output rows then
 // columns: a thread per kernel row (co, ky) with a sliding window as in conv2_wpart_kernel,
 // then the c1 biases.
+// H1C, HC: conv1's output side and the input side when known at compile time (the
+// paper's network: 24 and 28); 0 reads them from the arguments.
 constexpr int kW1Threads = 64;
+template <int H1C, int HC>
 __global__ void __launch_bounds__(kW1Threads) conv1_wpart_kernel(const __grid_constant__ ConvArgs a) {
   extern __shared__ float sm[];
   const long long gi = blockIdx.x;
   const int g = int(gi / a.b), i = int(gi % a.b);
-  const int H1 = a.H1, H = a.H;
+  const int H1 = H1C ? H1C : a.H1, H = HC ? HC : a.H;
   const int n_dz1 = a.c1 * H1 * H1;
   float* dzs = sm;                                  // [c1][H1][H1]
   float* xs = dzs + n_dz1;                          // [H][H]
@@ -522,9 +535,15 @@ int cnn_chunk(gem_cnn* N, const int32_t* workers, int G, const int32_t* rows_dev
   // the dense head: forward, loss, backward, and the feature gradient
   if ((rc = gem::mlp::mlp_chunk(N->head, workers, G, rows_dev, grads, grad_stride, losses))) return rc;
   pool2_back_kernel<<<blocks_for(n_pool2), kThreads, 0, st>>>(a);
-  conv2_back_kernel<<<samples, kBackThreads, N->smem[2], st>>>(a);
-  conv2_wpart_kernel<<<samples, kThreads, N->smem[3], st>>>(a);
-  conv1_wpart_kernel<<<samples, kW1Threads, N->smem[4], st>>>(a);
+  if (s.H == 28) {   // the paper's map sizes: loop bounds known at compile time
+    conv2_back_kernel<8, 12><<<samples, kBackThreads, N->smem[2], st>>>(a);
+    conv2_wpart_kernel<8, 12><<<samples, kThreads, N->smem[3], st>>>(a);
+    conv1_wpart_kernel<24, 28><<<samples, kW1Threads, N->smem[4], st>>>(a);
+  } else {
+    conv2_back_kernel<0, 0><<<samples, kBackThreads, N->smem[2], st>>>(a);
+    conv2_wpart_kernel<0, 0><<<samples, kThreads, N->smem[3], st>>>(a);
+    conv1_wpart_kernel<0, 0><<<samples, kW1Threads, N->smem[4], st>>>(a);
+  }
   conv_finish_kernel<<<blocks_for(G * ((long long)s.c1 * (kK * kK + 1) +
                                        (long long)s.c2 * (s.c1 * kK * kK + 1))),
                        kThreads, 0, st>>>(a);
@@ -602,9 +621,12 @@ int gem_cnn_create(gem_t* g, const int32_t* shape, int batch, gem_cnn_t** out) {
         f * (s.c2 * s.H2 * (s.H2 + 1) + (long long)s.c2 * s.c1 * kK * kK + s.c1 * s.P1 * s.P1),  // conv2_back
         f * (s.c2 * s.H2 * s.H2 + s.c1 * s.P1 * s.P1),                              // conv2_wpart
         f * (s.c1 * s.H1 * s.H1 + s.H * s.H)};                                      // conv1_wpart
-    const void* fn[5] = {(const void*)conv1_pool_kernel, (const void*)conv2_pool_kernel,
-                         (const void*)conv2_back_kernel, (const void*)conv2_wpart_kernel,
-                         (const void*)conv1_wpart_kernel};
+    // per kernel, the generic instantiation and the one for the paper's map sizes
+    const void* fn[5][2] = {{(const void*)conv1_pool_kernel, nullptr},
+                            {(const void*)conv2_pool_kernel, nullptr},
+                            {(const void*)conv2_back_kernel<0, 0>, (const void*)conv2_back_kernel<8, 12>},
+                            {(const void*)conv2_wpart_kernel<0, 0>, (const void*)conv2_wpart_kernel<8, 12>},
+                            {(const void*)conv1_wpart_kernel<0, 0>, (const void*)conv1_wpart_kernel<24, 28>}};
     for (int k = 0; k < 5; ++k) {
       if (need[k] > kMaxSampleSmem) {   // a sample's maps and weights must fit on chip
         gem::mlp::mlp_free(N->head);
@@ -612,9 +634,12 @@ int gem_cnn_create(gem_t* g, const int32_t* shape, int batch, gem_cnn_t** out) {
         return GEM_EINVAL;
       }
       N->smem[k] = int(need[k]);
-      if (need[k] > 48 * 1024 &&
-          cudaFuncSetAttribute(fn[k], cudaFuncAttributeMaxDynamicSharedMemorySize, int(need[k])) !=
-              cudaSuccess) {
+      bool ok = true;
+      for (int v = 0; v < 2 && need[k] > 48 * 1024; ++v)
+        if (fn[k][v] && cudaFuncSetAttribute(fn[k][v], cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             int(need[k])) != cudaSuccess)
+          ok = false;
+      if (!ok) {
         cudaGetLastError();
         gem::mlp::mlp_free(N->head);
         delete N;
