@@ -139,35 +139,44 @@ __device__ __forceinline__ void stage_wait() {
   __syncthreads();
 }
 
-// conv1 + bias, 2 x 2 max-pool, ReLU: thread per pooled output (co, py, px).
+// conv1 + bias, 2 x 2 max-pool, ReLU: thread per pooled output (co, py, px), the 6 x 6
+// input patch of its window and the channel's 25 weights in registers.  HC: the input side
+// when known at compile time (the paper's network: 28), 0 reads it from the arguments.
+template <int HC>
 __global__ void __launch_bounds__(kThreads) conv1_pool_kernel(const __grid_constant__ ConvArgs a) {
   extern __shared__ float sm[];
   const long long gi = blockIdx.x;
   const int g = int(gi / a.b), i = int(gi % a.b);
+  const int H = HC ? HC : a.H, H1 = H - (kK - 1), P1 = H1 / 2;
   const float* th = a.snap + (long long)a.workers[g] * a.snap_stride;
   float* xs = sm;                                   // [H * H]
-  float* ws = xs + a.H * a.H;                       // [c1][25]
+  float* ws = xs + H * H;                           // [c1][25]
   float* bs = ws + a.c1 * kK * kK;                  // [c1]
-  stage(xs, a.X + (long long)a.rows[gi] * a.H * a.H, a.H * a.H);
+  stage(xs, a.X + (long long)a.rows[gi] * H * H, H * H);
   stage(ws, th + a.w1, a.c1 * kK * kK);
   stage(bs, th + a.b1, a.c1);
   stage_wait();
-  float* z1s = a.scr + g * a.S + a.o_z1 + (long long)i * a.c1 * a.H1 * a.H1;
-  float* a1s = a.scr + g * a.S + a.o_a1 + (long long)i * a.c1 * a.P1 * a.P1;
-  for (int q = threadIdx.x; q < a.c1 * a.P1 * a.P1; q += blockDim.x) {
-    const int px = q % a.P1, py = q / a.P1 % a.P1, co = q / (a.P1 * a.P1);
-    const float* w = ws + co * kK * kK;
+  float* z1s = a.scr + g * a.S + a.o_z1 + (long long)i * a.c1 * H1 * H1;
+  float* a1s = a.scr + g * a.S + a.o_a1 + (long long)i * a.c1 * P1 * P1;
+  for (int q = threadIdx.x; q < a.c1 * P1 * P1; q += blockDim.x) {
+    const int px = q % P1, py = q / P1 % P1, co = q / (P1 * P1);
+    float x[kK + 1][kK + 1], w[kK * kK];
+#pragma unroll
+    for (int r = 0; r <= kK; ++r)
+#pragma unroll
+      for (int c = 0; c <= kK; ++c) x[r][c] = xs[(2 * py + r) * H + 2 * px + c];
+#pragma unroll
+    for (int k = 0; k < kK * kK; ++k) w[k] = ws[co * kK * kK + k];
     float v[4];
 #pragma unroll
     for (int d = 0; d < 4; ++d) {
-      const int y = 2 * py + (d >> 1), xx = 2 * px + (d & 1);
       float acc = bs[co];
 #pragma unroll
       for (int ky = 0; ky < kK; ++ky)
 #pragma unroll
-        for (int kx = 0; kx < kK; ++kx) acc = fmaf(w[ky * kK + kx], xs[(y + ky) * a.H + xx + kx], acc);
+        for (int kx = 0; kx < kK; ++kx) acc = fmaf(w[ky * kK + kx], x[(d >> 1) + ky][(d & 1) + kx], acc);
       v[d] = acc;
-      z1s[(co * a.H1 + y) * a.H1 + xx] = acc;
+      z1s[(co * H1 + 2 * py + (d >> 1)) * H1 + 2 * px + (d & 1)] = acc;
     }
     float m;
     first_max4(v, &m);
@@ -176,13 +185,18 @@ __global__ void __launch_bounds__(kThreads) conv1_pool_kernel(const __grid_const
 }
 
 // conv2 + bias, dropout scale, 2 x 2 max-pool, ReLU -> the head's features: thread per
-// pooled output (co, py, px).
-__global__ void __launch_bounds__(kThreads) conv2_pool_kernel(const __grid_constant__ ConvArgs a) {
+// pooled output (co, py, px), per input channel the 6 x 6 patch of its window and the 25
+// weights in registers.  P1C: conv1's pooled side when known at compile time (12), 0 reads
+// it from the arguments.
+constexpr int kPool2Threads = 320;
+template <int P1C>
+__global__ void __launch_bounds__(kPool2Threads) conv2_pool_kernel(const __grid_constant__ ConvArgs a) {
   extern __shared__ float sm[];
   const long long gi = blockIdx.x;
   const int g = int(gi / a.b), i = int(gi % a.b);
+  const int P1 = P1C ? P1C : a.P1, H2 = P1 - (kK - 1), P2 = H2 / 2;
   const float* th = a.snap + (long long)a.workers[g] * a.snap_stride;
-  const int n_a1 = a.c1 * a.P1 * a.P1, n_w = a.c2 * a.c1 * kK * kK;
+  const int n_a1 = a.c1 * P1 * P1, n_w = a.c2 * a.c1 * kK * kK;
   float* a1s = sm;                                  // [c1][P1][P1]
   float* ws = a1s + n_a1;                           // [c2][c1][25]
   float* bs = ws + n_w;                             // [c2]
@@ -190,33 +204,34 @@ __global__ void __launch_bounds__(kThreads) conv2_pool_kernel(const __grid_const
   stage(ws, th + a.w2, n_w);
   stage(bs, th + a.b2, a.c2);
   stage_wait();
-  for (int q = threadIdx.x; q < a.c2 * a.P2 * a.P2; q += blockDim.x) {
-    const int px = q % a.P2, py = q / a.P2 % a.P2, co = q / (a.P2 * a.P2);
-    const float* w = ws + co * a.c1 * kK * kK;
+  for (int q = threadIdx.x; q < a.c2 * P2 * P2; q += blockDim.x) {
+    const int px = q % P2, py = q / P2 % P2, co = q / (P2 * P2);
     const float s = a.drop[gi * a.c2 + co];
     float v[4];
 #pragma unroll
     for (int d = 0; d < 4; ++d) v[d] = bs[co];
     for (int ci = 0; ci < a.c1; ++ci) {
-      const float* in = a1s + ci * a.P1 * a.P1;
-      const float* wc = w + ci * kK * kK;
+      const float* in = a1s + ci * P1 * P1;
+      const float* wc = ws + (co * a.c1 + ci) * kK * kK;
+      float x[kK + 1][kK + 1], w[kK * kK];
+#pragma unroll
+      for (int r = 0; r <= kK; ++r)
+#pragma unroll
+        for (int c = 0; c <= kK; ++c) x[r][c] = in[(2 * py + r) * P1 + 2 * px + c];
+#pragma unroll
+      for (int k = 0; k < kK * kK; ++k) w[k] = wc[k];
 #pragma unroll
       for (int ky = 0; ky < kK; ++ky)
 #pragma unroll
-        for (int kx = 0; kx < kK; ++kx) {
-          const float wv = wc[ky * kK + kx];
+        for (int kx = 0; kx < kK; ++kx)
 #pragma unroll
-          for (int d = 0; d < 4; ++d) {
-            const int y = 2 * py + (d >> 1), xx = 2 * px + (d & 1);
-            v[d] = fmaf(wv, in[(y + ky) * a.P1 + xx + kx], v[d]);
-          }
-        }
+          for (int d = 0; d < 4; ++d) v[d] = fmaf(w[ky * kK + kx], x[(d >> 1) + ky][(d & 1) + kx], v[d]);
     }
-    float* z2 = a.scr + g * a.S + a.o_z2 + ((long long)i * a.c2 + co) * a.H2 * a.H2;
+    float* z2 = a.scr + g * a.S + a.o_z2 + ((long long)i * a.c2 + co) * H2 * H2;
 #pragma unroll
     for (int d = 0; d < 4; ++d) {
       v[d] = v[d] * s;   // dropout: the channel's scale
-      z2[(2 * py + (d >> 1)) * a.H2 + 2 * px + (d & 1)] = v[d];
+      z2[(2 * py + (d >> 1)) * H2 + 2 * px + (d & 1)] = v[d];
     }
     float m;
     first_max4(v, &m);
@@ -528,8 +543,13 @@ int cnn_chunk(gem_cnn* N, const int32_t* workers, int G, const int32_t* rows_dev
   const long long n_pool2 = G * b * s.c2 * s.P2 * s.P2;
   int rc;
   const unsigned samples = unsigned(G * b);
-  conv1_pool_kernel<<<samples, kThreads, N->smem[0], st>>>(a);
-  conv2_pool_kernel<<<samples, kThreads, N->smem[1], st>>>(a);
+  if (s.H == 28) {
+    conv1_pool_kernel<28><<<samples, kThreads, N->smem[0], st>>>(a);
+    conv2_pool_kernel<12><<<samples, kPool2Threads, N->smem[1], st>>>(a);
+  } else {
+    conv1_pool_kernel<0><<<samples, kThreads, N->smem[0], st>>>(a);
+    conv2_pool_kernel<0><<<samples, kPool2Threads, N->smem[1], st>>>(a);
+  }
   if ((rc = cuda_rc(cudaGetLastError()))) return rc;
   N->launches += 2;
   // the dense head: forward, loss, backward, and the feature gradient
@@ -622,8 +642,8 @@ int gem_cnn_create(gem_t* g, const int32_t* shape, int batch, gem_cnn_t** out) {
         f * (s.c2 * s.H2 * s.H2 + s.c1 * s.P1 * s.P1),                              // conv2_wpart
         f * (s.c1 * s.H1 * s.H1 + s.H * s.H)};                                      // conv1_wpart
     // per kernel, the generic instantiation and the one for the paper's map sizes
-    const void* fn[5][2] = {{(const void*)conv1_pool_kernel, nullptr},
-                            {(const void*)conv2_pool_kernel, nullptr},
+    const void* fn[5][2] = {{(const void*)conv1_pool_kernel<0>, (const void*)conv1_pool_kernel<28>},
+                            {(const void*)conv2_pool_kernel<0>, (const void*)conv2_pool_kernel<12>},
                             {(const void*)conv2_back_kernel<0, 0>, (const void*)conv2_back_kernel<8, 12>},
                             {(const void*)conv2_wpart_kernel<0, 0>, (const void*)conv2_wpart_kernel<8, 12>},
                             {(const void*)conv1_wpart_kernel<0, 0>, (const void*)conv1_wpart_kernel<24, 28>}};
