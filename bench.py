@@ -49,13 +49,16 @@ FALLBACK_HBM_GBS = 6800.0
 # DRAM traffic of one launch of the batched commit kernel, from an ncu capture of the
 # same workload (see profiles/commit_batch_p25m_n100.md).  Valid only for the kernel
 # source it was taken on; reported as null once that source changes.
-NCU_TRAFFIC_BYTES_PER_LAUNCH = 40_834_628_608   # mean of two full-size launches
-NCU_TRAFFIC_SOURCE_SHA = "0797a90967922f98"
+NCU_TRAFFIC_BYTES_PER_LAUNCH = 40_833_791_360   # mean of two full-size launches
+NCU_TRAFFIC_SOURCE_SHA = "c2e30690f811f1b4"
 
 
 def kernel_source_sha() -> str:
-    src = ROOT / "paper_1805_08469_gb300" / "csrc" / "gem_commit.cu"
-    return hashlib.sha256(src.read_bytes()).hexdigest()[:16]
+    """Hash of the commit kernel's sources (the kernel and its argument block)."""
+    h = hashlib.sha256()
+    for name in ("gem_commit.cu", "gem_internal.h"):
+        h.update((ROOT / "paper_1805_08469_gb300" / "csrc" / name).read_bytes())
+    return h.hexdigest()[:16]
 
 
 def measured_peaks() -> tuple[float, str]:

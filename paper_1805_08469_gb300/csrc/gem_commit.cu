@@ -129,10 +129,15 @@ __device__ __forceinline__ void commit_vec_fixed(float4& th, float4& s, const fl
 // A worker that commits again later in the launch can keep its m_w, s_w lanes on chip:
 // each thread owns lanes slot_mem[(2 slot + {0: m, 1: s}) L kThreads + l kThreads + tid]
 // of dynamic shared memory, so no synchronisation is needed.
-template <int L, int RULE, bool REC>
+template <int L, int RULE, bool REC, int KCAP>
 __global__ void __launch_bounds__(kThreads, RULE == kRuleScaled ? 2 : GEM_COMMIT_MIN_BLOCKS)
-commit_batch_kernel(const __grid_constant__ BatchArgs a) {
+commit_batch_kernel(const __grid_constant__ BatchArgsT<KCAP> a) {
   extern __shared__ float4 slot_mem[];
+  // Launched as a programmatic dependent of the previous kernel in the stream: wait until
+  // that grid has completed and its writes are visible (theta, m_w and s_w may be the ones
+  // it wrote), then let the next commit launch start its own setup early.
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   const size_t nvec = a.P >> 2;
   const size_t nthreads = size_t(gridDim.x) * kThreads;
   const size_t tid = size_t(blockIdx.x) * kThreads + threadIdx.x;
@@ -248,26 +253,31 @@ commit_batch_kernel(const __grid_constant__ BatchArgs a) {
 
 constexpr int kLanes = GEM_COMMIT_LANES;
 
-template <int RULE, bool REC>
-cudaError_t launch_rule(const BatchArgs& a, int sm_count, cudaStream_t stream) {
-  constexpr int smem = RULE == kRuleFixed ? 0 : kCommitSlots * 2 * kLanes * kThreads * 16;
-  static int blocks_per_sm = 0;
-  if (blocks_per_sm == 0) {
+// One launch of the kernel instantiation for KCAP commits.  The slot shared memory is
+// requested only when the launch keeps a worker on chip; without it more blocks fit on an
+// SM.  Occupancy is computed once per instantiation and shared-memory size.
+template <int RULE, bool REC, int KCAP>
+cudaError_t launch_kernel(const BatchArgsT<KCAP>& a, bool slots, int sm_count, cudaStream_t stream) {
+  const int smem = slots ? kCommitSlots * 2 * kLanes * kThreads * 16 : 0;
+  static int blocks_per_sm[2] = {0, 0};
+  int& bps = blocks_per_sm[slots ? 1 : 0];
+  if (bps == 0) {
     if (smem > 48 * 1024) {
-      cudaError_t e = cudaFuncSetAttribute(commit_batch_kernel<kLanes, RULE, REC>,
+      cudaError_t e = cudaFuncSetAttribute(commit_batch_kernel<kLanes, RULE, REC, KCAP>,
                                            cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
       if (e != cudaSuccess) return e;
     }
+    int b = 0;
     cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(
-        &blocks_per_sm, commit_batch_kernel<kLanes, RULE, REC>, kThreads, smem);
+        &b, commit_batch_kernel<kLanes, RULE, REC, KCAP>, kThreads, smem);
     if (e != cudaSuccess) return e;
-    if (GEM_COMMIT_MAX_BLOCKS_PER_SM > 0 && blocks_per_sm > GEM_COMMIT_MAX_BLOCKS_PER_SM)
-      blocks_per_sm = GEM_COMMIT_MAX_BLOCKS_PER_SM;
-    if (blocks_per_sm < 1) blocks_per_sm = 1;
+    if (GEM_COMMIT_MAX_BLOCKS_PER_SM > 0 && b > GEM_COMMIT_MAX_BLOCKS_PER_SM)
+      b = GEM_COMMIT_MAX_BLOCKS_PER_SM;
+    bps = b < 1 ? 1 : b;
   }
   const size_t nvec = a.P >> 2;
   const size_t per_block = size_t(kThreads) * kLanes;
-  const size_t max_grid = size_t(sm_count) * size_t(blocks_per_sm);
+  const size_t max_grid = size_t(sm_count) * size_t(bps);
   size_t grid = (nvec + per_block - 1) / per_block;
   if (grid > max_grid) {
     // Same number of rounds per thread as the full resident grid, with the grid trimmed
@@ -276,8 +286,49 @@ cudaError_t launch_rule(const BatchArgs& a, int sm_count, cudaStream_t stream) {
     grid = (nvec + rounds * per_block - 1) / (rounds * per_block);
   }
   if (grid < 1) grid = 1;
-  commit_batch_kernel<kLanes, RULE, REC><<<unsigned(grid), kThreads, smem, stream>>>(a);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(unsigned(grid));
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = size_t(smem);
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, commit_batch_kernel<kLanes, RULE, REC, KCAP>, a);
+}
+
+template <int RULE, bool REC>
+cudaError_t launch_rule(const BatchArgs& a, int sm_count, cudaStream_t stream) {
+  bool slots = false;
+  if (RULE != kRuleFixed)
+    for (int k = 0; k < a.K; ++k) slots = slots || a.slot_out[k] >= 0;
+  if (a.K > kSmallBatch) return launch_kernel<RULE, REC, kMaxBatchPerLaunch>(a, slots, sm_count, stream);
+  BatchArgsT<kSmallBatch> b;
+  b.theta = a.theta;
+  b.m = a.m;
+  b.s = a.s;
+  b.P = a.P;
+  b.stride = a.stride;
+  b.eta = a.eta;
+  b.mu = a.mu;
+  b.eps = a.eps;
+  b.K = a.K;
+  b.rule = a.rule;
+  b.energy_scale = a.energy_scale;
+  b.record_pi = a.record_pi;
+  for (int k = 0; k < kSmallBatch; ++k) {
+    const bool in = k < a.K;
+    b.grad[k] = in ? a.grad[k] : nullptr;
+    b.worker[k] = in ? a.worker[k] : 0;
+    b.pi[k] = in ? a.pi[k] : 0.f;
+    b.pi_out[k] = in ? a.pi_out[k] : nullptr;
+    b.slot_in[k] = in ? a.slot_in[k] : int8_t(-1);
+    b.slot_out[k] = in ? a.slot_out[k] : int8_t(-1);
+    b.keep_s[k] = in ? a.keep_s[k] : uint8_t(1);
+  }
+  return launch_kernel<RULE, REC, kSmallBatch>(b, slots, sm_count, stream);
 }
 
 }  // namespace

@@ -30,30 +30,36 @@ enum RuleKind : int {
   kRuleMomentum = 3,  // the proxy itself: theta += (m_w <- mu m_w + dtheta); no factor
 };
 
-struct BatchArgs {
+// Arguments of one launch of the fused commit kernel, for up to KCAP commits.  Launches of
+// at most kSmallBatch commits (single commits, the segments of the simulators) pass the
+// small form: the kernel parameters then take about 1 KB instead of 5.5 KB.
+template <int KCAP>
+struct BatchArgsT {
   float* theta;                            // [stride]
   float* m;                                // [n][stride]
   float* s;                                // [n][stride]
   size_t P;
   size_t stride;
   float eta, mu, eps;
-  int K;                                   // commits in this launch, 1..kMaxBatchPerLaunch
+  int K;                                   // commits in this launch, 1..KCAP
   int rule;                                // RuleKind
   float energy_scale;                      // kRuleScaled: factor on |m_w|
-  const float* grad[kMaxBatchPerLaunch];   // gradient of commit k, P floats
-  int worker[kMaxBatchPerLaunch];          // worker of commit k
-  float pi[kMaxBatchPerLaunch];            // kRuleFixed: scaling factor of commit k
+  const float* grad[KCAP];                 // gradient of commit k, P floats
+  int worker[KCAP];                        // worker of commit k
+  float pi[KCAP];                          // kRuleFixed: scaling factor of commit k
   int record_pi;                           // 1: pi_out[k] (when not null) receives pi
-  float* pi_out[kMaxBatchPerLaunch];       // scaling factors of commit k, P floats, or null
+  float* pi_out[KCAP];                     // scaling factors of commit k, P floats, or null
   // On-chip reuse of a worker that commits again later in the launch (energy rules):
   // commit k keeps its m_w, s_w lanes in shared-memory slot slot_out[k] instead of writing
   // them to global memory, and the worker's next commit reads them from slot_in[k];
   // -1 means global memory.  Fixed-factor rules: keep_s[k] = 0 skips the store of s_w
   // when the worker commits again in the launch (nothing reads it before that).
-  int8_t slot_in[kMaxBatchPerLaunch];
-  int8_t slot_out[kMaxBatchPerLaunch];
-  uint8_t keep_s[kMaxBatchPerLaunch];
+  int8_t slot_in[KCAP];
+  int8_t slot_out[KCAP];
+  uint8_t keep_s[KCAP];
 };
+using BatchArgs = BatchArgsT<kMaxBatchPerLaunch>;
+constexpr int kSmallBatch = 32;
 
 // Shared-memory slots of the commit kernel (m_w and s_w lanes of one worker per slot), and
 // the shortest repeat distance (in commits) given a slot: shorter repeats are served by L2.
