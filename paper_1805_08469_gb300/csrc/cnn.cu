@@ -25,6 +25,7 @@
 #include "../../include/gem_sim.h"
 #include "gem_internal.h"
 #include "mlp_internal.h"
+#include "pdl.h"
 
 struct gem_cnn;
 
@@ -144,6 +145,7 @@ __device__ __forceinline__ void stage_wait() {
 // when known at compile time (the paper's network: 28), 0 reads it from the arguments.
 template <int HC>
 __global__ void __launch_bounds__(kThreads) conv1_pool_kernel(const __grid_constant__ ConvArgs a) {
+  gem::pdl_entry();
   extern __shared__ float sm[];
   const long long gi = blockIdx.x;
   const int g = int(gi / a.b), i = int(gi % a.b);
@@ -191,6 +193,7 @@ __global__ void __launch_bounds__(kThreads) conv1_pool_kernel(const __grid_const
 constexpr int kPool2Threads = 320;
 template <int P1C>
 __global__ void __launch_bounds__(kPool2Threads) conv2_pool_kernel(const __grid_constant__ ConvArgs a) {
+  gem::pdl_entry();
   extern __shared__ float sm[];
   const long long gi = blockIdx.x;
   const int g = int(gi / a.b), i = int(gi % a.b);
@@ -242,6 +245,7 @@ __global__ void __launch_bounds__(kPool2Threads) conv2_pool_kernel(const __grid_
 // Gradient into conv2's (pre-dropout) output: the feature gradient through the ReLU, to
 // the window's first maximum, times the channel's dropout scale; zeros elsewhere.
 __global__ void __launch_bounds__(kThreads) pool2_back_kernel(const __grid_constant__ ConvArgs a) {
+  gem::pdl_entry();
   const long long total = (long long)a.G * a.b * a.c2 * a.P2 * a.P2;
   const long long q = blockIdx.x * (long long)kThreads + threadIdx.x;
   if (q >= total) return;
@@ -281,6 +285,7 @@ constexpr int kBackThreads = 128;
 // kernel rows.
 template <int H2C, int P1C>
 __global__ void __launch_bounds__(kBackThreads) conv2_back_kernel(const __grid_constant__ ConvArgs a) {
+  gem::pdl_entry();
   extern __shared__ float sm[];
   const long long gi = blockIdx.x;
   const int g = int(gi / a.b), i = int(gi % a.b);
@@ -356,6 +361,7 @@ __global__ void __launch_bounds__(kBackThreads) conv2_back_kernel(const __grid_c
 // H2C, P1C as in conv2_back_kernel.
 template <int H2C, int P1C>
 __global__ void __launch_bounds__(kThreads) conv2_wpart_kernel(const __grid_constant__ ConvArgs a) {
+  gem::pdl_entry();
   extern __shared__ float sm[];
   const long long gi = blockIdx.x;
   const int g = int(gi / a.b), i = int(gi % a.b);
@@ -413,6 +419,7 @@ __global__ void __launch_bounds__(kThreads) conv2_wpart_kernel(const __grid_cons
 constexpr int kW1Threads = 64;
 template <int H1C, int HC>
 __global__ void __launch_bounds__(kW1Threads) conv1_wpart_kernel(const __grid_constant__ ConvArgs a) {
+  gem::pdl_entry();
   extern __shared__ float sm[];
   const long long gi = blockIdx.x;
   const int g = int(gi / a.b), i = int(gi % a.b);
@@ -463,6 +470,7 @@ __global__ void __launch_bounds__(kW1Threads) conv1_wpart_kernel(const __grid_co
 
 // Convolution gradients: the partials summed over the minibatch in sample order.
 __global__ void __launch_bounds__(kThreads) conv_finish_kernel(const __grid_constant__ ConvArgs a) {
+  gem::pdl_entry();
   const int per1 = kK * kK + 1, per2 = a.c1 * kK * kK + 1;
   const long long n1 = (long long)a.c1 * per1, n2 = (long long)a.c2 * per2;
   const long long total = (long long)a.G * (n1 + n2);
@@ -544,29 +552,28 @@ int cnn_chunk(gem_cnn* N, const int32_t* workers, int G, const int32_t* rows_dev
   int rc;
   const unsigned samples = unsigned(G * b);
   if (s.H == 28) {
-    conv1_pool_kernel<28><<<samples, kThreads, N->smem[0], st>>>(a);
-    conv2_pool_kernel<12><<<samples, kPool2Threads, N->smem[1], st>>>(a);
+    gem::launch_pdl(conv1_pool_kernel<28>, samples, kThreads, N->smem[0], st, a);
+    gem::launch_pdl(conv2_pool_kernel<12>, samples, kPool2Threads, N->smem[1], st, a);
   } else {
-    conv1_pool_kernel<0><<<samples, kThreads, N->smem[0], st>>>(a);
-    conv2_pool_kernel<0><<<samples, kPool2Threads, N->smem[1], st>>>(a);
+    gem::launch_pdl(conv1_pool_kernel<0>, samples, kThreads, N->smem[0], st, a);
+    gem::launch_pdl(conv2_pool_kernel<0>, samples, kPool2Threads, N->smem[1], st, a);
   }
   if ((rc = cuda_rc(cudaGetLastError()))) return rc;
   N->launches += 2;
   // the dense head: forward, loss, backward, and the feature gradient
   if ((rc = gem::mlp::mlp_chunk(N->head, workers, G, rows_dev, grads, grad_stride, losses))) return rc;
-  pool2_back_kernel<<<blocks_for(n_pool2), kThreads, 0, st>>>(a);
+  gem::launch_pdl(pool2_back_kernel, blocks_for(n_pool2), kThreads, 0, st, a);
   if (s.H == 28) {   // the paper's map sizes: loop bounds known at compile time
-    conv2_back_kernel<8, 12><<<samples, kBackThreads, N->smem[2], st>>>(a);
-    conv2_wpart_kernel<8, 12><<<samples, kThreads, N->smem[3], st>>>(a);
-    conv1_wpart_kernel<24, 28><<<samples, kW1Threads, N->smem[4], st>>>(a);
+    gem::launch_pdl(conv2_back_kernel<8, 12>, samples, kBackThreads, N->smem[2], st, a);
+    gem::launch_pdl(conv2_wpart_kernel<8, 12>, samples, kThreads, N->smem[3], st, a);
+    gem::launch_pdl(conv1_wpart_kernel<24, 28>, samples, kW1Threads, N->smem[4], st, a);
   } else {
-    conv2_back_kernel<0, 0><<<samples, kBackThreads, N->smem[2], st>>>(a);
-    conv2_wpart_kernel<0, 0><<<samples, kThreads, N->smem[3], st>>>(a);
-    conv1_wpart_kernel<0, 0><<<samples, kW1Threads, N->smem[4], st>>>(a);
+    gem::launch_pdl(conv2_back_kernel<0, 0>, samples, kBackThreads, N->smem[2], st, a);
+    gem::launch_pdl(conv2_wpart_kernel<0, 0>, samples, kThreads, N->smem[3], st, a);
+    gem::launch_pdl(conv1_wpart_kernel<0, 0>, samples, kW1Threads, N->smem[4], st, a);
   }
-  conv_finish_kernel<<<blocks_for(G * ((long long)s.c1 * (kK * kK + 1) +
-                                       (long long)s.c2 * (s.c1 * kK * kK + 1))),
-                       kThreads, 0, st>>>(a);
+  gem::launch_pdl(conv_finish_kernel, blocks_for(G * ((long long)s.c1 * (kK * kK + 1) +
+                                       (long long)s.c2 * (s.c1 * kK * kK + 1))), kThreads, 0, st, a);
   if ((rc = cuda_rc(cudaGetLastError()))) return rc;
   N->launches += 5;
   return GEM_OK;

@@ -28,6 +28,7 @@
 #include "../../include/gem_sim.h"
 #include "gem_internal.h"
 #include "mlp_internal.h"
+#include "pdl.h"
 
 namespace gem {
 namespace mlp {
@@ -96,6 +97,7 @@ __device__ __forceinline__ float to_tf32(float x) {
 template <int TBM, bool A_KMAJOR, bool B_KMAJOR, int EPI, bool TF32>
 __global__ void __launch_bounds__(2 * TBM)
 gemm_grouped_kernel(const __grid_constant__ GemmArgs p) {
+  gem::pdl_entry();
   constexpr int T = 2 * TBM;                 // threads: 16 columns x TBM / 8 rows of them
   constexpr int kPadA = TBM + 4, kPadB = BN + 4;  // row pitches (floats), 16-byte aligned
   constexpr int kBPer = BN * BK / T;         // B elements staged per thread (A: always 8)
@@ -241,6 +243,7 @@ __device__ __forceinline__ void mma_tf32(float (&c)[4], const uint32_t (&a)[4], 
 template <int TBN, bool A_KMAJOR, bool B_KMAJOR, int EPI>
 __global__ void __launch_bounds__(256)
 gemm_mma_tf32_kernel(const __grid_constant__ GemmArgs p) {
+  gem::pdl_entry();
   constexpr int kT = 256;
   constexpr int kWN = TBN / 4;            // columns per warp
   constexpr int kNT = kWN / 8;            // n8 tiles per warp
@@ -479,6 +482,7 @@ __device__ __forceinline__ void ldsm_x4(uint32_t (&r)[4], const float* row_addr)
 template <int TBN, bool A_KMAJOR, bool B_KMAJOR, int EPI>
 __global__ void __launch_bounds__(256)
 gemm_mma_pipe_kernel(const __grid_constant__ GemmArgs p) {
+  gem::pdl_entry();
   constexpr int kWN = TBN / 4, kNT = kWN / 8;
   constexpr int kAF = pipe_tile_floats(kMmaBM, A_KMAJOR), kBF = pipe_tile_floats(TBN, B_KMAJOR);
   constexpr int kStageF = kAF + kBF;
@@ -604,6 +608,7 @@ gemm_mma_pipe_kernel(const __grid_constant__ GemmArgs p) {
 // epilogue of the product.
 template <int EPI, int V>
 __global__ void __launch_bounds__(256) splitk_reduce_kernel(const __grid_constant__ GemmArgs p) {
+  gem::pdl_entry();
   // one output row (g, m) per blockIdx.y; thread t of blockIdx.x covers V consecutive columns
   const int M = p.M, N = p.N;
   const int g = blockIdx.y / M, m = blockIdx.y - g * M;
@@ -658,6 +663,7 @@ __global__ void __launch_bounds__(256) splitk_reduce_kernel(const __grid_constan
 template <bool TF32>
 __global__ void __launch_bounds__(256)
 gemm_small_n_kernel(const __grid_constant__ GemmArgs p, int rows_per_block) {
+  gem::pdl_entry();
   extern __shared__ __align__(16) float Bsm[];
   const int g = blockIdx.y;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -742,7 +748,7 @@ bool launch_small_n(const GemmArgs& a, int groups, cudaStream_t st, cudaError_t*
   rows_per_block = rows_per_block < 8 ? 8 : (rows_per_block + 7) / 8 * 8;
   const int rpb = int(rows_per_block);
   dim3 grid(unsigned((a.M + rpb - 1) / rpb), unsigned(groups));
-  gemm_small_n_kernel<TF32><<<grid, 256, bytes, st>>>(a, rpb);
+  gem::launch_pdl(gemm_small_n_kernel<TF32>, grid, 256, bytes, st, a, rpb);
   *err = cudaGetLastError();
   return true;
 }
@@ -750,6 +756,7 @@ bool launch_small_n(const GemmArgs& a, int groups, cudaStream_t st, cudaError_t*
 // Minibatch gather: slot g's rows X[batch_rows[g][r]] -> Xs[g][r][:].
 __global__ void gather_rows_kernel(const float* X, int d0, const int32_t* batch_rows, int b,
                                    float* Xs, long long slot_stride) {
+  gem::pdl_entry();
   const int g = blockIdx.y, r = blockIdx.x;
   const long long row = batch_rows[(long long)g * b + r];
   const float* src = X + row * d0;
@@ -762,6 +769,7 @@ __global__ void gather_rows_kernel(const float* X, int d0, const int32_t* batch_
 __global__ void softmax_xent_kernel(const float* logits, float* delta, long long slot_stride,
                                    int b, int C, const int32_t* labels,
                                    const int32_t* batch_rows, float* losses) {
+  gem::pdl_entry();
   __shared__ float row_loss[kMaxBatch];
   const int g = blockIdx.x;
   const float* z = logits + g * slot_stride;
@@ -807,6 +815,7 @@ struct BiasGradArgs {
 __global__ void __launch_bounds__(256)
 bias_grad_kernel(const __grid_constant__ BiasGradArgs a, const float* delta,
                  long long slot_stride, float* grad, long long grad_stride) {
+  gem::pdl_entry();
   __shared__ float part[8][33];
   const int g = blockIdx.y;
   const int x = threadIdx.x & 31, y = threadIdx.x >> 5;
@@ -833,9 +842,9 @@ template <int TBM, bool AK, bool BK_, int EPI>
 void launch_tile(const GemmArgs& a, int groups, bool tf32, cudaStream_t st) {
   dim3 grid((a.N + BN - 1) / BN, (a.M + TBM - 1) / TBM, groups);
   if (tf32)
-    gemm_grouped_kernel<TBM, AK, BK_, EPI, true><<<grid, 2 * TBM, 0, st>>>(a);
+    gem::launch_pdl(gemm_grouped_kernel<TBM, AK, BK_, EPI, true>, grid, 2 * TBM, 0, st, a);
   else
-    gemm_grouped_kernel<TBM, AK, BK_, EPI, false><<<grid, 2 * TBM, 0, st>>>(a);
+    gem::launch_pdl(gemm_grouped_kernel<TBM, AK, BK_, EPI, false>, grid, 2 * TBM, 0, st, a);
 }
 
 bool operand_16b(const Operand& o) {
@@ -857,9 +866,9 @@ void launch_mma(const GemmArgs& a, int groups, cudaStream_t st) {
         return;   // the error is reported by the caller's cudaGetLastError
       if (dev >= 0 && dev < 64) configured[dev] = true;
     }
-    gemm_mma_pipe_kernel<TBN, AK, BK_, EPI><<<grid, 256, bytes, st>>>(a);
+    gem::launch_pdl(gemm_mma_pipe_kernel<TBN, AK, BK_, EPI>, grid, 256, bytes, st, a);
   } else {
-    gemm_mma_tf32_kernel<TBN, AK, BK_, EPI><<<grid, 256, 0, st>>>(a);
+    gem::launch_pdl(gemm_mma_tf32_kernel<TBN, AK, BK_, EPI>, grid, 256, 0, st, a);
   }
 }
 
@@ -913,9 +922,9 @@ cudaError_t launch_gemm(const GemmArgs& a_in, int groups, bool tf32, cudaStream_
     const int V = vec ? 4 : 1;
     dim3 grid(unsigned((a.N + 256 * V - 1) / (256 * V)), unsigned(a.M * groups));
     if (vec)
-      splitk_reduce_kernel<EPI, 4><<<grid, 256, 0, st>>>(a);
+      gem::launch_pdl(splitk_reduce_kernel<EPI, 4>, grid, 256, 0, st, a);
     else
-      splitk_reduce_kernel<EPI, 1><<<grid, 256, 0, st>>>(a);
+      gem::launch_pdl(splitk_reduce_kernel<EPI, 1>, grid, 256, 0, st, a);
   }
   return cudaGetLastError();
 }
@@ -951,7 +960,7 @@ int mlp_chunk(gem_mlp* M, const int32_t* workers, int G, const int32_t* batch_ro
 
   int rc = GEM_OK;
   if (!M->external_input) {
-    gather_rows_kernel<<<dim3(b, G), 256, 0, st>>>(M->X, M->dims[0], batch_rows, b,
+    gem::launch_pdl(gather_rows_kernel, dim3(b, G), 256, 0, st, M->X, M->dims[0], batch_rows, b,
                                                    scr + M->off_x, S);
     if ((rc = cuda_rc(cudaGetLastError()))) return rc;
     M->launches++;
@@ -987,7 +996,7 @@ int mlp_chunk(gem_mlp* M, const int32_t* workers, int G, const int32_t* batch_ro
     if ((rc = cuda_rc(e))) return rc;
     M->launches++;
   }
-  softmax_xent_kernel<<<G, 128, 0, st>>>(scr + M->off_logits, scr + M->off_delta[L], S, b,
+  gem::launch_pdl(softmax_xent_kernel, G, 128, 0, st, scr + M->off_logits, scr + M->off_delta[L], S, b,
                                          M->dims[L], M->labels, batch_rows, losses);
   if ((rc = cuda_rc(cudaGetLastError()))) return rc;
   M->launches++;
@@ -1051,7 +1060,7 @@ int mlp_chunk(gem_mlp* M, const int32_t* workers, int G, const int32_t* batch_ro
     ba.width[l] = M->dims[l + 1];
     ba.first[l + 1] = ba.first[l] + M->dims[l + 1];
   }
-  bias_grad_kernel<<<dim3((ba.first[L] + 31) / 32, G), 256, 0, st>>>(ba, scr, S, grads,
+  gem::launch_pdl(bias_grad_kernel, dim3((ba.first[L] + 31) / 32, G), 256, 0, st, ba, scr, S, grads,
                                                                       grad_stride);
   if ((rc = cuda_rc(cudaGetLastError()))) return rc;
   M->launches++;

@@ -21,6 +21,7 @@
 #include <cmath>
 
 #include "gem_internal.h"
+#include "pdl.h"
 
 namespace gem {
 namespace {
@@ -56,6 +57,7 @@ __device__ __forceinline__ float key_value(unsigned k) {
 }
 
 __global__ void select_init_kernel(const __grid_constant__ SelectArgs a) {
+  gem::pdl_entry();
   const int q = blockIdx.x * blockDim.x + threadIdx.x;     // problem k * nseg + s
   if (q >= a.K * a.nseg) return;
   const int s = q % a.nseg;
@@ -79,6 +81,7 @@ __device__ __forceinline__ void count_digit(unsigned* h, bool valid, unsigned ke
 }
 
 __global__ void __launch_bounds__(kThreads) select_hist_kernel(const __grid_constant__ SelectArgs a) {
+  gem::pdl_entry();
   __shared__ unsigned h[2 * kBins];
   const int b = blockIdx.x, k = blockIdx.y;
   int s = 0;
@@ -122,6 +125,7 @@ __global__ void __launch_bounds__(kThreads) select_hist_kernel(const __grid_cons
 }
 
 __global__ void __launch_bounds__(kThreads) select_pick_kernel(const __grid_constant__ SelectArgs a) {
+  gem::pdl_entry();
   constexpr int kPer = kBins / kThreads;     // bins per thread (8)
   __shared__ unsigned wsum[kThreads / 32];
   __shared__ unsigned sst[6];
@@ -221,15 +225,15 @@ cudaError_t pi_median_ordered(gem_ctx* h, const float* const* pi, int K, const i
     cudaError_t e = cudaMemsetAsync(a.hist, 0, size_t(kc) * nseg * 2 * kBins * sizeof(unsigned),
                                     h->stream);
     if (e != cudaSuccess) return e;
-    select_init_kernel<<<(kc * nseg + 127) / 128, 128, 0, h->stream>>>(a);
+    gem::launch_pdl(select_init_kernel, (kc * nseg + 127) / 128, 128, 0, h->stream, a);
     h->launches += 1;
     for (int p = 0; p < kPasses; ++p) {
       a.pass = p;
       if (blocks > 0) {
-        select_hist_kernel<<<dim3(unsigned(blocks), unsigned(kc)), kThreads, 0, h->stream>>>(a);
+        gem::launch_pdl(select_hist_kernel, dim3(unsigned(blocks), unsigned(kc)), kThreads, 0, h->stream, a);
         h->launches += 1;
       }
-      select_pick_kernel<<<unsigned(kc * nseg), kThreads, 0, h->stream>>>(a);
+      gem::launch_pdl(select_pick_kernel, unsigned(kc * nseg), kThreads, 0, h->stream, a);
       h->launches += 1;
     }
     e = cudaGetLastError();
