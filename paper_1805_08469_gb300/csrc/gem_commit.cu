@@ -135,9 +135,8 @@ commit_batch_kernel(const __grid_constant__ BatchArgsT<KCAP> a) {
   extern __shared__ float4 slot_mem[];
   // Launched as a programmatic dependent of the previous kernel in the stream: wait until
   // that grid has completed and its writes are visible (theta, m_w and s_w may be the ones
-  // it wrote), then let the next commit launch start its own setup early.
+  // it wrote).  The next launch is scheduled when this grid's blocks have exited.
   asm volatile("griddepcontrol.wait;" ::: "memory");
-  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   const size_t nvec = a.P >> 2;
   const size_t nthreads = size_t(gridDim.x) * kThreads;
   const size_t tid = size_t(blockIdx.x) * kThreads + threadIdx.x;
