@@ -199,10 +199,12 @@ int gem_commit_batch_pi(gem_t* h, const int* order, const float* const* grads, i
  * N / 2 (the same for odd N; their mean is the usual median); NaN for an empty segment.
  * pi is a host array of K device pointers (4-byte aligned); seg is a host array of nseg + 1
  * offsets with 0 <= seg[0] <= ... <= seg[nseg] <= P, 1 <= nseg <= 64; lo and hi are device
- * arrays of K * nseg floats.  Stream-ordered: three passes over the rows (radix selection,
- * 11 + 11 + 10 bits of an order-preserving key).  The first call, and any call with more
- * rows or segments than before (up to 200 rows per pass), allocates the select scratch:
- * 16 KB per row and segment. */
+ * arrays of K * nseg floats.  "Sorted" is the total order of the float bits: -0 below +0,
+ * NaNs with the sign bit set below everything, other NaNs above.  Stream-ordered: up to
+ * three passes over the rows (radix selection, 11 + 11 + 10 bits of an order-preserving
+ * key; a median that falls in a run of exact +0, as clamped factors give, is resolved by
+ * the first pass).  The first call, and any call with more rows or segments than before
+ * (up to 200 rows per pass), allocates the select scratch: 16 KB per row and segment. */
 int gem_pi_median(gem_t* h, const float* const* pi, int K, const int64_t* seg, int nseg,
                   float* lo, float* hi);
 

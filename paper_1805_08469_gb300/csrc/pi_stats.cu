@@ -18,6 +18,13 @@
 //     histogram for the next pass.
 // After the third pass the prefix is the target's key, which maps back to its float.
 // Each pass reads the factors once (4 bytes per element), so 12 bytes per element.
+// Runs of exact zeros: pi = max(0, .) makes +0 common (at P = 25M often more than half of
+// a commit's factors), and then every pass funnels those elements into one bin.  The first
+// pass therefore counts the elements equal to +0 apart (in word kBins of the histogram,
+// which the first pass does not otherwise use); every smaller key lies in the bins below
+// +0's first-pass bin, so a target whose rank falls in the run of zeros is resolved after
+// one pass (its mask becomes full), and later passes skip it, and skip a problem whose
+// targets are both resolved.
 #include <cmath>
 
 #include "gem_internal.h"
@@ -31,6 +38,8 @@ constexpr int kBins = 2048;                 // 11-bit digits (the last pass uses
 constexpr int kUnroll = 8;                  // independent loads per thread and step
 constexpr int kChunk = kThreads * kUnroll * 8;   // elements per histogram block
 constexpr int kPasses = 3;
+constexpr int kState = 6;                   // per problem: two (prefix, mask, rank)
+constexpr unsigned kZeroKey = 0x80000000u;  // order_key(+0.0f)
 
 __host__ __device__ constexpr int digit_shift(int pass) { return pass == 0 ? 21 : (pass == 1 ? 10 : 0); }
 __host__ __device__ constexpr int digit_bits(int pass) { return pass == 2 ? 10 : 11; }
@@ -41,7 +50,7 @@ struct SelectArgs {
   int block_start[kMaxPiSegments + 1];      // first histogram block of each segment
   int K, nseg, pass;
   unsigned* hist;                           // [K][nseg][2][kBins]
-  unsigned* state;                          // [K][nseg][2][3]: prefix, mask, rank
+  unsigned* state;                          // [K][nseg][kState]: 2 x (prefix, mask, rank)
   float* lo;                                // [K][nseg]
   float* hi;                                // [K][nseg]
 };
@@ -62,7 +71,7 @@ __global__ void select_init_kernel(const __grid_constant__ SelectArgs a) {
   if (q >= a.K * a.nseg) return;
   const int s = q % a.nseg;
   const long long N = a.seg[s + 1] - a.seg[s];
-  unsigned* st = a.state + size_t(q) * 6;
+  unsigned* st = a.state + size_t(q) * kState;
   st[0] = 0u;
   st[1] = 0u;
   st[2] = N > 0 ? unsigned((N - 1) / 2) : 0u;
@@ -72,14 +81,17 @@ __global__ void select_init_kernel(const __grid_constant__ SelectArgs a) {
 }
 
 // Adds one element's digit to a shared histogram when its key matches the prefix; every
-// lane of the warp must call it (the match is warp-wide).
+// lane of the warp must call it (the match is warp-wide).  FIRST: the first pass, whose
+// prefix is empty, so that every element matches.
+template <bool FIRST>
 __device__ __forceinline__ void count_digit(unsigned* h, bool valid, unsigned key, unsigned prefix,
                                             unsigned mask, unsigned digit, int lane) {
-  const unsigned bin = (valid && (key & mask) == prefix) ? digit : 0xffffffffu;
+  const unsigned bin = (valid && (FIRST || (key & mask) == prefix)) ? digit : 0xffffffffu;
   const unsigned peers = __match_any_sync(0xffffffffu, bin);
   if (bin != 0xffffffffu && lane == __ffs(peers) - 1) atomicAdd(h + bin, unsigned(__popc(peers)));
 }
 
+template <bool FIRST>
 __global__ void __launch_bounds__(kThreads) select_hist_kernel(const __grid_constant__ SelectArgs a) {
   gem::pdl_entry();
   __shared__ unsigned h[2 * kBins];
@@ -87,9 +99,12 @@ __global__ void __launch_bounds__(kThreads) select_hist_kernel(const __grid_cons
   int s = 0;
   while (b >= a.block_start[s + 1]) ++s;
   const int q = k * a.nseg + s;
-  const unsigned* st = a.state + size_t(q) * 6;
+  const unsigned* st = a.state + size_t(q) * kState;
   const unsigned p0 = st[0], m0 = st[1], p1 = st[3], m1 = st[4];
+  const bool done0 = m0 == 0xffffffffu, done1 = m1 == 0xffffffffu;
+  if (done0 && done1) return;               // both targets resolved: nothing to count
   const bool two = p0 != p1 || m0 != m1;
+  const bool need0 = !done0, need1 = two && !done1;
   for (int i = threadIdx.x; i < 2 * kBins; i += kThreads) h[i] = 0u;
   __syncthreads();
 
@@ -111,13 +126,17 @@ __global__ void __launch_bounds__(kThreads) select_hist_kernel(const __grid_cons
     for (int u = 0; u < kUnroll; ++u) {
       const bool valid = base + u * kThreads + threadIdx.x < end;
       const unsigned d = (key[u] >> shift) & dmask;
-      count_digit(h, valid, key[u], p0, m0, d, lane);
-      if (two) count_digit(h + kBins, valid, key[u], p1, m1, d, lane);
+      if (FIRST) {
+        count_digit<true>(h, valid, key[u], 0u, 0u, key[u] == kZeroKey ? unsigned(kBins) : d, lane);
+      } else {
+        if (need0) count_digit<false>(h, valid, key[u], p0, m0, d, lane);
+        if (need1) count_digit<false>(h + kBins, valid, key[u], p1, m1, d, lane);
+      }
     }
   }
   __syncthreads();
   unsigned* g = a.hist + size_t(q) * 2 * kBins;
-  const int used = two ? 2 * kBins : kBins;
+  const int used = FIRST ? kBins + 1 : (two ? 2 * kBins : kBins);
   for (int i = threadIdx.x; i < used; i += kThreads) {
     const unsigned c = h[i];
     if (c) atomicAdd(g + i, c);
@@ -128,14 +147,18 @@ __global__ void __launch_bounds__(kThreads) select_pick_kernel(const __grid_cons
   gem::pdl_entry();
   constexpr int kPer = kBins / kThreads;     // bins per thread (8)
   __shared__ unsigned wsum[kThreads / 32];
-  __shared__ unsigned sst[6];
+  __shared__ unsigned sst[kState];
+  __shared__ unsigned below_zero;           // first pass: elements with keys below +0
+  __shared__ unsigned zeros;                // first pass: elements equal to +0
   const int q = blockIdx.x;
   const int s = q % a.nseg;
   const long long N = a.seg[s + 1] - a.seg[s];
-  unsigned* st = a.state + size_t(q) * 6;
+  unsigned* st = a.state + size_t(q) * kState;
   unsigned* g = a.hist + size_t(q) * 2 * kBins;
-  if (threadIdx.x < 6) sst[threadIdx.x] = st[threadIdx.x];
+  if (threadIdx.x < kState) sst[threadIdx.x] = st[threadIdx.x];
+  if (threadIdx.x == 0) zeros = a.pass == 0 ? g[kBins] : 0u;
   __syncthreads();
+  const int zero_bin = int(kZeroKey >> digit_shift(0));   // +0's first-pass bin
   const bool two = sst[0] != sst[3] || sst[1] != sst[4];
   const int shift = digit_shift(a.pass);
   const unsigned nb = 1u << digit_bits(a.pass);
@@ -148,6 +171,7 @@ __global__ void __launch_bounds__(kThreads) select_pick_kernel(const __grid_cons
 #pragma unroll
     for (int j = 0; j < kPer; ++j) {
       local[j] = hh[threadIdx.x * kPer + j];
+      if (a.pass == 0 && threadIdx.x * kPer + j == zero_bin) local[j] += zeros;   // counted apart
       sum += local[j];
     }
     unsigned incl = sum;
@@ -162,7 +186,21 @@ __global__ void __launch_bounds__(kThreads) select_pick_kernel(const __grid_cons
     for (int w = 0; w < warp; ++w) before += wsum[w];
     const unsigned excl = before + incl - sum;
     const unsigned r = sst[3 * t + 2];
-    if (N > 0 && r >= excl && r - excl < sum) {
+    const bool active = sst[3 * t + 1] != 0xffffffffu;   // not resolved in an earlier pass
+    bool in_zeros = false;
+    if (a.pass == 0) {
+      // the keys below +0 fill exactly the bins below +0's bin
+      if (threadIdx.x * kPer == zero_bin) below_zero = excl;
+      __syncthreads();
+      in_zeros = N > 0 && r >= below_zero && r - below_zero < zeros;
+      if (in_zeros && threadIdx.x == 0) {
+        st[3 * t] = kZeroKey;
+        st[3 * t + 1] = 0xffffffffu;
+        st[3 * t + 2] = r - below_zero;
+        (t == 0 ? a.lo : a.hi)[q] = 0.0f;
+      }
+    }
+    if (active && !in_zeros && N > 0 && r >= excl && r - excl < sum) {
       unsigned c = excl;
       int d = 0;
 #pragma unroll
@@ -195,7 +233,7 @@ cudaError_t pi_median_ordered(gem_ctx* h, const float* const* pi, int K, const i
   if (K <= 0) return cudaSuccess;
   const int kc_max = K < kMaxPiBatch ? K : kMaxPiBatch;
   const size_t hist_bytes = size_t(kc_max) * nseg * 2 * kBins * sizeof(unsigned);
-  const size_t need = hist_bytes + size_t(kc_max) * nseg * 6 * sizeof(unsigned);
+  const size_t need = hist_bytes + size_t(kc_max) * nseg * kState * sizeof(unsigned);
   if (need > h->select_bytes) {
     cudaFree(h->select_scratch);   // waits for work still using the old buffer
     h->select_scratch = nullptr;
@@ -230,7 +268,10 @@ cudaError_t pi_median_ordered(gem_ctx* h, const float* const* pi, int K, const i
     for (int p = 0; p < kPasses; ++p) {
       a.pass = p;
       if (blocks > 0) {
-        gem::launch_pdl(select_hist_kernel, dim3(unsigned(blocks), unsigned(kc)), kThreads, 0, h->stream, a);
+        if (p == 0)
+          gem::launch_pdl(select_hist_kernel<true>, dim3(unsigned(blocks), unsigned(kc)), kThreads, 0, h->stream, a);
+        else
+          gem::launch_pdl(select_hist_kernel<false>, dim3(unsigned(blocks), unsigned(kc)), kThreads, 0, h->stream, a);
         h->launches += 1;
       }
       gem::launch_pdl(select_pick_kernel, unsigned(kc * nseg), kThreads, 0, h->stream, a);

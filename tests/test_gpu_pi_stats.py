@@ -111,6 +111,40 @@ def test_medians_of_ties_signs_and_infinities():
     _check_medians(rows, [0, P])
 
 
+def test_medians_at_the_edges_of_a_zero_run():
+    """Runs of exact +0 (the clamp of the factor) next to negatives, -0 and positives, with
+    the run ending between the lower and the upper middle element; compared bit for bit,
+    so a -0 returned for +0 (or the reverse) fails."""
+    rng = np.random.default_rng(4)
+    P = 50_000
+    pos = lambda n: (rng.exponential(size=n) + 1e-3).astype(np.float32)
+    parts = [
+        [np.zeros(25_000), pos(25_000)],                                  # lo = +0, hi > 0
+        [-pos(25_000), np.zeros(25_000)],                                 # lo < 0, hi = +0
+        [-pos(10_000), np.zeros(30_000), pos(10_000)],                    # both +0 after negatives
+        [-pos(20_000), np.full(10_000, -0.0), np.zeros(10_000), pos(10_000)],   # both -0
+        [np.full(25_000, -0.0), np.zeros(25_000)],                        # lo = -0, hi = +0
+    ]
+    rows = np.stack([rng.permutation(np.concatenate(p).astype(np.float32)) for p in parts])
+    dev = _padded(rows)
+    lo = torch.empty((len(parts), 1), device="cuda")
+    hi = torch.empty((len(parts), 1), device="cuda")
+    with gem.Gem(P, 1, ETA, MU, EPS) as G:
+        G.pi_median([dev[k, :P] for k in range(len(parts))], [0, P], lo, hi)
+        G.sync()
+    glo, ghi = lo.cpu().numpy(), hi.cpu().numpy()
+    for k in range(len(parts)):
+        # values as the oracle's sort gives them (IEEE order: -0 and +0 compare equal) ...
+        rlo, rhi = oracle.pi_median(rows[k], [0, P])
+        assert glo[k, 0] == rlo[0] and ghi[k, 0] == rhi[0], (k, glo[k], ghi[k], rlo, rhi)
+        # ... and the exact bits of the total order the library documents (-0 below +0)
+        u = rows[k].view(np.uint32)
+        keys = np.sort(np.where(u >> 31, ~u, u | np.uint32(0x80000000)))
+        back = lambda key: np.where(key >> 31, key & np.uint32(0x7FFFFFFF), ~key).astype(np.uint32)
+        assert np.float32(glo[k, 0]).view(np.uint32) == back(keys[(P - 1) // 2]), k
+        assert np.float32(ghi[k, 0]).view(np.uint32) == back(keys[P // 2]), k
+
+
 def test_medians_per_tensor_of_the_mlp_layout_and_odd_segments():
     dims = [784, 1000, 1000, 10]
     P = synth.mlp_param_count(dims)
