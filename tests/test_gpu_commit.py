@@ -268,6 +268,40 @@ def test_config5_batched_commits_sampled():
             _close(G.snapshot(w)[idx].cpu().numpy(), s[w], f"s_{w} (sampled)")
 
 
+def test_commits_read_gradients_written_by_the_kernel_just_before():
+    """Every commit launch is a programmatic dependent of the previous kernel in its
+    stream and waits for it at entry.  Here each gradient is written by a PyTorch kernel on
+    the same stream immediately before the commit that reads it, into a buffer that held
+    NaN: a commit that started reading early would see NaN or the previous gradient."""
+    P, n, T = 4_000_003, 3, 12
+    rng = np.random.default_rng(21)
+    theta0 = (0.05 * rng.standard_normal(P)).astype(np.float32)
+    base = (0.1 * rng.standard_normal((T, P))).astype(np.float32)
+    grads = base * np.float32(3.0)                       # what the device kernel writes
+    order = [int(w) for w in rng.integers(0, n, T)]
+    th, m, s = _fresh_cpu(theta0, n)
+    oracle.gem_run(th, m, s, grads, np.asarray(order, np.int32), eta=ETA, mu=MU, eps=EPS)
+
+    stream = torch.cuda.Stream()
+    src = _padded(base)
+    buf = torch.full_like(src[0], float("nan"))
+    with torch.cuda.stream(stream), gem.Gem(P, n, ETA, MU, EPS, stream=stream) as G:
+        G.set_theta(torch.from_numpy(theta0).cuda())
+        for t in range(T):
+            torch.mul(src[t], 3.0, out=buf)              # kernel on the commit's stream
+            G.commit(order[t], buf[:P])                  # single commit
+            buf.fill_(float("nan"))                      # and a kernel right after it
+        for t in range(0, T, 4):                         # batches of 4, fresh buffers
+            bufs = [torch.mul(src[t + k], 3.0) for k in range(4)]
+            G.commit_batch(order[t:t + 4], [b[:P] for b in bufs])
+        G.sync()
+        got = G.theta().cpu().numpy()
+    th2, m2, s2 = th.copy(), m.copy(), s.copy()
+    oracle.gem_run(th2, m2, s2, grads, np.asarray(order, np.int32), eta=ETA, mu=MU, eps=EPS)
+    assert np.isfinite(got).all()
+    _close(got, th2, "theta after single commits and batches fed by the previous kernel")
+
+
 def test_checkpoint_save_and_load_state():
     """gem_save_state / gem_load_state round trip (host and device buffers), then the
     resumed handle continues bit for bit like the original."""
