@@ -25,7 +25,11 @@
  *     host; a call that fails a check changes nothing and launches nothing.
  *   - Device work is asynchronous and ordered on the handle's stream (gem_set_stream;
  *     the legacy default stream until set).  A CUDA error raised by device work is
- *     reported by a later call, at the latest by gem_sync, as GEM_ECUDA.
+ *     reported by a later call, at the latest by gem_sync, as GEM_ECUDA.  Kernels are
+ *     launched as programmatic dependents of the previous kernel in the stream: each
+ *     waits, before it touches memory, until that kernel has completed and its writes
+ *     are visible, so stream order holds as for plain launches (also when captured
+ *     into a CUDA graph), while the launch itself overlaps the previous kernel.
  *   - Caller buffers are fp32, 16-byte aligned, and must stay valid and unmodified until
  *     the work that reads them has completed on the stream.  The library never keeps a
  *     caller pointer beyond that work.
