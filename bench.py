@@ -241,6 +241,43 @@ class OracleSample:
         return dt
 
 
+def oracle_mlp_rates(seconds_target: float = 4.0) -> dict:
+    """The oracle's end-to-end simulation (gradients in double, OpenMP over outputs, the
+    fp32 commit) on the first commits of each MLP workload, inputs from the host
+    generators: commits per second on the host cores."""
+    import numpy as np
+
+    import oracle
+    from paper_1805_08469_gb300 import synth
+
+    out = {}
+    for name, dims, n, b, precision, schedule, seed, _w, _t in MLP_WORKLOADS:
+        P = synth.mlp_param_count(dims)
+        sched = oracle.schedule_uniform if schedule == "uniform" else oracle.schedule_queue
+        order = np.asarray(sched(seed, n, 400)[0], np.int32)
+        batches = synth.schedule_batches(seed, order, b)
+        theta = synth.xavier_theta0(seed, dims)
+        m = np.zeros((n, P), np.float32)
+        s_ = np.tile(theta, (n, 1))
+
+        def run(t0, t1):
+            rows, inv = np.unique(batches[t0:t1], return_inverse=True)
+            X = synth.data_rows(seed, rows, dims[0])
+            y = synth.teacher_labels(seed, rows, dims[0], dims[-1])
+            local = inv.reshape(batches[t0:t1].shape).astype(np.int32)
+            start = time.perf_counter()
+            oracle.mlp_sim_run(dims, theta, m, s_, order[t0:t1], X, y, local, eta=ETA, mu=MU,
+                               eps=EPS, tf32=precision == 1)
+            return time.perf_counter() - start
+
+        dt1 = run(0, 1)
+        T = max(1, min(399, int(seconds_target / max(dt1, 1e-4))))
+        dt = run(1, 1 + T)
+        out[name] = {"commits_per_s": round(T / dt, 2), "commits": T, "seconds": round(dt, 2)}
+    out["threads"] = oracle.threads()
+    return out
+
+
 def cpu_baseline(seconds_target: float = 15.0) -> dict:
     import oracle
     sample = OracleSample(ORACLE_SAMPLE, SEED)
@@ -253,7 +290,8 @@ def cpu_baseline(seconds_target: float = 15.0) -> dict:
             "sample": f"coordinates [0, {S}) of P={P_FULL}, n={N_WORKERS}: {batches} batches of "
                       f"{K_BATCH} commits in {dt:.1f} s; same algorithmic bytes per coordinate",
             "commits_per_s_scaled_to_P": round(T / dt * S / P_FULL, 3),
-            "oracle_threads_available": oracle.threads()}
+            "oracle_threads_available": oracle.threads(),
+            "async_mlp_oracle": oracle_mlp_rates()}
 
 
 def run_reference(args, world, rank, pg):
