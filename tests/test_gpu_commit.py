@@ -268,6 +268,39 @@ def test_config5_batched_commits_sampled():
             _close(G.snapshot(w)[idx].cpu().numpy(), s[w], f"s_{w} (sampled)")
 
 
+def test_parameter_vector_beyond_two_to_the_31():
+    """P = 2^31 + 5 coordinates (about 34 GB of state and gradient): every index of theta,
+    m, s and the gradient needs 64 bits, and P mod 4 = 1 leaves a ragged tail.  Three
+    commits by one worker (its own moment and snapshot), checked on coordinates on both
+    sides of 2^31, the tail, and a random sample."""
+    seed, n = 5, 1
+    P = (1 << 31) + 5
+    order = [0, 0, 0]
+    rng = np.random.default_rng(31)
+    edge = np.concatenate([np.arange(8), (1 << 31) - 4 + np.arange(9), P - 1 - np.arange(8)])
+    cols = np.unique(np.concatenate([edge, rng.integers(0, P, 4096)])).astype(np.int64)
+    theta0 = synth.theta0_flat(seed, cols)
+    g_cpu = synth.grad_heavytail(seed, 0, cols)[None, :]
+    th, m, s = _fresh_cpu(theta0, n)
+    oracle.gem_run(th, m, s, g_cpu, np.asarray(order, np.int32), grad_index=np.zeros(3, np.int64),
+                   eta=ETA, mu=MU, eps=EPS)
+    stream = torch.cuda.Stream()
+    with torch.cuda.stream(stream), gem.Gem(P, n, ETA, MU, EPS, stream=stream) as G:
+        th0 = synth_gpu.theta0_flat(seed, torch.empty(P, device="cuda"), stream=stream)
+        G.set_theta(th0)
+        del th0
+        grad = torch.empty((1, P), device="cuda")
+        synth_gpu.grad_heavytail(seed, 0, grad, P, stream=stream)
+        G.commit(0, grad[0])                              # a single commit
+        G.commit_batch([0, 0], [grad[0], grad[0]])        # and a batch reusing it
+        G.sync()
+        idx = torch.from_numpy(cols).cuda()
+        _close(G.theta()[idx].cpu().numpy(), th, "theta beyond 2^31 (sampled)")
+        _close(G.moment(0)[idx].cpu().numpy(), m[0], "m beyond 2^31 (sampled)")
+        _close(G.snapshot(0)[idx].cpu().numpy(), s[0], "s beyond 2^31 (sampled)")
+        del grad
+
+
 def test_commits_read_gradients_written_by_the_kernel_just_before():
     """Every commit launch is a programmatic dependent of the previous kernel in its
     stream and waits for it at entry.  Here each gradient is written by a PyTorch kernel on
