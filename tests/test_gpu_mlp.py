@@ -74,12 +74,30 @@ def rel_l2(a, b):
     ([37, 19, 5, 3], 7, sim.GEM_MLP_TF32, 1e-4, 1e-2),
 ])
 def test_worker_gradients_match_oracle(dims, b, precision, tol, deep_tol):
+    _gradient_parity(dims, b, precision, tol, deep_tol, 3, [0, 2, 1, 2])
+
+
+@pytest.mark.parametrize("dims,b,precision,tol,deep_tol", [
+    ([64, 33, 16], 1024, sim.GEM_MLP_FP32, 1e-5, 1e-5),                  # the largest batch
+    ([64, 33, 16], 1024, sim.GEM_MLP_TF32, 1e-4, 1e-2),
+    ([40, 36, 32, 28, 24, 20, 16, 12, 10], 5, sim.GEM_MLP_FP32, 1e-5, 1e-5),   # eight layers
+    ([20, 9, 2], 1, sim.GEM_MLP_FP32, 1e-5, 1e-5),                       # one sample, two classes
+])
+def test_worker_gradients_at_the_engine_limits(dims, b, precision, tol, deep_tol):
+    _gradient_parity(dims, b, precision, tol, deep_tol, 3, [0, 2, 1, 2])
+
+
+def test_more_workers_in_one_call_than_group_slots():
+    """130 distinct workers in one gem_mlp_grad call: the engine works through them in
+    chunks of at most 128 groups."""
+    _gradient_parity([30, 12, 4], 8, sim.GEM_MLP_FP32, 1e-5, 1e-5, 130, list(range(129, -1, -1)))
+
+
+def _gradient_parity(dims, b, precision, tol, deep_tol, n, workers):
     seed = 21
     d0, C = dims[0], dims[-1]
     P = synth.mlp_param_count(dims)
-    n = 3
     theta0 = theta0_with_biases(seed, dims)
-    workers = [0, 2, 1, 2]
     batches = np.stack([synth.batch_indices(seed, w, k, b) for k, w in enumerate(workers)])
     X = torch.empty((ROWS, d0), device="cuda")
     y = torch.empty(ROWS, dtype=torch.int32, device="cuda")
