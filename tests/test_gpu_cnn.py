@@ -86,7 +86,9 @@ def _blocks(shape):
 @pytest.mark.parametrize("shape,b,G", [(cnn.CNN_MNIST, 64, 3), ((16, 3, 4, 5, 4, 3), 7, 2),
                                        ((20, 2, 3, 7, 6, 4), 5, 3),
                                        # pooled conv1 rows of 16: two row blocks, the second ragged
-                                       ((36, 2, 3, 6, 5, 3), 3, 2)])
+                                       ((36, 2, 3, 6, 5, 3), 3, 2),
+                                       (cnn.CNN_MNIST, 1, 2),                 # one sample
+                                       ((28, 16, 24, 32, 16, 2), 2, 2)])      # wider, two classes
 def test_gradients_match_the_oracle(shape, b, G):
     """G workers with different snapshots, in one batched call; every parameter tensor of
     every worker's gradient within 1e-5 relative L2 of the oracle's double gradient."""
@@ -192,6 +194,10 @@ def test_argument_checks():
     P = synth.cnn_param_count(shape)
     assert cnn.gem_cnn_param_count((17, 3, 4, 5, 4, 3)) == -1      # H - 4 odd
     assert cnn.gem_cnn_param_count((12, 3, 4, 5, 4, 3)) == -1      # conv2 output too small
+    wide = (28, 64, 64, 8, 8, 4)        # conv2's weights alone (400 KB) exceed a block's staging
+    with gem.Gem(synth.cnn_param_count(wide), 1, ETA, MU, EPS) as G:
+        with pytest.raises(GemError):
+            cnn.gem_cnn_create(G.h, wide, 4)
     with gem.Gem(P + 1, 2, ETA, MU, EPS) as G:
         with pytest.raises(GemError):
             cnn.gem_cnn_create(G.h, shape, 4)                       # P does not match
