@@ -301,6 +301,36 @@ def test_parameter_vector_beyond_two_to_the_31():
         del grad
 
 
+def test_worker_drop_out_on_the_device():
+    """Worker 2 of 4 stops committing after commit 40 of 300; batches before and after.
+    The device matches the oracle bit for bit, and the dropped worker's m_w and s_w on the
+    device do not change after its last commit."""
+    P, n, T, gone, after = 70_001, 4, 300, 2, 40
+    rng = np.random.default_rng(23)
+    theta0 = (0.05 * rng.standard_normal(P)).astype(np.float32)
+    grads = (0.1 * rng.standard_normal((T, P))).astype(np.float32)
+    base = rng.integers(0, n, 2 * T)
+    order = [int(w) for t, w in enumerate(base) if not (w == gone and t >= after)][:T]
+    last = max(t for t in range(T) if order[t] == gone)
+    th, m, s = _fresh_cpu(theta0, n)
+    oracle.gem_run(th, m, s, grads, np.asarray(order, np.int32), eta=ETA, mu=MU, eps=EPS)
+    g_dev = _padded(grads)
+    with gem.Gem(P, n, ETA, MU, EPS) as G:
+        G.set_theta(torch.from_numpy(theta0).cuda())
+        G.commit_batch(order[:last + 1], [g_dev[t, :P] for t in range(last + 1)])
+        G.sync()
+        m_gone, s_gone = G.moment(gone).clone(), G.snapshot(gone).clone()
+        for t0 in range(last + 1, T, 37):
+            t1 = min(T, t0 + 37)
+            G.commit_batch(order[t0:t1], [g_dev[t, :P] for t in range(t0, t1)])
+        G.sync()
+        assert torch.equal(G.moment(gone), m_gone) and torch.equal(G.snapshot(gone), s_gone)
+        _close(G.theta().cpu().numpy(), th, "theta")
+        for w in range(n):
+            _close(G.moment(w).cpu().numpy(), m[w], f"m_{w}")
+            _close(G.snapshot(w).cpu().numpy(), s[w], f"s_{w}")
+
+
 def test_commits_read_gradients_written_by_the_kernel_just_before():
     """Every commit launch is a programmatic dependent of the previous kernel in its
     stream and waits for it at entry.  Here each gradient is written by a PyTorch kernel on

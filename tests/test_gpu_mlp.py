@@ -288,6 +288,28 @@ def test_config1_free_running_trajectory():
     assert np.array_equal(final, recs[-1])
 
 
+def _drop_out_schedule(seed, n, T, gone=1, after=15):
+    """Uniform ticks with worker `gone` leaving after tick `after`."""
+    base = sim.gem_schedule_uniform(seed, n, 3 * T)[0]
+    order = np.array([w for t, w in enumerate(base) if not (w == gone and t >= after)][:T], np.int32)
+    return order, None
+
+
+def test_mlp_run_with_a_worker_dropping_out():
+    """The 784-64-10 network, n = 4, worker 1 leaving after tick 15: the segment planner
+    and the batched gradients follow any order; the device run stays within 1e-4 of the
+    oracle over 80 commits."""
+    dims, n, b, T, seed = [784, 64, 10], 4, 32, 80, 1
+    rec_at = [9, 39, 79]
+    recs, losses, final, inputs = _e2e(dims, n, b, T, seed, _drop_out_schedule,
+                                       sim.GEM_MLP_FP32, rec_at)
+    assert 1 not in set(inputs[0][20:].tolist())
+    ref, ref_losses = _oracle_e2e(dims, n, seed, inputs, T, rec_at, False)
+    for r, t in enumerate(rec_at):
+        assert rel_l2(recs[r], ref[r]) < 1e-4, (t, rel_l2(recs[r], ref[r]))
+    np.testing.assert_allclose(losses, ref_losses, rtol=1e-4)
+
+
 @pytest.mark.slow
 def test_config3_windows_and_prefix():
     """MLP 784-1000-1000-10, n = 30, b = 128, exponential-queue schedule (seed 3): windows

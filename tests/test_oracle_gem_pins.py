@@ -197,6 +197,33 @@ def test_round_robin_drift_is_the_other_workers_updates():
                                    rtol=1e-12, atol=1e-13)
 
 
+def test_worker_drop_out_freezes_its_state():
+    """A worker that stops committing (it dropped out, or stalled for good) keeps m_w and
+    s_w exactly as its last commit left them, and from then on the run is that of the
+    remaining workers alone, started from the same theta and the same per-worker state: a
+    commit reads and writes only theta and its own worker's row."""
+    rng = np.random.default_rng(17)
+    n, P, T, gone, after = 3, 64, 60, 2, 12
+    theta0 = rng.standard_normal(P).astype(np.float32)
+    g = (0.3 * rng.standard_normal((T, P))).astype(np.float32)
+    base = rng.integers(0, n, 4 * T)
+    order = np.array([w for t, w in enumerate(base) if not (w == gone and t >= after)][:T], np.int32)
+    last = max(t for t in range(T) if order[t] == gone)
+    theta, m, s = _fresh(theta0, n, np.float32)
+    oracle.gem_run(theta, m, s, g[:last + 1], order[:last + 1], eta=0.05, mu=0.9, eps=1e-8)
+    m_gone, s_gone = m[gone].copy(), s[gone].copy()
+    keep = [w for w in range(n) if w != gone]
+    th_b, m_b, s_b = theta.copy(), m[keep].copy(), s[keep].copy()
+    oracle.gem_run(theta, m, s, g[last + 1:], order[last + 1:], eta=0.05, mu=0.9, eps=1e-8)
+    assert np.array_equal(m[gone], m_gone) and np.array_equal(s[gone], s_gone)
+    remap = {w: i for i, w in enumerate(keep)}
+    oracle.gem_run(th_b, m_b, s_b, g[last + 1:], np.array([remap[w] for w in order[last + 1:]], np.int32),
+                   eta=0.05, mu=0.9, eps=1e-8)
+    assert np.array_equal(theta, th_b)
+    assert np.array_equal(m[keep], m_b) and np.array_equal(s[keep], s_b)
+    assert not np.array_equal(theta, s_gone)              # the others did move theta
+
+
 def test_literal_precommit_snapshot_reading_differs():
     # Contrast: taking s as the value pulled before the own commit breaks the reduction
     # of a single worker to SGD (its drift is then its own previous update).
