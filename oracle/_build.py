@@ -21,15 +21,22 @@ def _stale() -> bool:
     return any(p.stat().st_mtime > t for p in SOURCES + [Path(__file__)])
 
 
+def compile_library(sources, out: Path) -> Path:
+    """Compile the given oracle sources into the shared library `out` (same flags as the
+    oracle itself; the planted-mistake tests build altered copies with it)."""
+    out = Path(out)
+    tmp = out.with_suffix(f".so.tmp{os.getpid()}")
+    cmd = ["g++", "-std=c++17", "-O2", "-ffp-contract=off", "-fno-fast-math", "-fopenmp",
+           "-fPIC", "-shared", *map(str, sources), "-o", str(tmp)]
+    subprocess.run(cmd, check=True)
+    os.replace(tmp, out)
+    return out
+
+
 def build_oracle(force: bool = False) -> Path:
     if not force and not _stale():
         return LIB
-    tmp = LIB.with_suffix(f".so.tmp{os.getpid()}")
-    cmd = ["g++", "-std=c++17", "-O2", "-ffp-contract=off", "-fno-fast-math", "-fopenmp",
-           "-fPIC", "-shared", *map(str, SOURCES), "-o", str(tmp)]
-    subprocess.run(cmd, check=True)
-    os.replace(tmp, LIB)
-    return LIB
+    return compile_library(SOURCES, LIB)
 
 
 if __name__ == "__main__":

@@ -2,6 +2,7 @@
 from __future__ import annotations
 
 import ctypes as C
+import os
 
 import numpy as np
 
@@ -20,7 +21,9 @@ _lib = None
 def lib():
     global _lib
     if _lib is None:
-        _lib = C.CDLL(str(build_oracle()))
+        # ORACLE_LIBRARY: a library built from altered oracle sources, for the tests that
+        # check that a planted mistake makes the oracle's pins fail
+        _lib = C.CDLL(os.environ.get("ORACLE_LIBRARY") or str(build_oracle()))
         p = C.c_void_p
         i64, i32, f64 = C.c_int64, C.c_int, C.c_double
         run_args = [i64, i32, i32, p, p, p, i64, p, p, p, p, i64, f64, f64, f64, i32, f64,
