@@ -86,6 +86,33 @@ __device__ __forceinline__ float to_tf32(float x) {
   return __uint_as_float(u);
 }
 
+// Four consecutive elements (outer, inner .. inner + 3) of a row-major view with leading
+// dimension ld: one 16-byte load when the rows are 16-byte aligned (vec) and the quad lies
+// inside the operand, else element by element; zeros outside.  TF32: each value rounded.
+template <bool TF32>
+__device__ __forceinline__ float4 stage_quad(const float* base, long long ld, bool vec, int outer,
+                                             int inner, int outer_end, int inner_end) {
+  float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+  if (outer < outer_end) {
+    const float* q = base + (long long)outer * ld + inner;
+    if (vec && inner + 3 < inner_end) {
+      v = *reinterpret_cast<const float4*>(q);
+    } else {
+      if (inner < inner_end) v.x = q[0];
+      if (inner + 1 < inner_end) v.y = q[1];
+      if (inner + 2 < inner_end) v.z = q[2];
+      if (inner + 3 < inner_end) v.w = q[3];
+    }
+  }
+  if (TF32) {
+    v.x = to_tf32(v.x);
+    v.y = to_tf32(v.y);
+    v.z = to_tf32(v.z);
+    v.w = to_tf32(v.w);
+  }
+  return v;
+}
+
 // C[g] (M x N) = epilogue( op(A[g]) op(B[g]) ).  A_KMAJOR: A(m, k) at A[m*lda + k], else at
 // A[k*lda + m].  B_KMAJOR: B(k, n) at B[n*ldb + k], else at B[k*ldb + n].
 //
@@ -100,7 +127,6 @@ gemm_grouped_kernel(const __grid_constant__ GemmArgs p) {
   gem::pdl_entry();
   constexpr int T = 2 * TBM;                 // threads: 16 columns x TBM / 8 rows of them
   constexpr int kPadA = TBM + 4, kPadB = BN + 4;  // row pitches (floats), 16-byte aligned
-  constexpr int kBPer = BN * BK / T;         // B elements staged per thread (A: always 8)
   __shared__ __align__(16) float As[2][BK][kPadA];
   __shared__ __align__(16) float Bs[2][BK][kPadB];
   const int split = p.ksplit > 1 ? p.ksplit : 1;
@@ -114,40 +140,54 @@ gemm_grouped_kernel(const __grid_constant__ GemmArgs p) {
   const long long lda = p.A.ld, ldb = p.B.ld;
   const int M = p.M, N = p.N;
 
-  // staging: 8 A elements and 4 B elements per thread per k-tile
-  float ra[8], rb[kBPer];
+  // staging: the k-tile's A (TBM x 16) and B (64 x 16) elements as quads along each
+  // operand's contiguous index (k for a K-major operand, m or n otherwise), two quads of A
+  // and one or two of B per thread; quads are read with 16-byte loads where the operand's
+  // rows are 16-byte aligned (k0 and the tile origins are multiples of 4).
+  constexpr int kAQ = TBM * BK / 4 / T, kBQ = BN * BK / 4 / T;
+  const bool a_vec = (reinterpret_cast<uintptr_t>(A) & 15u) == 0 && (lda & 3) == 0;
+  const bool b_vec = (reinterpret_cast<uintptr_t>(B) & 15u) == 0 && (ldb & 3) == 0;
+  float4 ra[kAQ], rb[kBQ];
   auto load = [&](int k0) {
 #pragma unroll
-    for (int it = 0; it < 8; ++it) {
-      int m, k;
-      if (A_KMAJOR) { m = (tid >> 4) + (T / 16) * it; k = tid & 15; }
-      else          { m = tid % TBM;                  k = tid / TBM + 2 * it; }
-      const int gm = m0 + m, gk = k0 + k;
-      float v = 0.f;
-      if (gm < M && gk < kend) v = A_KMAJOR ? A[gm * lda + gk] : A[gk * lda + gm];
-      ra[it] = TF32 ? to_tf32(v) : v;
+    for (int it = 0; it < kAQ; ++it) {
+      const int q = tid + T * it;
+      if (A_KMAJOR) ra[it] = stage_quad<TF32>(A, lda, a_vec, m0 + (q >> 2), k0 + 4 * (q & 3), M, kend);
+      else ra[it] = stage_quad<TF32>(A, lda, a_vec, k0 + q / (TBM / 4), m0 + 4 * (q % (TBM / 4)), kend, M);
     }
 #pragma unroll
-    for (int it = 0; it < kBPer; ++it) {
-      int n, k;
-      if (B_KMAJOR) { n = (tid >> 4) + (T / 16) * it; k = tid & 15; }
-      else          { n = tid & 63;                   k = (tid >> 6) + (T / 64) * it; }
-      const int gn = n0 + n, gk = k0 + k;
-      float v = 0.f;
-      if (gn < N && gk < kend) v = B_KMAJOR ? B[gn * ldb + gk] : B[gk * ldb + gn];
-      rb[it] = TF32 ? to_tf32(v) : v;
+    for (int it = 0; it < kBQ; ++it) {
+      const int q = tid + T * it;
+      if (B_KMAJOR) rb[it] = stage_quad<TF32>(B, ldb, b_vec, n0 + (q >> 2), k0 + 4 * (q & 3), N, kend);
+      else rb[it] = stage_quad<TF32>(B, ldb, b_vec, k0 + q / (BN / 4), n0 + 4 * (q % (BN / 4)), kend, N);
     }
   };
   auto store = [&](int buf) {
 #pragma unroll
-    for (int it = 0; it < 8; ++it) {
-      if (A_KMAJOR) As[buf][tid & 15][(tid >> 4) + (T / 16) * it] = ra[it];
-      else          As[buf][tid / TBM + 2 * it][tid % TBM] = ra[it];
+    for (int it = 0; it < kAQ; ++it) {
+      const int q = tid + T * it;
+      if (A_KMAJOR) {
+        const int m = q >> 2, k = 4 * (q & 3);
+        As[buf][k][m] = ra[it].x;
+        As[buf][k + 1][m] = ra[it].y;
+        As[buf][k + 2][m] = ra[it].z;
+        As[buf][k + 3][m] = ra[it].w;
+      } else {
+        *reinterpret_cast<float4*>(&As[buf][q / (TBM / 4)][4 * (q % (TBM / 4))]) = ra[it];
+      }
     }
 #pragma unroll
-    for (int it = 0; it < kBPer; ++it) {
-      if (B_KMAJOR) Bs[buf][tid & 15][(tid >> 4) + (T / 16) * it] = rb[it];
-      else          Bs[buf][(tid >> 6) + (T / 64) * it][tid & 63] = rb[it];
+    for (int it = 0; it < kBQ; ++it) {
+      const int q = tid + T * it;
+      if (B_KMAJOR) {
+        const int n = q >> 2, k = 4 * (q & 3);
+        Bs[buf][k][n] = rb[it].x;
+        Bs[buf][k + 1][n] = rb[it].y;
+        Bs[buf][k + 2][n] = rb[it].z;
+        Bs[buf][k + 3][n] = rb[it].w;
+      } else {
+        *reinterpret_cast<float4*>(&Bs[buf][q / (BN / 4)][4 * (q % (BN / 4))]) = rb[it];
+      }
     }
   };
 
