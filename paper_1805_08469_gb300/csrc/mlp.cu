@@ -700,9 +700,23 @@ __global__ void __launch_bounds__(256) splitk_reduce_kernel(const __grid_constan
 // takes whole rows m: lane l accumulates k = l, l + 32, ... (coalesced A reads, conflict-free
 // shared reads), a fixed butterfly adds the 32 lane sums, and lane 0 writes the N outputs
 // of the row.  Deterministic.  rows_per_block rows per block.
-template <bool TF32>
+// The last layer's softmax cross-entropy, fused into the logits kernel (XENT): the lane
+// that finishes a row's logits z goes on, with the operations and order of
+// softmax_xent_kernel, to the row's loss gradient (softmax(z) - onehot(y)) / b and its
+// loss; the row losses are summed in row order by bias_grad_kernel.
+struct XentArgs {
+  const int32_t* labels;        // [rows of the data set]
+  const int32_t* batch_rows;    // [groups][b]
+  float* delta;                 // D_L [b][C] of group g at delta + g * group_stride
+  float* row_loss;              // [b] of group g at row_loss + g * group_stride
+  long long group_stride;
+  int b;
+};
+
+template <bool TF32, bool XENT>
 __global__ void __launch_bounds__(256)
-gemm_small_n_kernel(const __grid_constant__ GemmArgs p, int rows_per_block) {
+gemm_small_n_kernel(const __grid_constant__ GemmArgs p, int rows_per_block,
+                    const __grid_constant__ XentArgs x) {
   gem::pdl_entry();
   extern __shared__ __align__(16) float Bsm[];
   const int g = blockIdx.y;
@@ -763,14 +777,47 @@ gemm_small_n_kernel(const __grid_constant__ GemmArgs p, int rows_per_block) {
       float* c = p.C + (long long)g * p.c_group_stride + (long long)m * p.ldc;
 #pragma unroll
       for (int n = 0; n < kMaxClasses; ++n)
-        if (n < N) c[n] = acc[n] + bias[n];
+        if (n < N) {
+          acc[n] = acc[n] + bias[n];   // the logit z_n
+          c[n] = acc[n];
+        }
+      if (XENT) {
+        int y = x.labels[x.batch_rows[(long long)g * x.b + m]];
+        const bool bad_label = y < 0 || y >= N;   // reported as a NaN loss and gradient
+        if (bad_label) y = 0;
+        float zmax = acc[0];
+#pragma unroll
+        for (int n = 1; n < kMaxClasses; ++n)
+          if (n < N) zmax = fmaxf(zmax, acc[n]);
+        float e[kMaxClasses];
+        float sum = 0.f;
+#pragma unroll
+        for (int n = 0; n < kMaxClasses; ++n)
+          if (n < N) {
+            e[n] = expf(acc[n] - zmax);
+            sum += e[n];
+          }
+        const float inv_b = 1.0f / float(x.b);
+        const float poison = bad_label ? __int_as_float(0x7fc00000) : 0.f;
+        float* d = x.delta + (long long)g * x.group_stride + (long long)m * N;
+        float zy = acc[0];
+#pragma unroll
+        for (int n = 0; n < kMaxClasses; ++n)
+          if (n < N) {
+            d[n] = (e[n] / sum - (n == y ? 1.f : 0.f)) * inv_b + poison;
+            if (n == y) zy = acc[n];
+          }
+        x.row_loss[(long long)g * x.group_stride + m] = (logf(sum) + zmax) - zy + poison;
+      }
     }
   }
 }
 
 // Launch the logits product when B fits in shared memory; false otherwise.
+// xent: the fused loss (null for plain logits).
 template <bool TF32>
-bool launch_small_n(const GemmArgs& a, int groups, cudaStream_t st, cudaError_t* err) {
+bool launch_small_n(const GemmArgs& a, int groups, cudaStream_t st, cudaError_t* err,
+                    const XentArgs* xent) {
   const size_t bytes = sizeof(float) * size_t(a.N) * size_t(a.K);
   constexpr size_t kMaxBytes = 200 * 1024;
   if (bytes > kMaxBytes) return false;
@@ -778,8 +825,11 @@ bool launch_small_n(const GemmArgs& a, int groups, cudaStream_t st, cudaError_t*
   int dev = 0;
   cudaGetDevice(&dev);
   if (bytes > 48 * 1024 && (dev < 0 || dev >= 64 || !configured[dev])) {
-    *err = cudaFuncSetAttribute(gemm_small_n_kernel<TF32>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                int(kMaxBytes));
+    *err = cudaFuncSetAttribute(gemm_small_n_kernel<TF32, false>,
+                                cudaFuncAttributeMaxDynamicSharedMemorySize, int(kMaxBytes));
+    if (*err == cudaSuccess)
+      *err = cudaFuncSetAttribute(gemm_small_n_kernel<TF32, true>,
+                                  cudaFuncAttributeMaxDynamicSharedMemorySize, int(kMaxBytes));
     if (*err != cudaSuccess) return true;
     if (dev >= 0 && dev < 64) configured[dev] = true;
   }
@@ -788,7 +838,10 @@ bool launch_small_n(const GemmArgs& a, int groups, cudaStream_t st, cudaError_t*
   rows_per_block = rows_per_block < 8 ? 8 : (rows_per_block + 7) / 8 * 8;
   const int rpb = int(rows_per_block);
   dim3 grid(unsigned((a.M + rpb - 1) / rpb), unsigned(groups));
-  gem::launch_pdl(gemm_small_n_kernel<TF32>, grid, 256, bytes, st, a, rpb);
+  if (xent)
+    gem::launch_pdl(gemm_small_n_kernel<TF32, true>, grid, 256, bytes, st, a, rpb, *xent);
+  else
+    gem::launch_pdl(gemm_small_n_kernel<TF32, false>, grid, 256, bytes, st, a, rpb, XentArgs{});
   *err = cudaGetLastError();
   return true;
 }
@@ -843,6 +896,8 @@ __global__ void softmax_xent_kernel(const float* logits, float* delta, long long
 
 struct BiasGradArgs {
   int n_layers, b;
+  long long row_loss_off;           // with losses: the row losses of the fused loss kernel
+  float* losses;                    // [groups] minibatch losses, or null
   long long grad_off[kMaxLayers];   // offset of db_l in the flat gradient
   long long delta_off[kMaxLayers];  // offset of D_{l+1} in the slot scratch
   int width[kMaxLayers];            // d_{l+1}
@@ -851,7 +906,9 @@ struct BiasGradArgs {
 
 // db_l[o] = sum over the batch of D_{l+1}[r][o], every layer in one launch.
 // Block of 32 x 8 threads: lane x owns output q = 32 blockIdx.x + x; warp y sums rows
-// r = y, y + 8, ... in order, and lane x of warp 0 adds the 8 warp sums in order.
+// r = y, y + 8, ... in order, and lane x of warp 0 adds the 8 warp sums in order.  When
+// the logits kernel computed the loss (losses set), thread 0 of block (0, g) also adds
+// group g's row losses in row order and divides by b.
 __global__ void __launch_bounds__(256)
 bias_grad_kernel(const __grid_constant__ BiasGradArgs a, const float* delta,
                  long long slot_stride, float* grad, long long grad_stride) {
@@ -875,6 +932,12 @@ bias_grad_kernel(const __grid_constant__ BiasGradArgs a, const float* delta,
 #pragma unroll
     for (int w = 0; w < 8; ++w) t += part[w][x];
     grad[g * grad_stride + a.grad_off[l] + o] = t;
+  }
+  if (a.losses && blockIdx.x == 0 && threadIdx.x == 0) {   // the minibatch loss, rows in order
+    const float* rl = delta + g * slot_stride + a.row_loss_off;
+    float t = 0.f;
+    for (int r = 0; r < a.b; ++r) t += rl[r];
+    a.losses[g] = t / float(a.b);
   }
 }
 
@@ -1014,6 +1077,7 @@ int mlp_chunk(gem_mlp* M, const int32_t* workers, int G, const int32_t* batch_ro
   const long long wstride = (long long)h->stride;
 
   // forward
+  bool fused_loss = false;   // the logits kernel also produced the loss gradient
   for (int l = 0; l < L; ++l) {
     const int din = M->dims[l], dout = M->dims[l + 1];
     a.M = b; a.N = dout; a.K = din;
@@ -1026,9 +1090,18 @@ int mlp_chunk(gem_mlp* M, const int32_t* workers, int G, const int32_t* batch_ro
     a.c_group_stride = S;
     a.ldc = dout;
     cudaError_t e;
+    XentArgs xa;
+    xa.labels = M->labels;
+    xa.batch_rows = batch_rows;
+    xa.delta = scr + M->off_delta[L];
+    xa.row_loss = scr + M->off_row_loss;
+    xa.group_stride = S;
+    xa.b = b;
     if (last && dout <= kMaxClasses &&
-        (tf32 ? launch_small_n<true>(a, G, st, &e) : launch_small_n<false>(a, G, st, &e))) {
-      // the logits: few outputs per row, the worker's weights held in shared memory
+        (tf32 ? launch_small_n<true>(a, G, st, &e, &xa) : launch_small_n<false>(a, G, st, &e, &xa))) {
+      // the logits: few outputs per row, the worker's weights held in shared memory, and
+      // the loss with its gradient in the same kernel
+      fused_loss = true;
     } else {
       e = last ? launch_gemm<true, true, kBias>(a, G, tf32, st)
                : launch_gemm<true, true, kBiasRelu>(a, G, tf32, st);
@@ -1036,10 +1109,12 @@ int mlp_chunk(gem_mlp* M, const int32_t* workers, int G, const int32_t* batch_ro
     if ((rc = cuda_rc(e))) return rc;
     M->launches++;
   }
-  gem::launch_pdl(softmax_xent_kernel, G, 128, 0, st, scr + M->off_logits, scr + M->off_delta[L], S, b,
-                                         M->dims[L], M->labels, batch_rows, losses);
-  if ((rc = cuda_rc(cudaGetLastError()))) return rc;
-  M->launches++;
+  if (!fused_loss) {
+    gem::launch_pdl(softmax_xent_kernel, G, 128, 0, st, scr + M->off_logits, scr + M->off_delta[L], S,
+                    b, M->dims[L], M->labels, batch_rows, losses);
+    if ((rc = cuda_rc(cudaGetLastError()))) return rc;
+    M->launches++;
+  }
 
   // backward.  The weight-gradient products go to the side stream when there is one: each
   // waits for its delta D_{l+1} (event recorded on the main stream) and runs next to the
@@ -1093,6 +1168,8 @@ int mlp_chunk(gem_mlp* M, const int32_t* workers, int G, const int32_t* batch_ro
   std::memset(&ba, 0, sizeof(ba));
   ba.n_layers = L;
   ba.b = b;
+  ba.row_loss_off = M->off_row_loss;
+  ba.losses = fused_loss ? losses : nullptr;
   ba.first[0] = 0;
   for (int l = 0; l < L; ++l) {
     ba.grad_off[l] = M->b_off[l];
@@ -1144,6 +1221,8 @@ int mlp_build(gem_t* g, int n_layers, const int32_t* dims, int batch, int precis
     M->off_delta[l] = off;
     off += round32((long long)batch * dims[l]);
   }
+  M->off_row_loss = off;
+  off += round32(batch);
   M->slot_stride = off;
   M->slots = g->n < kMaxGroups ? g->n : kMaxGroups;
   int dev_prev = 0;
@@ -1452,6 +1531,8 @@ extern "C" int gem_mlp_grad_static(int n_layers, const int32_t* dims, int batch,
     M.off_delta[l] = off;
     off += round32((long long)batch * dims[l]);
   }
+  M.off_row_loss = off;
+  off += round32(batch);
   M.slot_stride = off;
   M.slots = 1;
   const long long rows_floats = round32(batch);  // minibatch rows stored after the slot

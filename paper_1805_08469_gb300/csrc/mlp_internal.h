@@ -39,6 +39,7 @@ struct gem_mlp {
   // per-slot scratch: X_s [b x d0], A_l [b x d_l] (l = 1..L-1), logits [b x C],
   // D_l [b x d_l] (l = 1..L, and l = 0 with input_grad)
   long long off_x = 0, off_act[gem::mlp::kMaxLayers + 1] = {}, off_logits = 0, off_delta[gem::mlp::kMaxLayers + 1] = {};
+  long long off_row_loss = 0;   // per-row losses of the minibatch [b] (fused loss)
   long long slot_stride = 0;
   int slots = 0;
   float* scratch = nullptr;
