@@ -47,6 +47,12 @@ constexpr long long kSmCountHint = 152;  // GB300
 #ifndef GEM_TF32_BIG_TILE_BLOCKS   // large tensor-core tiles once a launch has this many per SM
 #define GEM_TF32_BIG_TILE_BLOCKS 1
 #endif
+#ifndef GEM_SIMT_BIG_TILE_BLOCKS   // the same for the CUDA-core tiles
+#define GEM_SIMT_BIG_TILE_BLOCKS 2
+#endif
+#ifndef GEM_SIMT_MIN_CHUNK         // shortest split of K on the CUDA cores
+#define GEM_SIMT_MIN_CHUNK 64
+#endif
 constexpr int kMaxSplit = GEM_MAX_SPLIT;   // split-K factor at most
 
 enum Epilogue : int { kStore = 0, kBias = 1, kBiasRelu = 2, kMask = 3 };
@@ -991,7 +997,7 @@ cudaError_t launch_gemm(const GemmArgs& a_in, int groups, bool tf32, cudaStream_
   const bool tc = tf32 && a.M >= 32 && a.K >= 32;
   const long long mt = (a.M + 127) / 128, nt64 = (a.N + 63) / 64, nt128 = (a.N + 127) / 128;
   const long long big = (tc ? nt128 : nt64) * mt * groups;
-  if (big >= (tc ? GEM_TF32_BIG_TILE_BLOCKS : 2) * kSmCountHint) {
+  if (big >= (tc ? GEM_TF32_BIG_TILE_BLOCKS : GEM_SIMT_BIG_TILE_BLOCKS) * kSmCountHint) {
     if (tc)
       launch_mma<128, AK, BK_, EPI>(a, groups, st);
     else
@@ -1001,7 +1007,7 @@ cudaError_t launch_gemm(const GemmArgs& a_in, int groups, bool tf32, cudaStream_
   const long long small = tc ? nt64 * mt * groups : nt64 * ((a.M + 63) / 64) * groups;
   int split = 1;
   const long long mn = (long long)a.M * a.N * groups;
-  const int min_chunk = tc ? GEM_TF32_MIN_CHUNK : 128;   // the tensor cores get through K faster
+  const int min_chunk = tc ? GEM_TF32_MIN_CHUNK : GEM_SIMT_MIN_CHUNK;   // the tensor cores get through K faster
   if (a.ws && a.M <= 128)
     while (split < kMaxSplit && small * split < 4 * kSmCountHint && a.K / (2 * split) >= min_chunk &&
            mn * 2 * split <= a.ws_floats)
