@@ -2,8 +2,10 @@
 //
 // A segment of G distinct workers is processed together, each worker's layers reading
 // its snapshot s_w:
-//   conv1_pool_kernel      conv1 + bias, 2 x 2 max-pool, ReLU    (conv1 outputs kept)
+//   conv1_pool_kernel      conv1 + bias, 2 x 2 max-pool, ReLU
 //   conv2_pool_kernel      conv2 + bias, dropout scale, max-pool, ReLU -> the head's input
+//                          (both keep, per pooled output, the position of the window's
+//                          first maximum as one byte, for the backward routing)
 //   dense head             fc1 -> fc2 -> fc3, softmax cross-entropy and the backward pass
 //                          of the MLP engine, which also returns the gradient with respect
 //                          to the features
@@ -85,7 +87,7 @@ struct ConvArgs {
   const float* drop;           // [G][b][c2] dropout scales
   float* scr;                  // conv scratch, slot g at scr + g * S
   long long S;
-  long long o_z1, o_a1, o_z2, o_dz2, o_dz1, o_p1, o_p2;
+  long long o_k1, o_a1, o_k2, o_dz2, o_dz1, o_p1, o_p2;   // o_k*: byte codes (offsets in floats)
   float* head;                 // dense head scratch, slot g at head + g * head_S
   long long head_S, head_x, head_dx;   // offsets of its input rows and input gradient
   float* grads;                // gradient of group g at grads + g * grad_stride
@@ -158,7 +160,7 @@ __global__ void __launch_bounds__(kThreads) conv1_pool_kernel(const __grid_const
   stage(ws, th + a.w1, a.c1 * kK * kK);
   stage(bs, th + a.b1, a.c1);
   stage_wait();
-  float* z1s = a.scr + g * a.S + a.o_z1 + (long long)i * a.c1 * H1 * H1;
+  uint8_t* k1s = reinterpret_cast<uint8_t*>(a.scr + g * a.S + a.o_k1) + (long long)i * a.c1 * P1 * P1;
   float* a1s = a.scr + g * a.S + a.o_a1 + (long long)i * a.c1 * P1 * P1;
   for (int q = threadIdx.x; q < a.c1 * P1 * P1; q += blockDim.x) {
     const int px = q % P1, py = q / P1 % P1, co = q / (P1 * P1);
@@ -178,10 +180,9 @@ __global__ void __launch_bounds__(kThreads) conv1_pool_kernel(const __grid_const
 #pragma unroll
         for (int kx = 0; kx < kK; ++kx) acc = fmaf(w[ky * kK + kx], x[(d >> 1) + ky][(d & 1) + kx], acc);
       v[d] = acc;
-      z1s[(co * H1 + 2 * py + (d >> 1)) * H1 + 2 * px + (d & 1)] = acc;
     }
     float m;
-    first_max4(v, &m);
+    k1s[q] = uint8_t(first_max4(v, &m));
     a1s[q] = m > 0.f ? m : 0.f;
   }
 }
@@ -230,14 +231,11 @@ __global__ void __launch_bounds__(kPool2Threads) conv2_pool_kernel(const __grid_
 #pragma unroll
           for (int d = 0; d < 4; ++d) v[d] = fmaf(w[ky * kK + kx], x[(d >> 1) + ky][(d & 1) + kx], v[d]);
     }
-    float* z2 = a.scr + g * a.S + a.o_z2 + ((long long)i * a.c2 + co) * H2 * H2;
 #pragma unroll
-    for (int d = 0; d < 4; ++d) {
-      v[d] = v[d] * s;   // dropout: the channel's scale
-      z2[(2 * py + (d >> 1)) * H2 + 2 * px + (d & 1)] = v[d];
-    }
+    for (int d = 0; d < 4; ++d) v[d] = v[d] * s;   // dropout: the channel's scale
     float m;
-    first_max4(v, &m);
+    reinterpret_cast<uint8_t*>(a.scr + g * a.S + a.o_k2)[(long long)i * a.c2 * P2 * P2 + q] =
+        uint8_t(first_max4(v, &m));
     a.head[g * a.head_S + a.head_x + (long long)i * a.F + q] = m > 0.f ? m : 0.f;
   }
 }
@@ -258,13 +256,9 @@ __global__ void __launch_bounds__(kThreads) pool2_back_kernel(const __grid_const
   const float dfeat = a.head[g * a.head_S + a.head_dx + f];
   const float s = a.drop[gi * a.c2 + co];
   const long long base = g * a.S + ((long long)i * a.c2 + co) * a.H2 * a.H2;
-  const float* z2 = a.scr + a.o_z2 + base;
   float* dz2 = a.scr + a.o_dz2 + base;
-  float v[4];
-#pragma unroll
-  for (int d = 0; d < 4; ++d) v[d] = z2[(2 * py + (d >> 1)) * a.H2 + 2 * px + (d & 1)];
-  float vmax;
-  const int am = first_max4(v, &vmax);
+  const int am = reinterpret_cast<const uint8_t*>(a.scr + g * a.S + a.o_k2)
+      [((long long)i * a.c2 + co) * a.P2 * a.P2 + py * a.P2 + px];
   const float gval = feat > 0.f ? dfeat * s : 0.f;
 #pragma unroll
   for (int d = 0; d < 4; ++d) dz2[(2 * py + (d >> 1)) * a.H2 + 2 * px + (d & 1)] = d == am ? gval : 0.f;
@@ -301,7 +295,7 @@ __global__ void __launch_bounds__(kBackThreads) conv2_back_kernel(const __grid_c
   stage(a1s, a.scr + g * a.S + a.o_a1 + (long long)i * n_a1, n_a1);
   stage_wait();
   const int H1 = 2 * P1;
-  const float* z1s = a.scr + g * a.S + a.o_z1 + (long long)i * a.c1 * H1 * H1;
+  const uint8_t* k1s = reinterpret_cast<const uint8_t*>(a.scr + g * a.S + a.o_k1) + (long long)i * a.c1 * P1 * P1;
   float* dz1s = a.scr + g * a.S + a.o_dz1 + (long long)i * a.c1 * H1 * H1;
   const int nxb = (P1 + kBackRow - 1) / kBackRow;
   for (int q = threadIdx.x; q < a.c1 * P1 * nxb; q += blockDim.x) {
@@ -336,18 +330,13 @@ __global__ void __launch_bounds__(kBackThreads) conv2_back_kernel(const __grid_c
             if (col_ok[j - kx + kK - 1]) acc[j] = fmaf(d[j - kx + kK - 1], w[kx], acc[j]);
       }
     }
-    const float* z1 = z1s + ci * H1 * H1;
     float* dz1 = dz1s + ci * H1 * H1;
 #pragma unroll
     for (int j = 0; j < kBackRow; ++j) {
       const int px = px0 + j;
       if (px >= P1) break;
       const float dv = a1s[(ci * P1 + py) * P1 + px] > 0.f ? acc[j] : 0.f;
-      float v[4];
-#pragma unroll
-      for (int d = 0; d < 4; ++d) v[d] = z1[(2 * py + (d >> 1)) * H1 + 2 * px + (d & 1)];
-      float vmax;
-      const int am = first_max4(v, &vmax);
+      const int am = k1s[(ci * P1 + py) * P1 + px];
 #pragma unroll
       for (int d = 0; d < 4; ++d) dz1[(2 * py + (d >> 1)) * H1 + 2 * px + (d & 1)] = d == am ? dv : 0.f;
     }
@@ -505,7 +494,7 @@ struct gem_cnn {
   const float* X = nullptr;
   const int32_t* labels = nullptr;
   int64_t rows = 0;
-  long long o_z1 = 0, o_a1 = 0, o_z2 = 0, o_dz2 = 0, o_dz1 = 0, o_p1 = 0, o_p2 = 0;
+  long long o_k1 = 0, o_a1 = 0, o_k2 = 0, o_dz2 = 0, o_dz1 = 0, o_p1 = 0, o_p2 = 0;
   long long slot_stride = 0;
   int slots = 0;
   float* scratch = nullptr;
@@ -538,7 +527,7 @@ int cnn_chunk(gem_cnn* N, const int32_t* workers, int G, const int32_t* rows_dev
   a.drop = drop;
   a.scr = N->scratch;
   a.S = N->slot_stride;
-  a.o_z1 = N->o_z1; a.o_a1 = N->o_a1; a.o_z2 = N->o_z2; a.o_dz2 = N->o_dz2; a.o_dz1 = N->o_dz1;
+  a.o_k1 = N->o_k1; a.o_a1 = N->o_a1; a.o_k2 = N->o_k2; a.o_dz2 = N->o_dz2; a.o_dz1 = N->o_dz1;
   a.o_p1 = N->o_p1; a.o_p2 = N->o_p2;
   a.head = N->head->scratch;
   a.head_S = N->head->slot_stride;
@@ -631,9 +620,9 @@ int gem_cnn_create(gem_t* g, const int32_t* shape, int batch, gem_cnn_t** out) {
     off += round32(n);
     return o;
   };
-  N->o_z1 = take(b * s.c1 * s.H1 * s.H1);
+  N->o_k1 = take((b * s.c1 * s.P1 * s.P1 + 3) / 4);   // one byte per pooled output
   N->o_a1 = take(b * s.c1 * s.P1 * s.P1);
-  N->o_z2 = take(b * s.c2 * s.H2 * s.H2);
+  N->o_k2 = take((b * s.c2 * s.P2 * s.P2 + 3) / 4);
   N->o_dz2 = take(b * s.c2 * s.H2 * s.H2);
   N->o_dz1 = take(b * s.c1 * s.H1 * s.H1);
   N->o_p1 = take(b * s.c1 * (kK * kK + 1));
