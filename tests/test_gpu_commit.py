@@ -123,6 +123,31 @@ def test_host_gradient_batch_equals_device_batch():
         assert torch.equal(out, B.theta().cpu())
 
 
+def test_host_gradient_batches_back_to_back():
+    """Five gem_commit_batch_host calls issued without waiting, pageable gradients (each
+    call stages its chunks through the same two halves of the staging buffer, so a call
+    must not overwrite a half the previous one is still reading); the same as the device
+    path, bit for bit."""
+    P, n, K, calls = 50_001, 5, 11, 5
+    rng = np.random.default_rng(9)
+    theta0 = (0.05 * rng.standard_normal(P)).astype(np.float32)
+    grads = (0.05 * rng.standard_normal((calls * K, P))).astype(np.float32)
+    order = rng.integers(0, n, calls * K).tolist()
+    g_dev = _padded(grads)
+    with gem.Gem(P, n, ETA, MU, EPS) as A, gem.Gem(P, n, ETA, MU, EPS) as B:
+        for H in (A, B):
+            H.set_theta(torch.from_numpy(theta0).cuda())
+        for c in range(calls):
+            ks = range(c * K, (c + 1) * K)
+            A.commit_batch([order[k] for k in ks], [g_dev[k, :P] for k in ks])
+            B.commit_batch_host([order[k] for k in ks], [torch.from_numpy(grads[k].copy()) for k in ks])
+        A.sync()
+        B.sync()
+        assert torch.equal(A.theta(), B.theta())
+        for w in range(n):
+            assert torch.equal(A.moment(w), B.moment(w)) and torch.equal(A.snapshot(w), B.snapshot(w))
+
+
 def test_invalid_arguments_leave_the_handle_usable():
     P, n = 1000, 2
     g = torch.zeros(P + 4, dtype=torch.float32, device="cuda")
