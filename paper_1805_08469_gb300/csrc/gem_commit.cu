@@ -130,7 +130,7 @@ __device__ __forceinline__ void commit_vec_fixed(float4& th, float4& s, const fl
 // each thread owns lanes slot_mem[(2 slot + {0: m, 1: s}) L kThreads + l kThreads + tid]
 // of dynamic shared memory, so no synchronisation is needed.
 template <int L, int RULE, bool REC, int KCAP>
-__global__ void __launch_bounds__(kThreads, RULE == kRuleScaled ? 2 : GEM_COMMIT_MIN_BLOCKS)
+__global__ void __launch_bounds__(kThreads, RULE == kRuleFixed ? GEM_COMMIT_MIN_BLOCKS : 2)
 commit_batch_kernel(const __grid_constant__ BatchArgsT<KCAP> a) {
   extern __shared__ float4 slot_mem[];
   // Launched as a programmatic dependent of the previous kernel in the stream: wait until
@@ -150,6 +150,34 @@ commit_batch_kernel(const __grid_constant__ BatchArgsT<KCAP> a) {
 
   for (size_t base = tid; base < nvec; base += nthreads * L) {
     float4 th[L];
+    // the register slots (static indices only: a slot id selects among them)
+    float4 rm[kRegSlots > 0 ? kRegSlots : 1][L], rs[kRegSlots > 0 ? kRegSlots : 1][L];
+    auto get = [&](int sid, int l, float4& mv, float4* sv) {
+      if (sid < kCommitSlots) {
+        mv = slot_m(sid, l);
+        if (sv) *sv = slot_s(sid, l);
+        return;
+      }
+#pragma unroll
+      for (int r = 0; r < kRegSlots; ++r)
+        if (sid == kCommitSlots + r) {
+          mv = rm[r][l];
+          if (sv) *sv = rs[r][l];
+        }
+    };
+    auto put = [&](int sid, int l, const float4& mv, const float4* sv) {
+      if (sid < kCommitSlots) {
+        slot_m(sid, l) = mv;
+        if (sv) slot_s(sid, l) = *sv;
+        return;
+      }
+#pragma unroll
+      for (int r = 0; r < kRegSlots; ++r)
+        if (sid == kCommitSlots + r) {
+          rm[r][l] = mv;
+          if (sv) rs[r][l] = *sv;
+        }
+    };
 #pragma unroll
     for (int l = 0; l < L; ++l) {
       const size_t i = base + size_t(l) * nthreads;
@@ -168,11 +196,11 @@ commit_batch_kernel(const __grid_constant__ BatchArgsT<KCAP> a) {
         if (i < nvec) {
           g[l] = __ldcs(g4 + i);
           if (RULE == kRuleMomentum) {
-            m[l] = sin >= 0 ? slot_m(sin, l) : load_state(m4 + i);
+            if (sin >= 0) get(sin, l, m[l], nullptr);
+            else m[l] = load_state(m4 + i);
           } else if (RULE != kRuleFixed) {
             if (sin >= 0) {
-              m[l] = slot_m(sin, l);
-              s[l] = slot_s(sin, l);
+              get(sin, l, m[l], &s[l]);
             } else {
               m[l] = load_state(m4 + i);
               s[l] = load_state(s4 + i);
@@ -196,14 +224,13 @@ commit_batch_kernel(const __grid_constant__ BatchArgsT<KCAP> a) {
             commit_coord_momentum(th[l].w, m[l].w, s[l].w, g[l].w, a.eta, a.mu);
             const float nan = __int_as_float(0x7fc00000);
             pi = make_float4(nan, nan, nan, nan);
-            if (sout >= 0) slot_m(sout, l) = m[l];
+            if (sout >= 0) put(sout, l, m[l], nullptr);
             else store_state(m4 + i, m[l]);
             if (a.keep_s[k]) store_state(s4 + i, s[l]);
           } else {
             pi = commit_vec<RULE>(th[l], m[l], s[l], g[l], a.eta, a.mu, a.eps, a.energy_scale);
             if (sout >= 0) {
-              slot_m(sout, l) = m[l];
-              slot_s(sout, l) = s[l];
+              put(sout, l, m[l], &s[l]);
             } else {
               store_state(m4 + i, m[l]);
               store_state(s4 + i, s[l]);
@@ -302,7 +329,7 @@ template <int RULE, bool REC>
 cudaError_t launch_rule(const BatchArgs& a, int sm_count, cudaStream_t stream) {
   bool slots = false;
   if (RULE != kRuleFixed)
-    for (int k = 0; k < a.K; ++k) slots = slots || a.slot_out[k] >= 0;
+    for (int k = 0; k < a.K; ++k) slots = slots || (a.slot_out[k] >= 0 && a.slot_out[k] < kCommitSlots);
   if (a.K > kSmallBatch) return launch_kernel<RULE, REC, kMaxBatchPerLaunch>(a, slots, sm_count, stream);
   BatchArgsT<kSmallBatch> b;
   b.theta = a.theta;
@@ -358,9 +385,9 @@ void plan_slots(BatchArgs& a) {
     a.slot_out[k] = -1;
     a.keep_s[k] = next[k] < 0 ? 1 : 0;
   }
-  if (a.rule == kRuleFixed || kCommitSlots == 0) return;
-  // Choose repeat intervals (k, next[k]) longer than kSlotMinDistance, at most kCommitSlots
-  // open at a time, as many as possible: by increasing end, each into the free slot that
+  if (a.rule == kRuleFixed || kTotalSlots == 0) return;
+  // Choose repeat intervals (k, next[k]) longer than kSlotMinDistance, at most kTotalSlots
+  // (shared-memory and register slots) open at a time, as many as possible: by increasing end, each into the free slot that
   // became free last (greedy, optimal for interval graphs).
   int order[kMaxBatchPerLaunch], cnt = 0;
   for (int k = 0; k < a.K; ++k)
@@ -371,12 +398,12 @@ void plan_slots(BatchArgs& a) {
       order[y] = order[y - 1];
       order[y - 1] = t;
     }
-  int free_at[kCommitSlots > 0 ? kCommitSlots : 1];
-  for (int q = 0; q < kCommitSlots; ++q) free_at[q] = -1;
+  int free_at[kTotalSlots > 0 ? kTotalSlots : 1];
+  for (int q = 0; q < kTotalSlots; ++q) free_at[q] = -1;
   for (int x = 0; x < cnt; ++x) {
     const int k = order[x], e = next[k];
     int best = -1;
-    for (int q = 0; q < kCommitSlots; ++q)
+    for (int q = 0; q < kTotalSlots; ++q)
       if (free_at[q] <= k && (best < 0 || free_at[q] > free_at[best])) best = q;
     if (best < 0) continue;
     free_at[best] = e;

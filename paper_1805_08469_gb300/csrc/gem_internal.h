@@ -69,7 +69,14 @@ constexpr int kSmallBatch = 32;
 #ifndef GEM_COMMIT_SLOT_MIN_DISTANCE
 #define GEM_COMMIT_SLOT_MIN_DISTANCE 4
 #endif
+#ifndef GEM_COMMIT_REG_SLOTS
+#define GEM_COMMIT_REG_SLOTS 1
+#endif
 constexpr int kCommitSlots = GEM_COMMIT_SLOTS;
+// Slots held in registers: ids kCommitSlots .. kCommitSlots + kRegSlots - 1 (one measured
+// best: a second pushes the kernel past 64 registers into a spill).
+constexpr int kRegSlots = GEM_COMMIT_REG_SLOTS;
+constexpr int kTotalSlots = kCommitSlots + kRegSlots;
 constexpr int kSlotMinDistance = GEM_COMMIT_SLOT_MIN_DISTANCE;
 
 // Fill slot_in, slot_out and keep_s of a launch from its a.K workers.
