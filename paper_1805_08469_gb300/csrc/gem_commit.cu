@@ -123,14 +123,18 @@ __device__ __forceinline__ void commit_vec_fixed(float4& th, float4& s, const fl
 // touches 512 contiguous bytes per lane and array.  The fixed-factor rules read only the
 // gradient and write only s_w (12 bytes less per coordinate and commit).
 // The scaled rule asks for two resident blocks per SM: left free, the compiler fits it in
-// 40 registers for three blocks and spills, which costs about 4% of its bandwidth.
+// 40 registers for three blocks and spills, which costs about 4% of its bandwidth.  The
+// energy rules' launches of more than kSmallBatch commits also carry the register slot and
+// ask for two blocks (at most 64 registers); the smaller launches keep the compiler's
+// choice, which measured faster for single commits.
 // REC: the commits whose pi_out[k] is set also store their scaling factors there (4 more
 // bytes per coordinate).
 // A worker that commits again later in the launch can keep its m_w, s_w lanes on chip:
 // each thread owns lanes slot_mem[(2 slot + {0: m, 1: s}) L kThreads + l kThreads + tid]
 // of dynamic shared memory, so no synchronisation is needed.
 template <int L, int RULE, bool REC, int KCAP>
-__global__ void __launch_bounds__(kThreads, RULE == kRuleFixed ? GEM_COMMIT_MIN_BLOCKS : 2)
+__global__ void __launch_bounds__(kThreads, (RULE == kRuleScaled || (RULE != kRuleFixed && KCAP > kSmallBatch))
+                                                 ? 2 : GEM_COMMIT_MIN_BLOCKS)
 commit_batch_kernel(const __grid_constant__ BatchArgsT<KCAP> a) {
   extern __shared__ float4 slot_mem[];
   // Launched as a programmatic dependent of the previous kernel in the stream: wait until
@@ -150,8 +154,12 @@ commit_batch_kernel(const __grid_constant__ BatchArgsT<KCAP> a) {
 
   for (size_t base = tid; base < nvec; base += nthreads * L) {
     float4 th[L];
-    // the register slots (static indices only: a slot id selects among them)
-    float4 rm[kRegSlots > 0 ? kRegSlots : 1][L], rs[kRegSlots > 0 ? kRegSlots : 1][L];
+    // the register slots (static indices only: a slot id selects among them); launches of
+    // at most kSmallBatch commits are planned without them
+    constexpr int kR = KCAP > kSmallBatch ? kRegSlots : 0;
+    float4 rm[kR > 0 ? kR : 1][L], rs[kR > 0 ? kR : 1][L];
+    // slot access: shared-memory slots, and for the large launches also the register slots
+    // (static indices only: a slot id selects among them)
     auto get = [&](int sid, int l, float4& mv, float4* sv) {
       if (sid < kCommitSlots) {
         mv = slot_m(sid, l);
@@ -159,7 +167,7 @@ commit_batch_kernel(const __grid_constant__ BatchArgsT<KCAP> a) {
         return;
       }
 #pragma unroll
-      for (int r = 0; r < kRegSlots; ++r)
+      for (int r = 0; r < kR; ++r)
         if (sid == kCommitSlots + r) {
           mv = rm[r][l];
           if (sv) *sv = rs[r][l];
@@ -172,7 +180,7 @@ commit_batch_kernel(const __grid_constant__ BatchArgsT<KCAP> a) {
         return;
       }
 #pragma unroll
-      for (int r = 0; r < kRegSlots; ++r)
+      for (int r = 0; r < kR; ++r)
         if (sid == kCommitSlots + r) {
           rm[r][l] = mv;
           if (sv) rs[r][l] = *sv;
@@ -196,11 +204,20 @@ commit_batch_kernel(const __grid_constant__ BatchArgsT<KCAP> a) {
         if (i < nvec) {
           g[l] = __ldcs(g4 + i);
           if (RULE == kRuleMomentum) {
-            if (sin >= 0) get(sin, l, m[l], nullptr);
-            else m[l] = load_state(m4 + i);
+            if constexpr (kR > 0) {
+              if (sin >= 0) get(sin, l, m[l], nullptr);
+              else m[l] = load_state(m4 + i);
+            } else {
+              m[l] = sin >= 0 ? slot_m(sin, l) : load_state(m4 + i);
+            }
           } else if (RULE != kRuleFixed) {
             if (sin >= 0) {
-              get(sin, l, m[l], &s[l]);
+              if constexpr (kR > 0) {
+                get(sin, l, m[l], &s[l]);
+              } else {
+                m[l] = slot_m(sin, l);
+                s[l] = slot_s(sin, l);
+              }
             } else {
               m[l] = load_state(m4 + i);
               s[l] = load_state(s4 + i);
@@ -224,13 +241,23 @@ commit_batch_kernel(const __grid_constant__ BatchArgsT<KCAP> a) {
             commit_coord_momentum(th[l].w, m[l].w, s[l].w, g[l].w, a.eta, a.mu);
             const float nan = __int_as_float(0x7fc00000);
             pi = make_float4(nan, nan, nan, nan);
-            if (sout >= 0) put(sout, l, m[l], nullptr);
-            else store_state(m4 + i, m[l]);
+            if constexpr (kR > 0) {
+              if (sout >= 0) put(sout, l, m[l], nullptr);
+              else store_state(m4 + i, m[l]);
+            } else {
+              if (sout >= 0) slot_m(sout, l) = m[l];
+              else store_state(m4 + i, m[l]);
+            }
             if (a.keep_s[k]) store_state(s4 + i, s[l]);
           } else {
             pi = commit_vec<RULE>(th[l], m[l], s[l], g[l], a.eta, a.mu, a.eps, a.energy_scale);
             if (sout >= 0) {
-              put(sout, l, m[l], &s[l]);
+              if constexpr (kR > 0) {
+                put(sout, l, m[l], &s[l]);
+              } else {
+                slot_m(sout, l) = m[l];
+                slot_s(sout, l) = s[l];
+              }
             } else {
               store_state(m4 + i, m[l]);
               store_state(s4 + i, s[l]);
@@ -385,7 +412,8 @@ void plan_slots(BatchArgs& a) {
     a.slot_out[k] = -1;
     a.keep_s[k] = next[k] < 0 ? 1 : 0;
   }
-  if (a.rule == kRuleFixed || kTotalSlots == 0) return;
+  const int total = a.K > kSmallBatch ? kTotalSlots : kCommitSlots;   // see the kernel
+  if (a.rule == kRuleFixed || total == 0) return;
   // Choose repeat intervals (k, next[k]) longer than kSlotMinDistance, at most kTotalSlots
   // (shared-memory and register slots) open at a time, as many as possible: by increasing end, each into the free slot that
   // became free last (greedy, optimal for interval graphs).
@@ -399,11 +427,11 @@ void plan_slots(BatchArgs& a) {
       order[y - 1] = t;
     }
   int free_at[kTotalSlots > 0 ? kTotalSlots : 1];
-  for (int q = 0; q < kTotalSlots; ++q) free_at[q] = -1;
+  for (int q = 0; q < total; ++q) free_at[q] = -1;
   for (int x = 0; x < cnt; ++x) {
     const int k = order[x], e = next[k];
     int best = -1;
-    for (int q = 0; q < kTotalSlots; ++q)
+    for (int q = 0; q < total; ++q)
       if (free_at[q] <= k && (best < 0 || free_at[q] > free_at[best])) best = q;
     if (best < 0) continue;
     free_at[best] = e;
