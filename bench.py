@@ -49,8 +49,8 @@ FALLBACK_HBM_GBS = 6800.0
 # DRAM traffic of one launch of the batched commit kernel, from an ncu capture of the
 # same workload (see profiles/commit_batch_p25m_n100.md).  Valid only for the kernel
 # source it was taken on; reported as null once that source changes.
-NCU_TRAFFIC_BYTES_PER_LAUNCH = 40_241_617_152   # mean of two full-size launches
-NCU_TRAFFIC_SOURCE_SHA = "b8c11a7a7645b70e"
+NCU_TRAFFIC_BYTES_PER_LAUNCH = 40_243_673_600   # mean of two full-size launches
+NCU_TRAFFIC_SOURCE_SHA = "afca98bcd378a8a1"
 
 
 def kernel_source_sha() -> str:

@@ -154,12 +154,11 @@ commit_batch_kernel(const __grid_constant__ BatchArgsT<KCAP> a) {
 
   for (size_t base = tid; base < nvec; base += nthreads * L) {
     float4 th[L];
-    // the register slots (static indices only: a slot id selects among them); launches of
-    // at most kSmallBatch commits are planned without them
+    // Register slots, in launches of more than kSmallBatch commits only (smaller launches
+    // are planned without them, and compile to the shared-memory slots alone); get / put
+    // reach a slot by its id, the register slots through static indices.
     constexpr int kR = KCAP > kSmallBatch ? kRegSlots : 0;
     float4 rm[kR > 0 ? kR : 1][L], rs[kR > 0 ? kR : 1][L];
-    // slot access: shared-memory slots, and for the large launches also the register slots
-    // (static indices only: a slot id selects among them)
     auto get = [&](int sid, int l, float4& mv, float4* sv) {
       if (sid < kCommitSlots) {
         mv = slot_m(sid, l);
