@@ -148,7 +148,6 @@ __global__ void __launch_bounds__(kThreads) select_pick_kernel(const __grid_cons
   constexpr int kPer = kBins / kThreads;     // bins per thread (8)
   __shared__ unsigned wsum[kThreads / 32];
   __shared__ unsigned sst[kState];
-  __shared__ unsigned below_zero;           // first pass: elements with keys below +0
   __shared__ unsigned zeros;                // first pass: elements equal to +0
   const int q = blockIdx.x;
   const int s = q % a.nseg;
@@ -187,20 +186,7 @@ __global__ void __launch_bounds__(kThreads) select_pick_kernel(const __grid_cons
     const unsigned excl = before + incl - sum;
     const unsigned r = sst[3 * t + 2];
     const bool active = sst[3 * t + 1] != 0xffffffffu;   // not resolved in an earlier pass
-    bool in_zeros = false;
-    if (a.pass == 0) {
-      // the keys below +0 fill exactly the bins below +0's bin
-      if (threadIdx.x * kPer == zero_bin) below_zero = excl;
-      __syncthreads();
-      in_zeros = N > 0 && r >= below_zero && r - below_zero < zeros;
-      if (in_zeros && threadIdx.x == 0) {
-        st[3 * t] = kZeroKey;
-        st[3 * t + 1] = 0xffffffffu;
-        st[3 * t + 2] = r - below_zero;
-        (t == 0 ? a.lo : a.hi)[q] = 0.0f;
-      }
-    }
-    if (active && !in_zeros && N > 0 && r >= excl && r - excl < sum) {
+    if (active && N > 0 && r >= excl && r - excl < sum) {
       unsigned c = excl;
       int d = 0;
 #pragma unroll
@@ -211,11 +197,20 @@ __global__ void __launch_bounds__(kThreads) select_pick_kernel(const __grid_cons
         }
         c += local[j];
       }
-      const unsigned prefix = sst[3 * t] | (unsigned(d) << shift);
-      st[3 * t] = prefix;
-      st[3 * t + 1] = sst[3 * t + 1] | ((nb - 1u) << shift);
-      st[3 * t + 2] = r - c;
-      if (a.pass == kPasses - 1) (t == 0 ? a.lo : a.hi)[q] = key_value(prefix);
+      if (a.pass == 0 && d == zero_bin && r - c < zeros) {
+        // +0 is the smallest key of its bin, so the bin's first `zeros` ranks are exact
+        // zeros: the target is +0, resolved now
+        st[3 * t] = kZeroKey;
+        st[3 * t + 1] = 0xffffffffu;
+        st[3 * t + 2] = r - c;
+        (t == 0 ? a.lo : a.hi)[q] = 0.0f;
+      } else {
+        const unsigned prefix = sst[3 * t] | (unsigned(d) << shift);
+        st[3 * t] = prefix;
+        st[3 * t + 1] = sst[3 * t + 1] | ((nb - 1u) << shift);
+        st[3 * t + 2] = r - c;
+        if (a.pass == kPasses - 1) (t == 0 ? a.lo : a.hi)[q] = key_value(prefix);
+      }
     }
     __syncthreads();   // wsum is reused by the next target
   }
