@@ -60,7 +60,16 @@ MISTAKES = [
     ("dropout scale missing from the backward pass", "cnn_oracle.cpp",
      "da2[(size_t(co) * P2 + py) * P2 + px] * drop[int64_t(r) * n.c2 + co];",
      "da2[(size_t(co) * P2 + py) * P2 + px];", "cnn"),
+    ("conv1 as a convolution (flipped kernel) instead of a correlation", "cnn_oracle.cpp",
+     "acc += th[n.w1 + (int64_t(co) * kK + ky) * kK + kx] * x[(yy + ky) * H + xx + kx];",
+     "acc += th[n.w1 + (int64_t(co) * kK + (kK - 1 - ky)) * kK + (kK - 1 - kx)] * x[(yy + ky) * H + xx + kx];",
+     "cnn"),
+    ("conv2 reads the wrong input channel", "cnn_oracle.cpp",
+     "a1[(size_t(ci) * P1 + yy + ky) * P1 + xx + kx];",
+     "a1[(size_t((ci + 1) % n.c1) * P1 + yy + ky) * P1 + xx + kx];", "cnn"),
     # the schedules
+    ("queue commits the latest-finishing worker", "schedule_oracle.cpp",
+     "if (finish[w] < finish[best]) best = w;", "if (finish[w] > finish[best]) best = w;", "schedule"),
     ("uniform tick never picks the last worker", "schedule_oracle.cpp",
      "order[t] = int32_t((u32 * uint64_t(n)) >> 32);",
      "order[t] = int32_t((u32 * uint64_t(n - 1)) >> 32);", "schedule"),
