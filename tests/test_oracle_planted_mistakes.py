@@ -56,6 +56,10 @@ MISTAKES = [
     ("softmax gradient without 1/b", "mlp_oracle.cpp",
      "delta[int64_t(i) * C + c] = (p - (c == y[i] ? 1.0 : 0.0)) / double(b);",
      "delta[int64_t(i) * C + c] = (p - (c == y[i] ? 1.0 : 0.0));", "mlp"),
+    ("TF32 rounding truncates", "mlp_oracle.cpp",
+     "  u += 0x00001000u;\n  u &= 0xFFFFE000u;", "  u &= 0xFFFFE000u;", "mlp"),
+    ("TF32 keeps one mantissa bit too many", "mlp_oracle.cpp",
+     "  u += 0x00001000u;\n  u &= 0xFFFFE000u;", "  u += 0x00000800u;\n  u &= 0xFFFFF000u;", "mlp"),
     # the CNN gradient
     ("dropout scale missing from the backward pass", "cnn_oracle.cpp",
      "da2[(size_t(co) * P2 + py) * P2 + px] * drop[int64_t(r) * n.c2 + co];",
