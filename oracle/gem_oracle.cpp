@@ -1,9 +1,14 @@
 // ORACLE -- test infrastructure, not part of the product.
 //
-// A plain, slow, single-threaded restatement of Gradient Energy Matching (Hermans &
-// Louppe, "Gradient Energy Matching for Distributed Asynchronous Gradient Descent",
-// arXiv 1805.08469).  Only the tests, the smoke check and the CPU-baseline leg of the
-// benchmark may load it.  It shares no source, header or constant with the CUDA path.
+// A plain, slow restatement of Gradient Energy Matching (Hermans & Louppe, "Gradient
+// Energy Matching for Distributed Asynchronous Gradient Descent", arXiv 1805.08469).  Only
+// the tests, the smoke check and the CPU-baseline leg of the benchmark may load it.  It
+// shares no source, header or constant with the CUDA path.
+//
+// It runs on one thread unless oracle_set_commit_threads asks for more.  Then the
+// coordinates of each commit are split across threads: every step of Psi_GEM and of the
+// update is elementwise (Algorithm 1 uses the elementwise product), so coordinate j's
+// result depends only on element j of each input, and the split changes no result.
 //
 // Build with -O2 -ffp-contract=off: every floating-point operation below is one IEEE
 // operation with its own rounding (no fused multiply-add), in the precision of T.
@@ -23,8 +28,13 @@
 #include <cmath>
 #include <cstdint>
 #include <cstring>
+#ifdef _OPENMP
+#include <omp.h>
+#endif
 
 namespace {
+
+int g_commit_threads = 1;  // threads over the coordinates of one commit
 
 // Commit modes.  GEM is Algorithm 1; the others are the comparison rules of the
 // experiments section and the high-energy proxies of Appendix B.
@@ -99,6 +109,7 @@ int run(int64_t P, int n, int T_commits, const int32_t* order, const int32_t* ta
     T* sw = s + int64_t(w) * state_stride;
     const int tw = tau ? tau[t] : 0;
     T* pi_row = pi_record ? pi_record + int64_t(t) * P : nullptr;
+#pragma omp parallel for schedule(static) num_threads(g_commit_threads) if (g_commit_threads > 1)
     for (int64_t j = 0; j < P; ++j) {
       const T pi = commit_coordinate<T>(theta[j], mw[j], sw[j], g[j], eta, mu, eps, mode, kappa,
                                         tw, precommit_snapshot);
@@ -113,6 +124,14 @@ int run(int64_t P, int n, int T_commits, const int32_t* order, const int32_t* ta
 }  // namespace
 
 extern "C" {
+
+// Threads that split the coordinates of each commit (1, the default, runs the loop on the
+// calling thread; values below 1 are taken as 1).  Returns the previous value.
+int oracle_set_commit_threads(int threads) {
+  const int prev = g_commit_threads;
+  g_commit_threads = threads < 1 ? 1 : threads;
+  return prev;
+}
 
 // Apply T_commits commits in schedule order.  Commit t is made by worker order[t] with
 // the gradient row grads[grad_index[t] * grad_stride .. + P) (row t when grad_index is

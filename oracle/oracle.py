@@ -46,6 +46,8 @@ def lib():
         _lib.oracle_schedule_queue.restype = C.c_int
         _lib.oracle_tf32_rna.argtypes = [C.c_float]
         _lib.oracle_tf32_rna.restype = C.c_float
+        _lib.oracle_set_commit_threads.argtypes = [i32]
+        _lib.oracle_set_commit_threads.restype = C.c_int
         _lib.oracle_threads.argtypes = []
         _lib.oracle_threads.restype = C.c_int
         _lib.oracle_mlp_loss_grad_f64.argtypes = [i32, p, p, p, p, i32, p, i32]
@@ -177,6 +179,13 @@ def tf32_rna(x: float) -> float:
 
 def threads() -> int:
     return int(lib().oracle_threads())
+
+
+def set_commit_threads(threads: int) -> int:
+    """Threads that split the coordinates of each commit of gem_run (1 by default).  The
+    result does not depend on it: every coordinate is updated independently.  Returns the
+    previous value."""
+    return int(lib().oracle_set_commit_threads(int(threads)))
 
 
 def mlp_loss_grad(dims, theta, X, y, *, tf32=False):

@@ -292,3 +292,29 @@ def test_kappa_variants():
                    mode=oracle.MODE_KAPPA_LINEAR, kappa=2.0)
     nz = g[0] != 0
     np.testing.assert_allclose(th[nz], theta0[nz] - 2 * 0.01 * g[0][nz].astype(np.float64), rtol=1e-12)
+
+
+def test_commit_threads_change_no_bit():
+    # Psi_GEM and the update are elementwise (Algorithm 1), so splitting each commit's
+    # coordinates across threads (the CPU baseline's multi-core run) must leave every bit
+    # of theta, m, s and the recorded factors unchanged, for every commit rule.
+    rng = np.random.default_rng(31)
+    n, P, T = 5, 10_007, 40
+    theta0 = (0.05 * rng.standard_normal(P)).astype(np.float32)
+    g = (0.1 * rng.standard_normal((T, P))).astype(np.float32)
+    order = rng.integers(0, n, T)
+    tau = rng.integers(0, 7, T)
+    for mode in (oracle.MODE_GEM, oracle.MODE_ADAPTIVE, oracle.MODE_KAPPA_LINEAR,
+                 oracle.MODE_MOMENTUM):
+        out = []
+        for threads in (1, 4):
+            prev = oracle.set_commit_threads(threads)
+            try:
+                st = _fresh(theta0, n, np.float32)
+                pi = oracle.gem_run(*st, g, order, tau=tau, eta=0.01, mu=0.9, eps=1e-8,
+                                    mode=mode, kappa=2.0, record_pi=True)
+            finally:
+                oracle.set_commit_threads(prev)
+            out.append((*st, pi))
+        for a, b in zip(*out):
+            assert np.array_equal(a, b, equal_nan=True), mode

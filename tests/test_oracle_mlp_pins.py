@@ -150,11 +150,8 @@ def test_gem_on_the_mlp_amplifies_tiny_differences():
     commit 99.  Two correct fp32 implementations that sum in different orders therefore
     agree to 1e-4 over the first 100 commits only; this sets the free-running horizon of the
     GPU trajectory tests (the windowed tests cover the rest)."""
-    from paper_1805_08469_gb300 import sim
-    from paper_1805_08469_gb300._build import build_library
-    build_library()
     dims, n, b, T, seed = [784, 64, 10], 4, 32, 200, 1
-    order = sim.gem_schedule_uniform(seed, n, T)[0]
+    order = oracle.schedule_uniform(seed, n, T)[0]
     batches = synth.schedule_batches(seed, order, b)
     rows, inv = np.unique(batches, return_inverse=True)
     X = synth.data_rows(seed, rows, 784)
