@@ -193,68 +193,73 @@ def _oracle_e2e(dims, n, seed, inputs, T, record_at, tf32):
     return rec, losses
 
 
-def _oracle_states(dims, n, seed, inputs, checkpoints, tf32):
-    """Oracle state (theta, m, s) right before commit c, for every c in checkpoints."""
-    order, batches, theta0 = inputs
-    T = max(checkpoints)
-    Xh, yh, local = host_rows(seed, batches[:T])
-    P = theta0.size
-    th = theta0.copy()
-    m = np.zeros((n, P), np.float32)
-    s = np.tile(theta0, (n, 1))
-    states, losses, t = {}, np.empty(T), 0
-    for c in sorted(set(checkpoints)):
-        if c > t:
-            _r, ls = oracle.mlp_sim_run(dims, th, m, s, order[t:c], Xh, yh, local[t:c], eta=ETA, mu=MU,
-                                        eps=EPS, tf32=tf32, want_losses=True)
-            losses[t:c] = ls
-        states[c] = (th.copy(), m.copy(), s.copy())
-        t = c
-    return states, losses
-
-
 def _windows(dims, n, b, seed, schedule, precision, starts, W, tol):
-    """Windowed trajectory parity: the GPU resumes from the oracle's full state before
-    commit c (gem_load_state), runs commits c .. c+W-1 and must land on the oracle's state."""
+    """Windowed trajectory parity: the oracle runs the schedule from theta_0; before each
+    commit c in `starts` the GPU takes the oracle's full state (theta, m, s through
+    gem_load_state), runs commits c .. c+W-1, and must land on the oracle's state after
+    them.  The oracle's state is advanced in place, so a late window costs the oracle the
+    whole run up to it but holds only one copy of the state."""
     P = synth.mlp_param_count(dims)
     T = max(starts) + W
     order = schedule(seed, n, T)[0]
     batches = synth.schedule_batches(seed, order, b)
     theta0 = synth.xavier_theta0(seed, dims)
     tf32 = precision == sim.GEM_MLP_TF32
-    states, ref_losses = _oracle_states(dims, n, seed, (order, batches, theta0),
-                                        list(starts) + [c + W for c in starts], tf32)
+    lay = synth.mlp_layout(dims)
+    Xh, yh, local = host_rows(seed, batches)
+    th = theta0.copy()
+    m = np.zeros((n, P), np.float32)
+    s = np.tile(theta0, (n, 1))
+
+    def advance(t0, t1):
+        _r, ls = oracle.mlp_sim_run(dims, th, m, s, order[t0:t1], Xh, yh, local[t0:t1], eta=ETA,
+                                    mu=MU, eps=EPS, tf32=tf32, want_losses=True)
+        return ls
+
     X, y = device_data(seed)
-    worst = 0.0
+    worst, t = 0.0, 0
     with gem.Gem(P, n, ETA, MU, EPS) as G:
         M = sim.gem_mlp_create(G.h, dims, b, precision)
         try:
             sim.gem_mlp_set_data(M, X, y)
             losses = torch.empty(W, device="cuda")
-            for c in starts:
-                th, m, s = states[c]
+            for c in sorted(starts):
+                if c > t:
+                    advance(t, c)
                 gem.gem_load_state(G.h, th, m, s)
                 sim.gem_mlp_run(M, order[c:c + W], batches[c:c + W], losses)
                 G.sync()
-                th1, m1, s1 = states[c + W]
+                ref_losses = advance(c, c + W)
+                t = c + W
                 got = G.theta().cpu().numpy()
-                err = rel_l2(got, th1)
+                err = rel_l2(got, th)
                 worst = max(worst, err)
                 assert err < tol, (c, err)
                 for w in set(order[c:c + W].tolist()):
-                    # m_w is gradient-sized: a ReLU pre-activation within fp32 rounding of
-                    # zero (about one per gradient) flips a mask and moves one gradient row,
-                    # visible in m's norm but not in theta's.  Most elements must agree.
+                    # m_w is gradient-sized, and a ReLU pre-activation within fp32 rounding
+                    # of zero may take either side (both are right at fp32 accuracy).  A flip
+                    # in the first hidden layer moves one row of W_1's gradient; a flip in a
+                    # later hidden layer changes one sample's delta for every unit below it,
+                    # so every element of the deeper blocks by that sample's share (measured:
+                    # one layer-2 decision at -3e-8 of its scale moved W_1's gradient by 1.4e-3
+                    # relative L2, and flipping it in the oracle reproduced the GPU's gradient
+                    # to 3e-7).  So every block of m is compared in L2, and element by element
+                    # only the last layer's blocks, which no hidden-layer decision reaches.
                     # With TF32 operands the deeper layers' gradients are themselves
                     # sensitive at the 1% level (see the gradient test), so m gets that bar.
-                    gm, om = G.moment(w).cpu().numpy(), m1[w]
+                    gm, om = G.moment(w).cpu().numpy(), m[w]
                     if tf32:
                         assert rel_l2(gm, om) < 5e-2, (c, w, "m", rel_l2(gm, om))
                     else:
-                        close = np.abs(gm - om) <= 1e-3 * np.abs(om) + 1e-3 * np.sqrt(np.mean(om ** 2))
-                        assert close.mean() > 0.999 and rel_l2(gm, om) < 1e-2, (c, w, "m", close.mean())
-                    assert rel_l2(G.snapshot(w).cpu().numpy(), s1[w]) < tol, (c, w, "s")
-                np.testing.assert_allclose(losses.cpu().numpy(), ref_losses[c:c + W], rtol=10 * tol)
+                        for li, (wo, bo, fo, fi) in enumerate(lay):
+                            for a0, a1 in ((wo, wo + fo * fi), (bo, bo + fo)):
+                                assert rel_l2(gm[a0:a1], om[a0:a1]) < 1e-2, (c, w, "m", li, a0)
+                        wo, bo, fo, fi = lay[-1]
+                        gl, ol = gm[wo:bo + fo], om[wo:bo + fo]
+                        close = np.abs(gl - ol) <= 1e-3 * np.abs(ol) + 1e-3 * np.sqrt(np.mean(ol ** 2))
+                        assert close.mean() > 0.999, (c, w, "m last layer", close.mean())
+                    assert rel_l2(G.snapshot(w).cpu().numpy(), s[w]) < tol, (c, w, "s")
+                np.testing.assert_allclose(losses.cpu().numpy(), ref_losses, rtol=10 * tol)
         finally:
             sim.gem_mlp_destroy(M)
     return worst
@@ -264,7 +269,7 @@ def _windows(dims, n, b, seed, schedule, precision, starts, W, tol):
 def test_config1_windows_cover_the_whole_run():
     """MLP 784-64-10, n = 4, b = 32, 200 uniform-tick commits (seed 1): ten windows of 20
     commits, each resumed from the oracle's state, cover the whole run at 1e-4."""
-    _windows([784, 64, 10], 4, 32, 1, sim.gem_schedule_uniform, sim.GEM_MLP_FP32,
+    _windows([784, 64, 10], 4, 32, 1, oracle.schedule_uniform, sim.GEM_MLP_FP32,
              list(range(0, 200, 20)), 20, 1e-4)
 
 
@@ -276,7 +281,7 @@ def test_config1_free_running_trajectory():
     by 2e-3 at commit 199; see test_oracle_mlp_pins)."""
     dims, n, b, T, seed = [784, 64, 10], 4, 32, 200, 1
     rec_at = [0, 1, 9, 49, 99, 199]
-    recs, losses, final, inputs = _e2e(dims, n, b, T, seed, sim.gem_schedule_uniform,
+    recs, losses, final, inputs = _e2e(dims, n, b, T, seed, oracle.schedule_uniform,
                                        sim.GEM_MLP_FP32, rec_at)
     ref, ref_losses = _oracle_e2e(dims, n, seed, inputs, T, rec_at, False)
     for r, t in enumerate(rec_at[:-1]):
@@ -290,7 +295,7 @@ def test_config1_free_running_trajectory():
 
 def _drop_out_schedule(seed, n, T, gone=1, after=15):
     """Uniform ticks with worker `gone` leaving after tick `after`."""
-    base = sim.gem_schedule_uniform(seed, n, 3 * T)[0]
+    base = oracle.schedule_uniform(seed, n, 3 * T)[0]
     order = np.array([w for t, w in enumerate(base) if not (w == gone and t >= after)][:T], np.int32)
     return order, None
 
@@ -315,11 +320,11 @@ def test_config3_windows_and_prefix():
     """MLP 784-1000-1000-10, n = 30, b = 128, exponential-queue schedule (seed 3): windows
     of 20 commits resumed from the oracle at commits 0, 40 and 80 (1e-4), and the
     free-running trajectory for the first 60 commits (1e-4)."""
-    _windows([784, 1000, 1000, 10], 30, 128, 3, sim.gem_schedule_queue, sim.GEM_MLP_FP32,
+    _windows([784, 1000, 1000, 10], 30, 128, 3, oracle.schedule_queue, sim.GEM_MLP_FP32,
              [0, 40, 80], 20, 1e-4)
     dims, n, b, T, seed = [784, 1000, 1000, 10], 30, 128, 60, 3
     rec_at = [0, 29, 59]
-    recs, losses, _f, inputs = _e2e(dims, n, b, T, seed, sim.gem_schedule_queue, sim.GEM_MLP_FP32, rec_at)
+    recs, losses, _f, inputs = _e2e(dims, n, b, T, seed, oracle.schedule_queue, sim.GEM_MLP_FP32, rec_at)
     ref, ref_losses = _oracle_e2e(dims, n, seed, inputs, T, rec_at, False)
     for r, t in enumerate(rec_at):
         assert rel_l2(recs[r], ref[r]) < 1e-4, (t, rel_l2(recs[r], ref[r]))
@@ -331,11 +336,11 @@ def test_config4_windows_and_prefix_tf32():
     """MLP 784-1000-1000-10, n = 100, b = 128, TF32 products, uniform tick (seed 4):
     windows at commits 0, 50 and 100 and the free-running first 120 commits, at 2e-3
     against the oracle's TF32 mode."""
-    _windows([784, 1000, 1000, 10], 100, 128, 4, sim.gem_schedule_uniform, sim.GEM_MLP_TF32,
+    _windows([784, 1000, 1000, 10], 100, 128, 4, oracle.schedule_uniform, sim.GEM_MLP_TF32,
              [0, 50, 100], 20, 2e-3)
     dims, n, b, T, seed = [784, 1000, 1000, 10], 100, 128, 120, 4
     rec_at = [0, 59, 119]
-    recs, losses, _final, inputs = _e2e(dims, n, b, T, seed, sim.gem_schedule_uniform,
+    recs, losses, _final, inputs = _e2e(dims, n, b, T, seed, oracle.schedule_uniform,
                                         sim.GEM_MLP_TF32, rec_at)
     ref, ref_losses = _oracle_e2e(dims, n, seed, inputs, T, rec_at, True)
     for r, t in enumerate(rec_at):
@@ -344,13 +349,36 @@ def test_config4_windows_and_prefix_tf32():
 
 
 @pytest.mark.slow
+def test_config3_late_windows():
+    """Config 3 late in its 2,000-commit run: windows of 20 commits resumed from the oracle's
+    state before commits 500, 1,000 and 1,980 land within 1e-4.  This is the regime the
+    early windows never reach: a lower loss, fresh gradients small beside the workers'
+    moments, median factors well below 1.  The oracle runs the whole schedule to get there
+    (about 80 s on 16 host cores)."""
+    worst = _windows([784, 1000, 1000, 10], 30, 128, 3, oracle.schedule_queue, sim.GEM_MLP_FP32,
+                     [500, 1000, 1980], 20, 1e-4)
+    print(f"config 3 late windows: worst relative L2 {worst:.2e}")
+
+
+@pytest.mark.slow
+def test_config4_late_windows_tf32():
+    """Config 4 (TF32 products, n = 100) late in its 5,000-commit run: windows of 20 commits
+    resumed from the oracle's state before commits 1,000, 2,500 and 4,980 land within 2e-3
+    of the oracle's TF32 mode.  The oracle runs the whole schedule to get there (about
+    5.5 minutes on 16 host cores)."""
+    worst = _windows([784, 1000, 1000, 10], 100, 128, 4, oracle.schedule_uniform,
+                     sim.GEM_MLP_TF32, [1000, 2500, 4980], 20, 2e-3)
+    print(f"config 4 late windows: worst relative L2 {worst:.2e}")
+
+
+@pytest.mark.slow
 @pytest.mark.parametrize("n,T,schedule,precision", [
-    (30, 2000, sim.gem_schedule_queue, sim.GEM_MLP_FP32),
-    (100, 5000, sim.gem_schedule_uniform, sim.GEM_MLP_TF32),
+    (30, 2000, oracle.schedule_queue, sim.GEM_MLP_FP32),
+    (100, 5000, oracle.schedule_uniform, sim.GEM_MLP_TF32),
 ])
 def test_full_length_runs_train(n, T, schedule, precision):
     """Full-length configs 3 and 4 on the GPU: theta stays finite and the minibatch loss
-    falls (the oracle would need tens of minutes here; the prefixes above pin parity)."""
+    falls.  Parity along these runs is pinned by the early and late windows above."""
     dims, b, seed = [784, 1000, 1000, 10], 128, 3 if n == 30 else 4
     _r, losses, final, _inp = _e2e(dims, n, b, T, seed, schedule, precision, [])
     assert np.all(np.isfinite(final)) and np.all(np.isfinite(losses))
