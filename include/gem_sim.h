@@ -115,14 +115,18 @@ uint64_t gem_mlp_launch_count(const gem_mlp_t* mlp);
  * device-wide synchronisation is not allowed.  Nothing is allocated and no handle is needed:
  * the caller passes the inputs (theta [P] in device memory, the data set X [rows][dims[0]]
  * and labels [rows] in device memory, the minibatch batch_rows [batch] as a host array,
- * checked and copied before the call returns) and the outputs (grad [P], device, 16-byte
- * aligned; loss, device, may be NULL).  The scratch is one file-scope device array of 4 MiB
- * (1,048,576 floats) held by every GPU that loads the library until the process exits; a
- * network whose per-minibatch activations and deltas do not fit in it is rejected with
- * GEM_EINVAL.  The first call on a device looks up the array's device address, so make it
- * before any stream capture.  Calls share the array: calls that overlap on the GPU (other
- * streams, other host threads) race; order them on one stream.  The paper has no
- * counterpart to this entry point. */
+ * checked and passed by value in a kernel's argument block, so the host array may be reused
+ * as soon as the call returns) and the outputs (grad [P], device, 16-byte aligned; loss,
+ * device, may be NULL).  The scratch is one file-scope device array of 4 MiB (1,048,576
+ * floats) held by every GPU that loads the library until the process exits; a network whose
+ * per-minibatch activations and deltas (plus the batch's row indices) do not fit in it is
+ * rejected with GEM_EINVAL.  The first call on a device looks up the array's device
+ * address, so make it before any stream capture; the address is looked up again if the
+ * device's current context changes (after a reset of its primary context, say).  Calls
+ * share the array and keep nothing in it between calls: calls queued one after another on
+ * one stream are ordered, while calls that overlap on the GPU (other streams, other host
+ * threads) race; order them on one stream.  The paper has no counterpart to this entry
+ * point. */
 int gem_mlp_grad_static(int n_layers, const int32_t* dims, int batch, int precision,
                         const float* theta, const float* X, const int32_t* labels,
                         int64_t rows, const int32_t* batch_rows, float* grad, float* loss,

@@ -19,6 +19,8 @@
 // Precision.  Every product runs in one grouped SIMT GEMM kernel that reads either operand
 // layout; with GEM_MLP_TF32 it rounds each operand to TF32 as it loads it (products of TF32
 // values are exact in fp32; the sums stay fp32).
+#include <cuda.h>
+
 #include <cstdint>
 #include <cstring>
 #include <mutex>
@@ -1464,7 +1466,7 @@ int gem_mlp_run_pi(gem_mlp_t* M, const int32_t* order, int T, const int32_t* bat
 // Gradient without allocation (gem_mlp_grad_static).  Its scratch is this file-scope device
 // array: every GPU that loads the library holds it until the process exits.  Host code
 // cannot pass the symbol itself to a kernel (on the host it names a stand-in object, not
-// device memory), so its device address is looked up once per device.
+// device memory), so its device address is looked up once per device and context.
 namespace {
 
 constexpr long long kStaticScratchFloats = 1ll << 20;  // 4 MiB
@@ -1472,22 +1474,62 @@ __device__ __align__(256) float g_static_scratch[kStaticScratchFloats];
 
 constexpr int kMaxDevices = 64;
 std::mutex g_static_mutex;
-float* g_static_addr[kMaxDevices] = {};
+struct StaticAddress {
+  CUcontext ctx;  // the context the address was looked up in
+  float* addr;
+};
+StaticAddress g_static_addr[kMaxDevices] = {};
 
-// Device address of g_static_scratch on the current device (looked up on first use).
+// The driver's current context, through the runtime's entry-point query (the library does
+// not link the driver library itself, so it loads on machines without a GPU driver).
+CUcontext current_context() {
+  using GetCurrent = CUresult (*)(CUcontext*);
+  static GetCurrent fn = nullptr;
+  static bool looked = false;
+  if (!looked) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess && q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<GetCurrent>(p);
+    cudaGetLastError();
+    looked = true;
+  }
+  CUcontext ctx = nullptr;
+  if (!fn || fn(&ctx) != CUDA_SUCCESS) return nullptr;
+  return ctx;
+}
+
+// Device address of g_static_scratch on the current device.  Looked up on the first call
+// in a context, and again when the current context is another one (after a reset of the
+// device's primary context, for instance).  Called with g_static_mutex held.
 int static_scratch(int device, float** out) {
   if (device < 0 || device >= kMaxDevices) return GEM_EINVAL;
-  std::lock_guard<std::mutex> lock(g_static_mutex);
-  if (!g_static_addr[device]) {
+  StaticAddress& e = g_static_addr[device];
+  CUcontext ctx = current_context();
+  if (!e.addr || !ctx || e.ctx != ctx) {
     void* ptr = nullptr;
     if (cudaGetSymbolAddress(&ptr, g_static_scratch) != cudaSuccess || !ptr) {
       cudaGetLastError();
       return GEM_ECUDA;
     }
-    g_static_addr[device] = static_cast<float*>(ptr);
+    // the lookup makes the device's primary context current if none was
+    e.ctx = current_context();
+    e.addr = static_cast<float*>(ptr);
   }
-  *out = g_static_addr[device];
+  *out = e.addr;
   return GEM_OK;
+}
+
+// The minibatch rows of one call, passed by value in the argument block and stored in the
+// static array where the gradient kernels read them (no copy from pageable host memory).
+struct StaticRows {
+  int32_t row[kMaxBatch];
+  int count;
+};
+
+__global__ void static_rows_kernel(const __grid_constant__ StaticRows a, int32_t* dst) {
+  for (int i = threadIdx.x; i < a.count; i += blockDim.x) dst[i] = a.row[i];
 }
 
 }  // namespace
@@ -1550,6 +1592,7 @@ extern "C" int gem_mlp_grad_static(int n_layers, const int32_t* dims, int batch,
     return GEM_ECUDA;
   }
   float* scratch = nullptr;
+  std::lock_guard<std::mutex> lock(g_static_mutex);
   int rc = static_scratch(device, &scratch);
   if (rc) return rc;
   h.device = device;
@@ -1560,9 +1603,13 @@ extern "C" int gem_mlp_grad_static(int n_layers, const int32_t* dims, int batch,
   h.stream = static_cast<cudaStream_t>(stream);
   M.scratch = scratch;
   int32_t* rows_dev = reinterpret_cast<int32_t*>(scratch + off);
-  if (cudaMemcpyAsync(rows_dev, batch_rows, sizeof(int32_t) * size_t(batch), cudaMemcpyHostToDevice,
-                      h.stream) != cudaSuccess)
-    return GEM_ECUDA;
+  // an ordinary launch: it starts after all earlier work on the stream, including the
+  // kernels of a previous call that still read the rows it overwrites
+  StaticRows ra;
+  std::memcpy(ra.row, batch_rows, sizeof(int32_t) * size_t(batch));
+  ra.count = batch;
+  static_rows_kernel<<<1, 256, 0, h.stream>>>(ra, rows_dev);
+  if (cudaGetLastError() != cudaSuccess) return GEM_ECUDA;
   const int32_t worker = 0;
   rc = mlp_chunk(&M, &worker, 1, rows_dev, grad, 0, loss);
   M.gem = nullptr;

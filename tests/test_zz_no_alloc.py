@@ -5,13 +5,16 @@ device memory through its own pool, or in a loop where cudaMalloc's device-wide
 synchronisation is not allowed.  For them the library offers a gradient call whose scratch is
 a fixed file-scope device array.  This test checks, through the C ABI, that two calls in a
 row give the same gradients and losses as the allocating entry point (gem_mlp_grad, at its
-worker's snapshot), within the precision's rounding tolerance, and that a network
-too large for the array is refused.  It sits in a file of its own, collected last.
+worker's snapshot), within the precision's rounding tolerance; that two calls queued on one
+caller-created stream with no synchronisation between them (they share the array and its
+row slot) each give their own minibatch's gradient, pinned in fp32 to the oracle's; and that
+a network too large for the array is refused.  It sits in a file of its own, collected last.
 """
 import numpy as np
 import pytest
 import torch
 
+import oracle
 from paper_1805_08469_gb300 import gem, sim, synth, synth_gpu
 from paper_1805_08469_gb300._build import build_library
 from paper_1805_08469_gb300._lib import GemError
@@ -66,6 +69,46 @@ def test_static_scratch_gradient_matches_allocating_entry_point(dims, b, precisi
                 assert abs(float(loss) - float(ref_loss)) <= bar * abs(float(ref_loss))
         finally:
             sim.gem_mlp_destroy(M)
+
+
+@pytest.mark.parametrize("dims,b", [([784, 64, 10], 32), ([37, 19, 5, 3], 7)])
+def test_static_scratch_calls_queued_on_one_stream(dims, b):
+    """Two calls with different minibatches queued back to back on one stream the caller
+    created, with no synchronisation between them: the second call's rows and activations
+    overwrite the first's in the shared array only after the first call's kernels are done,
+    so each gradient is its own minibatch's.  Both are checked against the oracle's gradient
+    (double, rounded to fp32) at 1e-5 relative L2, the fp32 gradient bar."""
+    build_library()
+    torch.cuda.set_device(0)
+    seed = 37
+    P = synth.mlp_param_count(dims)
+    X = torch.empty((synth.DATA_ROWS, dims[0]), device="cuda")
+    y = torch.empty(synth.DATA_ROWS, dtype=torch.int32, device="cuda")
+    synth_gpu.data(seed, X, y, dims[-1])
+    theta0 = synth.xavier_theta0(seed, dims)
+    for (_wo, bo, fo, _fi) in synth.mlp_layout(dims):
+        theta0[bo:bo + fo] = 0.05 * synth.normal(synth.key(seed, 78), np.arange(bo, bo + fo))
+    theta = torch.from_numpy(theta0).cuda()
+    rows = [synth.batch_indices(seed, 0, k, b) for k in range(2)]
+    stream = torch.cuda.Stream()
+    grads = [torch.full((P,), float("nan"), device="cuda") for _ in rows]
+    losses = [torch.full((1,), float("nan"), device="cuda") for _ in rows]
+    torch.cuda.synchronize()
+    for k in range(2):
+        sim.gem_mlp_grad_static(dims, b, sim.GEM_MLP_FP32, theta, X, y, rows[k], grads[k],
+                                losses[k], stream=stream)
+    stream.synchronize()
+    got = [g.cpu().numpy() for g in grads]
+    got_loss = [float(l.cpu()) for l in losses]
+    for k in range(2):
+        uniq, inv = np.unique(rows[k], return_inverse=True)
+        Xh = synth.data_rows(seed, uniq, dims[0]).astype(np.float64)
+        yh = synth.teacher_labels(seed, uniq, dims[0], dims[-1])
+        loss, g = oracle.mlp_loss_grad(dims, theta0.astype(np.float64), Xh[inv], yh[inv])
+        err = float(np.linalg.norm(got[k] - g) / np.linalg.norm(g))
+        assert err < 1e-5, (k, err)
+        assert abs(got_loss[k] - loss) <= 1e-5 * abs(loss), (k, got_loss[k], loss)
+    assert not np.array_equal(got[0], got[1])
 
 
 def test_static_scratch_rejects_networks_that_do_not_fit():
