@@ -212,6 +212,20 @@ int gem_commit_batch_pi(gem_t* h, const int* order, const float* const* grads, i
 int gem_pi_median(gem_t* h, const float* const* pi, int K, const int64_t* seg, int nseg,
                   float* lo, float* hi);
 
+/* gem_commit_batch_pi with every factor recorded (each pi[k] set, 16-byte aligned), followed
+ * by gem_pi_median of the K recorded rows with segments seg[0..nseg], in one call, with the
+ * same results bit for bit (commits, recorded rows, lo and hi).  The commit kernel also
+ * counts, for every row and segment, the factors below +0 and equal to +0 as it writes them
+ * (the median of the experiments section is often +0 at many workers, where most clamped
+ * factors are exactly 0): a middle element inside the run of +0 is then known without a
+ * selection pass, and a row and segment whose two middle elements both lie there is never
+ * read back.  Commits are taken in chunks of at most 200 (at most 2048 / nseg), each a
+ * commit launch followed by the selection of its rows.  The first call, and any call with
+ * more rows per chunk or segments than before, allocates the select scratch. */
+int gem_commit_batch_pi_median(gem_t* h, const int* order, const float* const* grads, int K,
+                               float* const* pi, const int64_t* seg, int nseg, float* lo,
+                               float* hi);
+
 /* Number of kernels this handle has launched since it was created. */
 uint64_t gem_launch_count(const gem_t* h);
 

@@ -80,8 +80,15 @@ int ensure_staging(gem_t* h) {
 namespace gem {
 
 cudaError_t commit_ordered(gem_ctx* h, const int* order, const float* const* grads, int K,
-                           float* const* pi_out) {
+                           float* const* pi_out, unsigned* pi_counts, const long long* pi_seg,
+                           int pi_nseg) {
+  if (pi_counts && (K > kMaxBatchPerLaunch || K * pi_nseg * 2 > kMaxCountWords || !pi_out))
+    return cudaErrorInvalidValue;   // counts are kept by one launch
   BatchArgs a;
+  a.pi_counts = pi_counts;
+  a.pi_seg = pi_seg;
+  a.pi_nseg = pi_nseg;
+  a.count_smem_at = 0;
   a.theta = h->theta;
   a.m = h->m;
   a.s = h->s;
@@ -382,6 +389,34 @@ int gem_pi_median(gem_t* h, const float* const* pi, int K, const int64_t* seg, i
   DeviceScope scope(h->device);
   if (!scope.ok()) return GEM_ECUDA;
   const cudaError_t e = gem::pi_median_ordered(h, pi, K, seg, nseg, lo, hi);
+  if (e == cudaErrorMemoryAllocation) {
+    cudaGetLastError();
+    return GEM_ENOMEM;
+  }
+  return cuda_status(h, e);
+}
+
+int gem_commit_batch_pi_median(gem_t* h, const int* order, const float* const* grads, int K,
+                               float* const* pi, const int64_t* seg, int nseg, float* lo,
+                               float* hi) {
+  int rc = check_handle(h);
+  if (rc) return rc;
+  rc = check_batch(h, order, grads, K);
+  if (rc) return rc;
+  if (nseg < 1 || nseg > gem::kMaxPiSegments || !seg) return GEM_EINVAL;
+  if (seg[0] < 0 || seg[nseg] > int64_t(h->P)) return GEM_EINVAL;
+  for (int i = 0; i < nseg; ++i)
+    if (seg[i + 1] < seg[i] || seg[i + 1] - seg[i] > int64_t(UINT32_MAX)) return GEM_EINVAL;
+  if (K == 0) return GEM_OK;
+  if (!pi || !lo || !hi) return GEM_EINVAL;
+  const uintptr_t align4 = 3u;
+  if ((reinterpret_cast<uintptr_t>(lo) & align4) || (reinterpret_cast<uintptr_t>(hi) & align4))
+    return GEM_EINVAL;
+  for (int k = 0; k < K; ++k)
+    if (!pi[k] || !aligned16(pi[k])) return GEM_EINVAL;
+  DeviceScope scope(h->device);
+  if (!scope.ok()) return GEM_ECUDA;
+  const cudaError_t e = gem::commit_pi_median_ordered(h, order, grads, K, pi, seg, nseg, lo, hi);
   if (e == cudaErrorMemoryAllocation) {
     cudaGetLastError();
     return GEM_ENOMEM;

@@ -100,6 +100,26 @@ __device__ __forceinline__ void commit_coord_momentum(float& theta, float& m, fl
   s = theta;
 }
 
+// Segment s with seg[s] <= j < seg[s + 1] (the last such s when segments are empty), or -1
+// when j lies outside [seg[0], seg[nseg]).
+__device__ __forceinline__ int segment_of(const long long* seg, int nseg, long long j) {
+  if (j < seg[0] || j >= seg[nseg]) return -1;
+  int lo = 0, hi = nseg;   // seg[lo] <= j < seg[hi]
+  while (hi - lo > 1) {
+    const int mid = (lo + hi) >> 1;
+    if (seg[mid] <= j) lo = mid;
+    else hi = mid;
+  }
+  return lo;
+}
+
+// Factors below +0 (sign bit set: negatives, -0, negative NaN) and equal to +0.
+__device__ __forceinline__ void count_factor(float x, unsigned& below, unsigned& zero) {
+  const unsigned u = __float_as_uint(x);
+  below += u >> 31;
+  zero += u == 0u ? 1u : 0u;
+}
+
 template <int RULE>
 __device__ __forceinline__ float4 commit_vec(float4& th, float4& m, float4& s, const float4 g,
                                              float eta, float mu, float eps, float scale) {
@@ -128,7 +148,10 @@ __device__ __forceinline__ void commit_vec_fixed(float4& th, float4& s, const fl
 // ask for two blocks (at most 64 registers); the smaller launches keep the compiler's
 // choice, which measured faster for single commits.
 // REC: the commits whose pi_out[k] is set also store their scaling factors there (4 more
-// bytes per coordinate).
+// bytes per coordinate), and with pi_counts set count them per segment (factors below +0
+// and equal to +0): per warp with one reduction, into the block's counters in shared
+// memory, added to pi_counts when the block ends.  The lane loop of these launches runs
+// while any lane of the warp has coordinates, so the warp reductions see every lane.
 // A worker that commits again later in the launch can keep its m_w, s_w lanes on chip:
 // each thread owns lanes slot_mem[(2 slot + {0: m, 1: s}) L kThreads + l kThreads + tid]
 // of dynamic shared memory, so no synchronisation is needed.
@@ -145,6 +168,16 @@ commit_batch_kernel(const __grid_constant__ BatchArgsT<KCAP> a) {
   const size_t nthreads = size_t(gridDim.x) * kThreads;
   const size_t tid = size_t(blockIdx.x) * kThreads + threadIdx.x;
   float4* theta4 = reinterpret_cast<float4*>(a.theta);
+  const unsigned lane = threadIdx.x & 31u;
+  // factor counters of this block (recording launches with counts only)
+  unsigned* cnt = nullptr;
+  if constexpr (REC) {
+    if (a.pi_counts) {
+      cnt = reinterpret_cast<unsigned*>(slot_mem + a.count_smem_at);
+      for (int q = threadIdx.x; q < a.K * a.pi_nseg * 2; q += kThreads) cnt[q] = 0u;
+      __syncthreads();
+    }
+  }
   auto slot_m = [&](int slot, int l) -> float4& {
     return slot_mem[(2 * slot) * L * kThreads + l * kThreads + threadIdx.x];
   };
@@ -152,8 +185,24 @@ commit_batch_kernel(const __grid_constant__ BatchArgsT<KCAP> a) {
     return slot_mem[(2 * slot + 1) * L * kThreads + l * kThreads + threadIdx.x];
   };
 
-  for (size_t base = tid; base < nvec; base += nthreads * L) {
+  for (size_t base = tid; (REC ? base - lane : base) < nvec; base += nthreads * L) {
     float4 th[L];
+    // segment of each lane's four coordinates: >= 0 one segment, -1 outside every segment
+    // (or no coordinates), -2 the four straddle a boundary; uni: the warp's lanes share one
+    int sid[L];
+    bool uni[L];
+    if constexpr (REC) {
+#pragma unroll
+      for (int l = 0; l < L; ++l) {
+        const size_t i = base + size_t(l) * nthreads;
+        sid[l] = -1;
+        if (cnt && i < nvec) {
+          sid[l] = segment_of(a.pi_seg, a.pi_nseg, (long long)(4 * i));
+          if (segment_of(a.pi_seg, a.pi_nseg, (long long)(4 * i + 3)) != sid[l]) sid[l] = -2;
+        }
+        uni[l] = __all_sync(0xffffffffu, sid[l] == __shfl_sync(0xffffffffu, sid[l], 0));
+      }
+    }
     // Register slots, in launches of more than kSmallBatch commits only (smaller launches
     // are planned without them, and compile to the shared-memory slots alone); get / put
     // reach a slot by its id, the register slots through static indices.
@@ -197,6 +246,7 @@ commit_batch_kernel(const __grid_constant__ BatchArgsT<KCAP> a) {
       float4* s4 = reinterpret_cast<float4*>(a.s + row);
       const int sin = a.slot_in[k], sout = a.slot_out[k];
       float4 g[L], m[L], s[L];
+      float4 pi_l[L];   // the factors of this commit (recording launches)
 #pragma unroll
       for (int l = 0; l < L; ++l) {
         const size_t i = base + size_t(l) * nthreads;
@@ -263,6 +313,46 @@ commit_batch_kernel(const __grid_constant__ BatchArgsT<KCAP> a) {
             }
           }
           if (REC && a.pi_out[k]) reinterpret_cast<float4*>(a.pi_out[k])[i] = pi;
+          if constexpr (REC) pi_l[l] = pi;
+        }
+      }
+      if constexpr (REC) {
+        if (cnt && a.pi_out[k]) {
+#pragma unroll
+          for (int l = 0; l < L; ++l) {
+            const size_t i = base + size_t(l) * nthreads;
+            unsigned below = 0u, zero = 0u;
+            if (i < nvec && sid[l] != -1) {
+              count_factor(pi_l[l].x, below, zero);
+              count_factor(pi_l[l].y, below, zero);
+              count_factor(pi_l[l].z, below, zero);
+              count_factor(pi_l[l].w, below, zero);
+            }
+            if (uni[l]) {
+              // one segment (or none) for the whole warp: one reduction, one lane adds
+              below = __reduce_add_sync(0xffffffffu, below);
+              zero = __reduce_add_sync(0xffffffffu, zero);
+              if (lane == 0 && sid[l] >= 0) {
+                unsigned* c = cnt + 2 * (k * a.pi_nseg + sid[l]);
+                if (below) atomicAdd(c, below);
+                if (zero) atomicAdd(c + 1, zero);
+              }
+            } else if (sid[l] >= 0) {
+              unsigned* c = cnt + 2 * (k * a.pi_nseg + sid[l]);
+              if (below) atomicAdd(c, below);
+              if (zero) atomicAdd(c + 1, zero);
+            } else if (sid[l] == -2) {
+              // the four coordinates straddle a segment boundary: one by one
+              const float v[4] = {pi_l[l].x, pi_l[l].y, pi_l[l].z, pi_l[l].w};
+#pragma unroll
+              for (int e = 0; e < 4; ++e) {
+                const int se = segment_of(a.pi_seg, a.pi_nseg, (long long)(4 * i + e));
+                unsigned b1 = 0u, z1 = 0u;
+                count_factor(v[e], b1, z1);
+                if (se >= 0 && (b1 | z1)) atomicAdd(cnt + 2 * (k * a.pi_nseg + se) + (b1 ? 0 : 1), 1u);
+              }
+            }
+          }
         }
       }
     }
@@ -297,9 +387,24 @@ commit_batch_kernel(const __grid_constant__ BatchArgsT<KCAP> a) {
         a.m[row + j] = m;
       }
       a.s[row + j] = s;
-      if (REC && a.pi_out[k]) a.pi_out[k][j] = pi;
+      if (REC && a.pi_out[k]) {
+        a.pi_out[k][j] = pi;
+        if (cnt) {
+          const int se = segment_of(a.pi_seg, a.pi_nseg, (long long)j);
+          unsigned b1 = 0u, z1 = 0u;
+          count_factor(pi, b1, z1);
+          if (se >= 0 && (b1 | z1)) atomicAdd(cnt + 2 * (k * a.pi_nseg + se) + (b1 ? 0 : 1), 1u);
+        }
+      }
     }
     a.theta[j] = th;
+  }
+  if constexpr (REC) {
+    if (cnt) {
+      __syncthreads();
+      for (int q = threadIdx.x; q < a.K * a.pi_nseg * 2; q += kThreads)
+        if (cnt[q]) atomicAdd(a.pi_counts + q, cnt[q]);
+    }
   }
 }
 
@@ -309,15 +414,27 @@ constexpr int kLanes = GEM_COMMIT_LANES;
 // requested only when the launch keeps a worker on chip; without it more blocks fit on an
 // SM.  Occupancy is computed once per instantiation and shared-memory size.
 template <int RULE, bool REC, int KCAP>
-cudaError_t launch_kernel(const BatchArgsT<KCAP>& a, bool slots, int sm_count, cudaStream_t stream) {
-  const int smem = slots ? kCommitSlots * 2 * kLanes * kThreads * 16 : 0;
+cudaError_t launch_kernel(BatchArgsT<KCAP> a, bool slots, int sm_count, cudaStream_t stream) {
+  const int slot_bytes = slots ? kCommitSlots * 2 * kLanes * kThreads * 16 : 0;
+  // factor counters after the slots, in whole float4 (recording launches with counts)
+  const int count_bytes = (REC && a.pi_counts) ? (a.K * a.pi_nseg * 2 * 4 + 15) / 16 * 16 : 0;
+  a.count_smem_at = slot_bytes / 16;
+  const int smem = slot_bytes + count_bytes;
   static int blocks_per_sm[2] = {0, 0};
-  int& bps = blocks_per_sm[slots ? 1 : 0];
+  int counted_bps = 0;
+  int& bps = count_bytes ? counted_bps : blocks_per_sm[slots ? 1 : 0];
   if (bps == 0) {
-    if (smem > 48 * 1024) {
-      cudaError_t e = cudaFuncSetAttribute(commit_batch_kernel<kLanes, RULE, REC, KCAP>,
-                                           cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-      if (e != cudaSuccess) return e;
+    static bool attr_set = false;
+    if (!attr_set) {
+      // the most any launch of this instantiation asks for: every slot and the largest
+      // counter block
+      const int most = kCommitSlots * 2 * kLanes * kThreads * 16 + (REC ? kMaxCountWords * 4 : 0);
+      if (most > 48 * 1024) {
+        cudaError_t e = cudaFuncSetAttribute(commit_batch_kernel<kLanes, RULE, REC, KCAP>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, most);
+        if (e != cudaSuccess) return e;
+      }
+      attr_set = true;
     }
     int b = 0;
     cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(
@@ -370,6 +487,10 @@ cudaError_t launch_rule(const BatchArgs& a, int sm_count, cudaStream_t stream) {
   b.rule = a.rule;
   b.energy_scale = a.energy_scale;
   b.record_pi = a.record_pi;
+  b.pi_counts = a.pi_counts;
+  b.pi_seg = a.pi_seg;
+  b.pi_nseg = a.pi_nseg;
+  b.count_smem_at = 0;
   for (int k = 0; k < kSmallBatch; ++k) {
     const bool in = k < a.K;
     b.grad[k] = in ? a.grad[k] : nullptr;

@@ -49,6 +49,15 @@ struct BatchArgsT {
   float pi[KCAP];                          // kRuleFixed: scaling factor of commit k
   int record_pi;                           // 1: pi_out[k] (when not null) receives pi
   float* pi_out[KCAP];                     // scaling factors of commit k, P floats, or null
+  // Factor counts of a recording launch (null: none).  For every commit k with pi_out[k]
+  // set and every segment s = [pi_seg[s], pi_seg[s + 1]) of the coordinates, the number of
+  // recorded factors whose sign bit is set (below +0 in the total order of the medians) is
+  // added to pi_counts[2 (k pi_nseg + s)] and the number equal to +0 to the word after it.
+  // The block keeps its counts in dynamic shared memory from float4 count_smem_at on.
+  unsigned* pi_counts;
+  const long long* pi_seg;                 // device array [pi_nseg + 1], non-decreasing
+  int pi_nseg;
+  int count_smem_at;
   // On-chip reuse of a worker that commits again later in the launch (energy rules):
   // commit k keeps its m_w, s_w lanes in shared-memory slot slot_out[k] instead of writing
   // them to global memory, and the worker's next commit reads them from slot_in[k];
@@ -85,6 +94,10 @@ void plan_slots(BatchArgs& a);
 // Launch the fused commit kernel for a.K commits on `stream`.
 cudaError_t launch_commit_batch(const BatchArgs& a, int sm_count, cudaStream_t stream);
 
+// Shared-memory words a recording launch may use for its factor counts (2 per commit and
+// segment); callers split their commits so that K * pi_nseg * 2 stays within it.
+constexpr int kMaxCountWords = 4096;
+
 }  // namespace gem
 
 struct gem_ctx {
@@ -120,8 +133,11 @@ namespace gem {
 // Launch commits [0, K) of the handle in order, in chunks of kMaxBatchPerLaunch, with the
 // handle's commit rule; advances the commit clock and counts the launches.  The arguments
 // must have been checked.
+// With pi_counts set (K * pi_nseg * 2 <= kMaxCountWords, one launch), the recording launch
+// also adds the factor counts of every commit and segment to pi_counts (see BatchArgsT).
 cudaError_t commit_ordered(gem_ctx* h, const int* order, const float* const* grads, int K,
-                           float* const* pi_out = nullptr);
+                           float* const* pi_out = nullptr, unsigned* pi_counts = nullptr,
+                           const long long* pi_seg = nullptr, int pi_nseg = 0);
 
 // Segments per median call and commits per select launch.
 constexpr int kMaxPiSegments = 64;
@@ -133,5 +149,14 @@ constexpr int kMaxPiBatch = 200;
 // caller.
 cudaError_t pi_median_ordered(gem_ctx* h, const float* const* pi, int K, const int64_t* seg,
                               int nseg, float* lo, float* hi);
+
+// Commits [0, K) in order with every factor recorded in pi[k] (all set), then the lower and
+// upper medians of each row and segment as pi_median_ordered.  The recording launches also
+// count each row's factors below and equal to +0 per segment, so a middle element that lies
+// in the run of zeros is known before any selection pass, and a row and segment whose two
+// middle elements both lie there is never read again.  Arguments checked by the caller.
+cudaError_t commit_pi_median_ordered(gem_ctx* h, const int* order, const float* const* grads,
+                                     int K, float* const* pi, const int64_t* seg, int nseg,
+                                     float* lo, float* hi);
 
 }  // namespace gem

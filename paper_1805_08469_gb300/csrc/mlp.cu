@@ -1430,14 +1430,15 @@ int mlp_run(gem_mlp_t* M, const int32_t* order, int T, const int32_t* batch_rows
         gptr[size_t(k)] = M->grads + (long long)(k - a) * h->stride;
         if (want_pi) pptr[size_t(k)] = M->pi_rows + (long long)(k - a) * h->stride;
       }
-      rc = cuda_rc(gem::commit_ordered(h, order + a, gptr.data() + a, e - a,
-                                       want_pi ? pptr.data() + a : nullptr));
-    }
-    if (rc == GEM_OK && want_pi) {
-      const cudaError_t ce = gem::pi_median_ordered(h, pptr.data() + a, e - a, tensors, nseg,
-                                                     pi_lo + (long long)a * nseg,
-                                                     pi_hi + (long long)a * nseg);
-      rc = ce == cudaErrorMemoryAllocation ? GEM_ENOMEM : cuda_rc(ce);
+      if (!want_pi) {
+        rc = cuda_rc(gem::commit_ordered(h, order + a, gptr.data() + a, e - a));
+      } else {
+        // commits with their factors recorded and counted, then the per-tensor medians
+        const cudaError_t ce = gem::commit_pi_median_ordered(
+            h, order + a, gptr.data() + a, e - a, pptr.data() + a, tensors, nseg,
+            pi_lo + (long long)a * nseg, pi_hi + (long long)a * nseg);
+        rc = ce == cudaErrorMemoryAllocation ? GEM_ENOMEM : cuda_rc(ce);
+      }
     }
   }
   if (rc == GEM_ECUDA) h->broken = true;

@@ -25,6 +25,10 @@
 // +0's first-pass bin, so a target whose rank falls in the run of zeros is resolved after
 // one pass (its mask becomes full), and later passes skip it, and skip a problem whose
 // targets are both resolved.
+// Fused with the commit (commit_pi_median_ordered): the recording commit kernel counts, per
+// row and segment, the factors below +0 and equal to +0 while it writes them.  With those
+// counts the init kernel resolves every target whose rank lies in the run of zeros before
+// any pass, and a problem with both targets resolved is never read.
 #include <cmath>
 
 #include "gem_internal.h"
@@ -51,6 +55,7 @@ struct SelectArgs {
   int K, nseg, pass;
   unsigned* hist;                           // [K][nseg][2][kBins]
   unsigned* state;                          // [K][nseg][kState]: 2 x (prefix, mask, rank)
+  const unsigned* counts;                   // [K][nseg][2]: factors below +0, equal to +0; or null
   float* lo;                                // [K][nseg]
   float* hi;                                // [K][nseg]
 };
@@ -78,6 +83,37 @@ __global__ void select_init_kernel(const __grid_constant__ SelectArgs a) {
   st[3] = 0u;
   st[4] = 0u;
   st[5] = unsigned(N / 2);
+  if (a.counts && N > 0) {
+    // elements below +0 come first in the order, then the run of +0: a target whose rank
+    // falls in that run is +0, resolved without a pass
+    const unsigned below = a.counts[2 * q], zeros = a.counts[2 * q + 1];
+    for (int t = 0; t < 2; ++t) {
+      const unsigned r = st[3 * t + 2];
+      if (r >= below && r - below < zeros) {
+        st[3 * t] = kZeroKey;
+        st[3 * t + 1] = 0xffffffffu;
+        st[3 * t + 2] = r - below;
+        (t == 0 ? a.lo : a.hi)[q] = 0.0f;
+      }
+    }
+  }
+}
+
+// Counts of a fused commit: clears them and stores the segment offsets where the commit
+// kernel reads them.
+struct CountInitArgs {
+  unsigned* counts;                         // [K][nseg][2]
+  int words;
+  long long* seg_dev;                       // [nseg + 1]
+  long long seg[kMaxPiSegments + 1];
+  int nseg;
+};
+
+__global__ void count_init_kernel(const __grid_constant__ CountInitArgs a) {
+  gem::pdl_entry();
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i < a.words) a.counts[i] = 0u;
+  if (i <= a.nseg) a.seg_dev[i] = a.seg[i];
 }
 
 // Adds one element's digit to a shared histogram when its key matches the prefix; every
@@ -158,7 +194,9 @@ __global__ void __launch_bounds__(kThreads) select_pick_kernel(const __grid_cons
   if (threadIdx.x == 0) zeros = a.pass == 0 ? g[kBins] : 0u;
   __syncthreads();
   const int zero_bin = int(kZeroKey >> digit_shift(0));   // +0's first-pass bin
-  const bool two = sst[0] != sst[3] || sst[1] != sst[4];
+  // the first pass fills one histogram for both targets (a target resolved by the fused
+  // counts is skipped below, so their prefixes may differ then)
+  const bool two = a.pass > 0 && (sst[0] != sst[3] || sst[1] != sst[4]);
   const int shift = digit_shift(a.pass);
   const unsigned nb = 1u << digit_bits(a.pass);
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -223,12 +261,24 @@ __global__ void __launch_bounds__(kThreads) select_pick_kernel(const __grid_cons
 
 }  // namespace
 
-cudaError_t pi_median_ordered(gem_ctx* h, const float* const* pi, int K, const int64_t* seg,
-                              int nseg, float* lo, float* hi) {
-  if (K <= 0) return cudaSuccess;
-  const int kc_max = K < kMaxPiBatch ? K : kMaxPiBatch;
-  const size_t hist_bytes = size_t(kc_max) * nseg * 2 * kBins * sizeof(unsigned);
-  const size_t need = hist_bytes + size_t(kc_max) * nseg * kState * sizeof(unsigned);
+namespace {
+
+// The handle's select scratch for chunks of up to kc rows of nseg segments: histograms,
+// per-problem state, factor counts and the segment offsets (grown on demand).
+struct SelectScratch {
+  unsigned* hist;
+  unsigned* state;
+  unsigned* counts;
+  long long* seg;
+};
+
+cudaError_t select_scratch(gem_ctx* h, int kc, int nseg, SelectScratch* out) {
+  const size_t problems = size_t(kc) * nseg;
+  const size_t hist_bytes = problems * 2 * kBins * sizeof(unsigned);
+  const size_t state_bytes = problems * kState * sizeof(unsigned);
+  const size_t count_bytes = (problems * 2 * sizeof(unsigned) + 15) / 16 * 16;
+  const size_t seg_bytes = size_t(kMaxPiSegments + 1) * sizeof(long long);
+  const size_t need = hist_bytes + state_bytes + count_bytes + seg_bytes;
   if (need > h->select_bytes) {
     cudaFree(h->select_scratch);   // waits for work still using the old buffer
     h->select_scratch = nullptr;
@@ -237,7 +287,16 @@ cudaError_t pi_median_ordered(gem_ctx* h, const float* const* pi, int K, const i
     if (e != cudaSuccess) return e;
     h->select_bytes = need;
   }
-  SelectArgs a;
+  char* base = static_cast<char*>(h->select_scratch);
+  out->hist = reinterpret_cast<unsigned*>(base);
+  out->state = reinterpret_cast<unsigned*>(base + hist_bytes);
+  out->counts = reinterpret_cast<unsigned*>(base + hist_bytes + state_bytes);
+  out->seg = reinterpret_cast<long long*>(base + hist_bytes + state_bytes + count_bytes);
+  return cudaSuccess;
+}
+
+// Segment offsets and histogram blocks of a select.
+int prepare_args(SelectArgs& a, const int64_t* seg, int nseg) {
   a.nseg = nseg;
   a.block_start[0] = 0;
   for (int s = 0; s <= nseg; ++s) a.seg[s] = seg[s];
@@ -245,34 +304,92 @@ cudaError_t pi_median_ordered(gem_ctx* h, const float* const* pi, int K, const i
     const long long N = seg[s + 1] - seg[s];
     a.block_start[s + 1] = a.block_start[s] + int((N + kChunk - 1) / kChunk);
   }
-  const int blocks = a.block_start[nseg];
-  a.hist = static_cast<unsigned*>(h->select_scratch);
-  a.state = reinterpret_cast<unsigned*>(static_cast<char*>(h->select_scratch) + hist_bytes);
+  return a.block_start[nseg];
+}
+
+// The select of rows a.pi[0 .. kc) (a.lo, a.hi, a.counts set by the caller).
+cudaError_t select_rows(gem_ctx* h, SelectArgs& a, int kc, int blocks) {
+  a.K = kc;
+  a.pass = 0;
+  cudaError_t e = cudaMemsetAsync(a.hist, 0, size_t(kc) * a.nseg * 2 * kBins * sizeof(unsigned),
+                                  h->stream);
+  if (e != cudaSuccess) return e;
+  gem::launch_pdl(select_init_kernel, (kc * a.nseg + 127) / 128, 128, 0, h->stream, a);
+  h->launches += 1;
+  for (int p = 0; p < kPasses; ++p) {
+    a.pass = p;
+    if (blocks > 0) {
+      if (p == 0)
+        gem::launch_pdl(select_hist_kernel<true>, dim3(unsigned(blocks), unsigned(kc)), kThreads, 0, h->stream, a);
+      else
+        gem::launch_pdl(select_hist_kernel<false>, dim3(unsigned(blocks), unsigned(kc)), kThreads, 0, h->stream, a);
+      h->launches += 1;
+    }
+    gem::launch_pdl(select_pick_kernel, unsigned(kc * a.nseg), kThreads, 0, h->stream, a);
+    h->launches += 1;
+  }
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t pi_median_ordered(gem_ctx* h, const float* const* pi, int K, const int64_t* seg,
+                              int nseg, float* lo, float* hi) {
+  if (K <= 0) return cudaSuccess;
+  const int kc_max = K < kMaxPiBatch ? K : kMaxPiBatch;
+  SelectScratch sc;
+  cudaError_t e = select_scratch(h, kc_max, nseg, &sc);
+  if (e != cudaSuccess) return e;
+  SelectArgs a;
+  const int blocks = prepare_args(a, seg, nseg);
+  a.hist = sc.hist;
+  a.state = sc.state;
+  a.counts = nullptr;
   for (int k0 = 0; k0 < K; k0 += kMaxPiBatch) {
     const int kc = (K - k0) < kMaxPiBatch ? (K - k0) : kMaxPiBatch;
-    a.K = kc;
     for (int k = 0; k < kc; ++k) a.pi[k] = pi[k0 + k];
     a.lo = lo + size_t(k0) * nseg;
     a.hi = hi + size_t(k0) * nseg;
-    a.pass = 0;
-    cudaError_t e = cudaMemsetAsync(a.hist, 0, size_t(kc) * nseg * 2 * kBins * sizeof(unsigned),
-                                    h->stream);
+    e = select_rows(h, a, kc, blocks);
     if (e != cudaSuccess) return e;
-    gem::launch_pdl(select_init_kernel, (kc * nseg + 127) / 128, 128, 0, h->stream, a);
+  }
+  return cudaSuccess;
+}
+
+cudaError_t commit_pi_median_ordered(gem_ctx* h, const int* order, const float* const* grads,
+                                     int K, float* const* pi, const int64_t* seg, int nseg,
+                                     float* lo, float* hi) {
+  if (K <= 0) return cudaSuccess;
+  // commits per chunk: one commit launch, one select, and the counters in shared memory
+  int per = kMaxCountWords / (2 * nseg);
+  if (per > kMaxBatchPerLaunch) per = kMaxBatchPerLaunch;
+  if (per > kMaxPiBatch) per = kMaxPiBatch;
+  const int kc_max = K < per ? K : per;
+  SelectScratch sc;
+  cudaError_t e = select_scratch(h, kc_max, nseg, &sc);
+  if (e != cudaSuccess) return e;
+  SelectArgs a;
+  const int blocks = prepare_args(a, seg, nseg);
+  a.hist = sc.hist;
+  a.state = sc.state;
+  a.counts = sc.counts;
+  CountInitArgs ci;
+  ci.counts = sc.counts;
+  ci.seg_dev = sc.seg;
+  ci.nseg = nseg;
+  for (int s = 0; s <= nseg; ++s) ci.seg[s] = seg[s];
+  for (int k0 = 0; k0 < K; k0 += per) {
+    const int kc = (K - k0) < per ? (K - k0) : per;
+    ci.words = kc * nseg * 2;
+    const int n_init = ci.words > nseg + 1 ? ci.words : nseg + 1;
+    gem::launch_pdl(count_init_kernel, (n_init + 255) / 256, 256, 0, h->stream, ci);
     h->launches += 1;
-    for (int p = 0; p < kPasses; ++p) {
-      a.pass = p;
-      if (blocks > 0) {
-        if (p == 0)
-          gem::launch_pdl(select_hist_kernel<true>, dim3(unsigned(blocks), unsigned(kc)), kThreads, 0, h->stream, a);
-        else
-          gem::launch_pdl(select_hist_kernel<false>, dim3(unsigned(blocks), unsigned(kc)), kThreads, 0, h->stream, a);
-        h->launches += 1;
-      }
-      gem::launch_pdl(select_pick_kernel, unsigned(kc * nseg), kThreads, 0, h->stream, a);
-      h->launches += 1;
-    }
-    e = cudaGetLastError();
+    e = commit_ordered(h, order + k0, grads + k0, kc, pi + k0, sc.counts, sc.seg, nseg);
+    if (e != cudaSuccess) return e;
+    for (int k = 0; k < kc; ++k) a.pi[k] = pi[k0 + k];
+    a.lo = lo + size_t(k0) * nseg;
+    a.hi = hi + size_t(k0) * nseg;
+    e = select_rows(h, a, kc, blocks);
     if (e != cudaSuccess) return e;
   }
   return cudaSuccess;

@@ -127,6 +127,22 @@ def gem_pi_median(h: int, pi: Sequence, seg: Sequence[int], lo, hi) -> None:
           "gem_pi_median")
 
 
+def gem_commit_batch_pi_median(h: int, order: Sequence[int], grads: Sequence, pi: Sequence,
+                               seg: Sequence[int], lo, hi) -> None:
+    """gem_commit_batch_pi with every factor recorded in pi[k] ([P] float32 CUDA tensors),
+    then the per-segment lower / upper medians of those rows into lo, hi [K, nseg], with the
+    factor counts taken by the commit kernel.  Stream-ordered."""
+    o, g, K = _batch_arrays(order, [_dev_ptr(x, "grads[k]") for x in grads])
+    if len(pi) != K:
+        raise ValueError("order and pi differ in length")
+    rows = (C.c_void_p * max(K, 1))(*[_dev_ptr(x, "pi[k]") for x in pi])
+    sg = (C.c_int64 * len(seg))(*[int(x) for x in seg])
+    check(lib().gem_commit_batch_pi_median(C.c_void_p(h), o, g, K, rows, sg, len(seg) - 1,
+                                           C.c_void_p(_dev_ptr(lo, "lo")),
+                                           C.c_void_p(_dev_ptr(hi, "hi"))),
+          "gem_commit_batch_pi_median")
+
+
 def gem_commit_batch_host(h: int, order: Sequence[int], grads: Sequence) -> None:
     ptrs = []
     for x in grads:
@@ -281,6 +297,9 @@ class Gem:
 
     def commit_batch_pi(self, order, grads, pi):
         gem_commit_batch_pi(self.h, order, grads, pi)
+
+    def commit_batch_pi_median(self, order, grads, pi, seg, lo, hi):
+        gem_commit_batch_pi_median(self.h, order, grads, pi, seg, lo, hi)
 
     def pi_median(self, pi, seg, lo, hi):
         gem_pi_median(self.h, pi, seg, lo, hi)

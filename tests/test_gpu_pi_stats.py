@@ -112,18 +112,26 @@ def test_medians_of_ties_signs_and_infinities():
 
 
 def test_medians_at_the_edges_of_a_zero_run():
-    """Runs of exact +0 (the clamp of the factor) next to negatives, -0 and positives, with
-    the run ending between the lower and the upper middle element; compared bit for bit,
-    so a -0 returned for +0 (or the reverse) fails."""
+    """Runs of exact +0 (the clamp of the factor) next to negatives, -0, positives and
+    positive subnormals, with the run ending between the lower and the upper middle element
+    or just before both; compared bit for bit, so a -0 returned for +0 (or the reverse), or
+    a subnormal ranked as if the zeros were not counted, fails."""
     rng = np.random.default_rng(4)
     P = 50_000
     pos = lambda n: (rng.exponential(size=n) + 1e-3).astype(np.float32)
+    sub = lambda n: rng.integers(1, 0x200000, n).astype(np.uint32).view(np.float32)
     parts = [
         [np.zeros(25_000), pos(25_000)],                                  # lo = +0, hi > 0
         [-pos(25_000), np.zeros(25_000)],                                 # lo < 0, hi = +0
         [-pos(10_000), np.zeros(30_000), pos(10_000)],                    # both +0 after negatives
         [-pos(20_000), np.full(10_000, -0.0), np.zeros(10_000), pos(10_000)],   # both -0
         [np.full(25_000, -0.0), np.zeros(25_000)],                        # lo = -0, hi = +0
+        # positive subnormals (bit patterns 1 .. 0x1FFFFF) share the first pass's bin with
+        # +0: middle elements just past the zeros must be ranked among the subnormals
+        [np.zeros(24_990), sub(25_010)],                                  # both subnormal
+        [np.zeros(25_000), sub(25_000)],                                  # lo = +0, hi subnormal
+        [-pos(1_000), np.zeros(23_998), sub(25_002)],                     # both just past the zeros
+        [-pos(1_000), np.full(500, -0.0), np.zeros(22_000), sub(26_500)],
     ]
     rows = np.stack([rng.permutation(np.concatenate(p).astype(np.float32)) for p in parts])
     dev = _padded(rows)
@@ -352,3 +360,130 @@ def test_mlp_run_pi_windows_resumed_from_the_oracle():
                     np.testing.assert_allclose(ghi[i], rhi, rtol=1e-3, atol=1e-7, err_msg=f"commit {c + i}")
         finally:
             sim.gem_mlp_destroy(M)
+
+
+def _segments(P, kind):
+    if kind == "one":
+        return [0, P]
+    # empty segments, a segment of one coordinate, boundaries inside float4 groups
+    a, b = max(1, P // 3), max(2, P - 2)
+    return sorted({0, 1, a, b, P} | {1}) if P > 4 else [0, 1, 1, 2, 2, P]
+
+
+@pytest.mark.parametrize("mode,omode,kappa", [
+    (gem.GEM_MODE_GEM, oracle.MODE_GEM, 1.0),
+    (gem.GEM_MODE_KAPPA_LINEAR, oracle.MODE_KAPPA_LINEAR, 2.0),
+    (gem.GEM_MODE_ADAPTIVE, oracle.MODE_ADAPTIVE, 1.0),
+    (gem.GEM_MODE_MOMENTUM, oracle.MODE_MOMENTUM, 1.0),
+])
+@pytest.mark.parametrize("P,kind", [(5, "one"), (5, "many"), (4099, "many"), (100_003, "one"),
+                                    (100_003, "many")])
+def test_fused_commit_medians_equal_separate_calls_and_oracle(mode, omode, kappa, P, kind):
+    """gem_commit_batch_pi_median against gem_commit_batch_pi + gem_pi_median on a second
+    handle: theta, m, s, the recorded rows and both medians bit for bit; the medians also
+    bit for bit against the oracle's sorted factors.  230 commits (two chunks)."""
+    n, T = 5, 230
+    seg = _segments(P, kind)
+    nseg = len(seg) - 1
+    theta0, grads, order, tau = _inputs(P, n, T, 700 + P)
+    th, m, s = theta0.copy(), np.zeros((n, P), np.float32), np.tile(theta0, (n, 1))
+    ref_pi = oracle.gem_run(th, m, s, grads, order, eta=ETA, mu=MU, eps=EPS, tau=tau, mode=omode,
+                            kappa=kappa, record_pi=True)
+    g_dev = _padded(grads)
+    Pp = (P + 3) // 4 * 4
+    pa = torch.full((T, Pp), -1.0, device="cuda")
+    pb = torch.full((T, Pp), -1.0, device="cuda")
+    lo_a, hi_a = (torch.full((T, nseg), -2.0, device="cuda") for _ in range(2))
+    lo_b, hi_b = (torch.full((T, nseg), -2.0, device="cuda") for _ in range(2))
+    gl = [g_dev[k, :P] for k in range(T)]
+    with gem.Gem(P, n, ETA, MU, EPS) as A, gem.Gem(P, n, ETA, MU, EPS) as B:
+        for G in (A, B):
+            G.set_mode(mode, kappa)
+            G.set_theta(torch.from_numpy(theta0).cuda())
+        A.commit_batch_pi_median(order.tolist(), gl, [pa[k, :P] for k in range(T)], seg, lo_a, hi_a)
+        B.commit_batch_pi(order.tolist(), gl, [pb[k, :P] for k in range(T)])
+        B.pi_median([pb[k, :P] for k in range(T)], seg, lo_b, hi_b)
+        A.sync()
+        B.sync()
+        assert torch.equal(A.theta(), B.theta())
+        for w in range(n):
+            assert torch.equal(A.moment(w), B.moment(w)) and torch.equal(A.snapshot(w), B.snapshot(w))
+        assert np.array_equal(A.theta().cpu().numpy(), th)
+    bits = lambda t: t.cpu().numpy().view(np.uint32)
+    assert np.array_equal(bits(pa), bits(pb))
+    assert np.array_equal(pa.cpu().numpy()[:, :P], ref_pi, equal_nan=True)
+    for x, y in ((lo_a, lo_b), (hi_a, hi_b)):
+        assert np.array_equal(bits(x), bits(y))
+    glo, ghi = lo_a.cpu().numpy(), hi_a.cpu().numpy()
+    for k in range(T):
+        rlo, rhi = oracle.pi_median(ref_pi[k], seg)
+        assert np.array_equal(glo[k], rlo, equal_nan=True), (k, glo[k], rlo)
+        assert np.array_equal(ghi[k], rhi, equal_nan=True), (k, ghi[k], rhi)
+
+
+@pytest.mark.parametrize("P", [1000, 40_002])
+def test_fused_counts_at_the_edges_of_the_zero_run(P):
+    """One worker without momentum: the factor of a coordinate is exactly +0 where its
+    gradient is 0 and positive elsewhere (no drift, m = dtheta), so each row's run of zeros
+    can be set exactly.  Rows whose zeros end just before the lower middle element, between
+    the two middle elements, and just after the upper one, in two segments and over all of
+    P: the targets that the commit kernel's counts resolve and the ones a selection pass
+    finds must together equal the oracle's sorted medians bit for bit."""
+    rng = np.random.default_rng(P)
+    half = P // 2
+    seg = [0, half, P]
+    rows = []
+    for zl, zr in ((half // 2 - 1, half // 2), (half // 2, (P - half) // 2 + 1), (half // 2 + 1, 0),
+                   (0, P - half), (half, (P - half) // 2 - 1), (3, 5)):
+        g = (0.1 * rng.standard_normal(P) + 0.3).astype(np.float32)
+        g[g == 0] = 0.5
+        g[rng.choice(half, zl, replace=False)] = 0.0
+        g[half + rng.choice(P - half, zr, replace=False)] = 0.0
+        rows.append(g)
+    grads = np.stack(rows)
+    T = grads.shape[0]
+    order = np.zeros(T, np.int32)
+    theta0 = (0.05 * rng.standard_normal(P)).astype(np.float32)
+    th, m, s = theta0.copy(), np.zeros((1, P), np.float32), theta0.copy()[None, :]
+    ref_pi = oracle.gem_run(th, m, s, grads, order, eta=ETA, mu=0.0, eps=EPS, record_pi=True)
+    for k in range(T):                    # the construction holds in the oracle
+        assert np.array_equal(ref_pi[k] == 0, grads[k] == 0) and np.all(ref_pi[k] >= 0)
+    g_dev = _padded(grads)
+    pi = torch.empty((T, (P + 3) // 4 * 4), device="cuda")
+    for sg in (seg, [0, P]):
+        nseg = len(sg) - 1
+        lo, hi = torch.empty((T, nseg), device="cuda"), torch.empty((T, nseg), device="cuda")
+        with gem.Gem(P, 1, ETA, 0.0, EPS) as G:
+            G.set_theta(torch.from_numpy(theta0).cuda())
+            G.commit_batch_pi_median(order.tolist(), [g_dev[k, :P] for k in range(T)],
+                                     [pi[k, :P] for k in range(T)], sg, lo, hi)
+            G.sync()
+            assert np.array_equal(G.theta().cpu().numpy(), th)
+        glo, ghi = lo.cpu().numpy(), hi.cpu().numpy()
+        for k in range(T):
+            rlo, rhi = oracle.pi_median(ref_pi[k], sg)
+            assert np.array_equal(glo[k].view(np.uint32), rlo.view(np.uint32)), (sg, k, glo[k], rlo)
+            assert np.array_equal(ghi[k].view(np.uint32), rhi.view(np.uint32)), (sg, k, ghi[k], rhi)
+
+
+def test_fused_medians_with_64_segments_in_chunks():
+    """64 segments allow 32 commits per chunk (the counters of a launch live in shared
+    memory): 100 commits in four chunks, medians bit for bit against the oracle."""
+    P, n, T = 70_001, 7, 100
+    theta0, grads, order, tau = _inputs(P, n, T, 64)
+    seg = np.linspace(0, P, 65).astype(np.int64).tolist()
+    th, m, s = theta0.copy(), np.zeros((n, P), np.float32), np.tile(theta0, (n, 1))
+    ref_pi = oracle.gem_run(th, m, s, grads, order, eta=ETA, mu=MU, eps=EPS, record_pi=True)
+    g_dev = _padded(grads)
+    pi = torch.empty((T, (P + 3) // 4 * 4), device="cuda")
+    lo, hi = torch.empty((T, 64), device="cuda"), torch.empty((T, 64), device="cuda")
+    with gem.Gem(P, n, ETA, MU, EPS) as G:
+        G.set_theta(torch.from_numpy(theta0).cuda())
+        G.commit_batch_pi_median(order.tolist(), [g_dev[k, :P] for k in range(T)],
+                                 [pi[k, :P] for k in range(T)], seg, lo, hi)
+        G.sync()
+        assert np.array_equal(G.theta().cpu().numpy(), th)
+    glo, ghi = lo.cpu().numpy(), hi.cpu().numpy()
+    for k in range(T):
+        rlo, rhi = oracle.pi_median(ref_pi[k], seg)
+        assert np.array_equal(glo[k], rlo) and np.array_equal(ghi[k], rhi), k
