@@ -46,11 +46,15 @@ RULE_BYTES = {0: 20, 1: 8, 2: 8, 3: 20, 4: 20, 5: 16}
 BYTES_PER_BATCH = P_FULL * (20 * K_BATCH + 8)
 FALLBACK_HBM_GBS = 6800.0
 
-# DRAM traffic of one launch of the batched commit kernel, from an ncu capture of the
-# same workload (see profiles/commit_batch_p25m_n100.md).  Valid only for the kernel
-# source it was taken on; reported as null once that source changes.
-NCU_TRAFFIC_BYTES_PER_LAUNCH = 40_243_673_600   # mean of two full-size launches
-NCU_TRAFFIC_SOURCE_SHA = "afca98bcd378a8a1"
+# DRAM traffic (bytes read + written) of one launch of the batched commit kernel at the
+# full workload size, from an ncu capture of dram__bytes_read.sum and dram__bytes_write.sum
+# on a smaller case of the same workload (P = 5,000,000, n = 100, batches of 100: about 6 GB
+# on the device), scaled by P: the traffic per coordinate does not depend on P (captures at
+# P = 2,500,000 and 5,000,000 agree within 1%).  Valid only for the kernel source it was
+# taken on (NCU_TRAFFIC_SOURCE_SHA, a hash of the kernel's sources); null once that changes.
+NCU_TRAFFIC_BYTES_PER_LAUNCH = 5 * (8_138_659_840 + 7_833_025_792) // 2   # mean of two launches at P = 5M
+NCU_TRAFFIC_SOURCE_SHA = "368c534035347631"
+NCU_TRAFFIC_HOW = "two launches captured at P=5,000,000 (n=100, K=100), scaled by P to 25,000,000"
 
 
 def kernel_source_sha() -> str:
@@ -278,27 +282,53 @@ def oracle_mlp_rates(seconds_target: float = 4.0) -> dict:
     return out
 
 
-def cpu_baseline(seconds_target: float = 15.0) -> dict:
+def host_threads() -> int:
+    """Host cores available to this process (the oracle's OpenMP thread count)."""
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count() or 1
+
+
+def cpu_baseline(seconds_target: float = 12.0) -> dict:
+    """The oracle's commit loop on a bounded sample of the workload, once on every host
+    core (its coordinates split across threads, which changes no result) and once on one
+    thread, plus the oracle's end-to-end MLP rates."""
     import oracle
-    sample = OracleSample(ORACLE_SAMPLE, SEED)
-    dt1 = sample.run(1)
-    batches = max(1, min(150, int(seconds_target / max(dt1, 1e-3))))
-    dt = sample.run(batches)
-    S, T = ORACLE_SAMPLE, batches * K_BATCH
-    gbs = S * (20 * T + 8 * batches) / dt / 1e9
-    return {"value": round(gbs, 3), "unit": "GB/s", "cores": 1, "kind": "oracle",
-            "sample": f"coordinates [0, {S}) of P={P_FULL}, n={N_WORKERS}: {batches} batches of "
-                      f"{K_BATCH} commits in {dt:.1f} s; same algorithmic bytes per coordinate",
-            "commits_per_s_scaled_to_P": round(T / dt * S / P_FULL, 3),
-            "oracle_threads_available": oracle.threads(),
-            "async_mlp_oracle": oracle_mlp_rates()}
+    cores = host_threads()
+    out = {}
+    for threads in (cores, 1):
+        prev = oracle.set_commit_threads(threads)
+        try:
+            sample = OracleSample(ORACLE_SAMPLE, SEED)
+            dt1 = sample.run(1)
+            batches = max(1, min(150, int(seconds_target / max(dt1, 1e-3))))
+            dt = sample.run(batches)
+        finally:
+            oracle.set_commit_threads(prev)
+        S, T = ORACLE_SAMPLE, batches * K_BATCH
+        gbs = S * (20 * T + 8 * batches) / dt / 1e9
+        out[threads] = {"value": round(gbs, 3), "unit": "GB/s", "cores": threads, "kind": "oracle",
+                        "sample": f"coordinates [0, {S}) of P={P_FULL}, n={N_WORKERS}: {batches} batches "
+                                  f"of {K_BATCH} commits in {dt:.1f} s on {threads} thread(s); same "
+                                  "algorithmic bytes per coordinate",
+                        "commits_per_s_scaled_to_P": round(T / dt * S / P_FULL, 3)}
+    line = dict(out[cores])
+    if cores != 1:
+        line["single_thread"] = out[1]
+    line["oracle_threads_available"] = oracle.threads()
+    line["async_mlp_oracle"] = oracle_mlp_rates()
+    return line
 
 
 def run_reference(args, world, rank, pg):
     """Reference arm: the oracle as it stands, on the host cores, one bounded sample per step."""
     if rank != 0:
         return
+    import oracle
     S = ORACLE_SAMPLE
+    cores = host_threads()
+    oracle.set_commit_threads(cores)
     sample = OracleSample(S, SEED, max_batches=args.warmup + args.steps + 1)
     for _ in range(args.warmup):
         sample.run(1)
@@ -312,8 +342,9 @@ def run_reference(args, world, rank, pg):
         "config": {"workload": "gem_commit_batch P=25M n=100, batches of 100 commits, heavy-tailed gradient pool",
                    "P": P_FULL, "n": N_WORKERS, "commits_per_step": K_BATCH,
                    "sample": f"coordinates [0, {S}) per step"},
-        "cpu_baseline": {"value": round(gbs, 3), "unit": "GB/s", "cores": 1, "kind": "oracle",
-                         "sample": f"coordinates [0, {S}) of P={P_FULL}, one batch of {K_BATCH} commits per step"},
+        "cpu_baseline": {"value": round(gbs, 3), "unit": "GB/s", "cores": cores, "kind": "oracle",
+                         "sample": f"coordinates [0, {S}) of P={P_FULL}, one batch of {K_BATCH} commits "
+                                   f"per step, the coordinates split over {cores} thread(s)"},
         "e2e": {"value": round(gbs, 3), "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
@@ -369,6 +400,34 @@ def run_gem(args, world, rank, local, pg):
         total_ms = starts[0].elapsed_time(ends[-1])
         total_ms = max_over_ranks(pg, total_ms)
         barrier(pg)
+        # the fewest bytes a batch can move: every gradient read once, theta read and
+        # written once, and m_w, s_w read and written once per distinct worker of the batch
+        distinct = [len(set(o)) for o, _g in batches]
+        reuse_min_bytes = P_FULL * (4 * K_BATCH + 8 + 16 * sum(distinct) / len(distinct))
+
+        # single commits (one gem_commit call each, 28 bytes per parameter: g, m_w, s_w and
+        # theta read, m_w, s_w and theta written) on the same state, back to back
+        single = None
+        if not args.no_single:
+            n_single = max(20, min(4 * args.steps, 200))
+            singles = [(int(order[k]), pool[k % POOL_ROWS]) for k in range(n_single)]
+            for w, g in singles[:5]:
+                G.commit(w, g)
+            stream.synchronize()
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            for w, g in singles:
+                G.commit(w, g)
+            e1.record(stream)
+            e1.synchronize()
+            ms_single = e0.elapsed_time(e1) / n_single
+            gbs_single = 28 * P_FULL / (ms_single * 1e-3) / 1e9
+            single = {"commits_per_s": round(1e3 / ms_single, 1), "ms_per_commit": round(ms_single, 5),
+                      "GB_per_s": round(gbs_single, 1), "commits": n_single,
+                      "bytes_per_param": 28, "kernel": "commit_batch_kernel (one commit per launch)",
+                      "note": "gem_commit calls back to back at P=25M, n=100; each launch waits on "
+                              "its predecessor, so ms_per_commit bounds the kernel time from above"}
 
         # the other commit rules on the same workload, each with its own algorithmic bytes
         rules = None
@@ -408,6 +467,19 @@ def run_gem(args, world, rank, local, pg):
             ev[-1].synchronize()
             commit_ms = sum(ev[3 * r].elapsed_time(ev[3 * r + 1]) for r in range(reps)) / reps
             select_ms = sum(ev[3 * r + 1].elapsed_time(ev[3 * r + 2]) for r in range(reps)) / reps
+            # the same batches through the fused call: the commit kernel counts each row's
+            # zeros, and rows whose medians lie in the run of zeros are not read again
+            flo = torch.empty((reps, K_BATCH, 1), device="cuda")
+            fhi = torch.empty((reps, K_BATCH, 1), device="cuda")
+            G.commit_batch_pi_median(*batch(reps + 1), rows, [0, P_FULL], flo[0], fhi[0])
+            fev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+            stream.synchronize()
+            fev[0].record(stream)
+            for r in range(reps):
+                G.commit_batch_pi_median(*batch(reps + 2 + r), rows, [0, P_FULL], flo[r], fhi[r])
+            fev[1].record(stream)
+            fev[1].synchronize()
+            fused_ms = fev[0].elapsed_time(fev[1]) / reps
             # bytes the selection needs: one pass of 4 bytes per factor for a row whose two
             # middle elements lie in its run of exact +0 (resolved by the first pass), three
             # passes otherwise
@@ -426,7 +498,12 @@ def run_gem(args, world, rank, local, pg):
                                 "of exact +0, else 3",
                 "median_rows_in_one_pass": int(one_pass.sum()),
                 "median_rows": int(reps * K_BATCH),
-                "commits_per_s_with_median": round(K_BATCH / ((commit_ms + select_ms) * 1e-3), 1),
+                "commits_per_s_with_median_separate_calls": round(K_BATCH / ((commit_ms + select_ms) * 1e-3), 1),
+                "fused_ms": round(fused_ms, 4),
+                "commits_per_s_with_median": round(K_BATCH / (fused_ms * 1e-3), 1),
+                "fused_note": "gem_commit_batch_pi_median: factors recorded and their +0 counts taken "
+                              "by the commit kernel; rows whose medians lie in the run of zeros "
+                              "are not read again",
                 "median_pi_last_batch": float(lo[reps - 1, -1, 0]),
             }
             del pi_rows, rows
@@ -475,6 +552,9 @@ def run_gem(args, world, rank, local, pg):
     achieved = BYTES_PER_BATCH / (avg_launch_ms * 1e-3) / 1e9
     value = world * BYTES_PER_BATCH * args.steps / (total_ms * 1e-3) / 1e9
     traffic = NCU_TRAFFIC_BYTES_PER_LAUNCH if NCU_TRAFFIC_SOURCE_SHA == kernel_source_sha() else None
+    if single is not None:
+        single["frac_of_hbm_peak"] = round(single["GB_per_s"] / peak, 4)
+        single["frac_of_8tbs_nominal"] = round(single["GB_per_s"] / 8000.0, 4)
     line = {
         "metric": METRIC, "value": round(value, 1), "unit": "GB/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(total_ms / args.steps, 4),
@@ -493,7 +573,16 @@ def run_gem(args, world, rank, local, pg):
                      "frac": round(achieved / peak, 4), "traffic": traffic,
                      "peak_source": f"{peak_src} copy bandwidth (burst)",
                      "kernel": "commit_batch_kernel", "algorithmic_bytes_per_launch": BYTES_PER_BATCH,
-                     "launch_ms_min": round(min(per_step_ms), 4), "launch_ms_max": round(max(per_step_ms), 4)},
+                     "launch_ms_min": round(min(per_step_ms), 4), "launch_ms_max": round(max(per_step_ms), 4),
+                     # the DRAM rate the captured traffic implies, and the rate of the fewest
+                     # bytes a batch with its repeated workers can move, both against the peak
+                     "dram_frac": None if traffic is None else
+                     round(traffic / (avg_launch_ms * 1e-3) / 1e9 / peak, 4),
+                     "traffic_how": NCU_TRAFFIC_HOW,
+                     "reuse_min_bytes_per_launch": int(reuse_min_bytes),
+                     "reuse_min_frac": round(reuse_min_bytes / (avg_launch_ms * 1e-3) / 1e9 / peak, 4),
+                     "distinct_workers_per_batch": round(sum(distinct) / len(distinct), 2)},
+        "single_commit": single,
         "gpu_launches": int(launches),
         "commit_rules": rules,
         "pi_statistics": pi_stats,
@@ -726,6 +815,7 @@ def main():
     ap.add_argument("--no-mlp", action="store_true")
     ap.add_argument("--no-rules", action="store_true", help="skip timing the other commit rules")
     ap.add_argument("--no-flat", action="store_true", help="skip the flat P=1.2M single-commit run")
+    ap.add_argument("--no-single", action="store_true", help="skip the single commits at the full size")
     ap.add_argument("--only", choices=["all", "commit", "mlp", "cnn"], default="all",
                     help="profiling aid: run only the commit batches, the async MLP or CNN runs")
     ap.add_argument("--mlp-workload", default="",
@@ -760,6 +850,7 @@ def main():
                 args.no_mlp = True
                 args.no_flat = True
                 args.no_rules = True
+                args.no_single = True
             run_gem(args, world, rank, local, pg)
     if pg is not None:
         pg.destroy_process_group()
