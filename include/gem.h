@@ -226,6 +226,19 @@ int gem_commit_batch_pi_median(gem_t* h, const int* order, const float* const* g
                                float* const* pi, const int64_t* seg, int nseg, float* lo,
                                float* hi);
 
+/* Parameter sharding.  Every step of a commit is elementwise (Algorithm 1 applies Psi_GEM
+ * with an elementwise product, and pi is a per-parameter vector), so coordinate j of theta,
+ * m_w and s_w depends only on coordinate j of the gradients.  A parameter vector can
+ * therefore be split into contiguous shards, each held by its own handle (one per GPU, or
+ * several on one GPU), and committing the matching slice of every gradient to every shard
+ * gives, shard by shard, the same bits as one handle over all P: no data is exchanged
+ * between shards on the commit path.  This call gives shard `rank` of `world`:
+ * [*begin, *end) with boundaries on multiples of 32 floats (128 bytes), so the slice of a
+ * 16-byte-aligned gradient stays 16-byte aligned; shards differ in size by at most 32
+ * floats, and the last non-empty one ends at P.  A shard with *begin == *end holds nothing
+ * (world larger than P / 32, rounded up).  Host-only; needs no GPU. */
+int gem_shard_range(size_t P, int world, int rank, size_t* begin, size_t* end);
+
 /* Number of kernels this handle has launched since it was created. */
 uint64_t gem_launch_count(const gem_t* h);
 

@@ -46,6 +46,7 @@ def _declare(L):
         "gem_pi_median": ([p, p, i, p, i, p, p], i),
         "gem_commit_batch_pi_median": ([p, p, p, i, p, p, i, p, p], i),
         "gem_status_string": ([i], C.c_char_p),
+        "gem_shard_range": ([C.c_size_t, i, i, p, p], i),
         "gem_schedule_uniform": ([C.c_uint64, i, i, p, p], i),
         "gem_schedule_queue": ([C.c_uint64, i, i, C.c_double, p, p], i),
         "gem_plan_segments": ([p, i, i, p], i),

@@ -336,6 +336,18 @@ int gem_shape(const gem_t* h, size_t* P, int* n, size_t* stride) {
 
 uint64_t gem_launch_count(const gem_t* h) { return h ? h->launches : 0; }
 
+int gem_shard_range(size_t P, int world, int rank, size_t* begin, size_t* end) {
+  if (P < 1 || world < 1 || rank < 0 || rank >= world || !begin || !end) return GEM_EINVAL;
+  const size_t units = (P + gem::kStrideAlign - 1) / gem::kStrideAlign;   // 128-byte units
+  const size_t w = size_t(world), r = size_t(rank);
+  const size_t per = units / w, extra = units % w;
+  const size_t u0 = r * per + (r < extra ? r : extra);
+  const size_t u1 = u0 + per + (r < extra ? 1 : 0);
+  *begin = u0 * gem::kStrideAlign < P ? u0 * gem::kStrideAlign : P;
+  *end = u1 * gem::kStrideAlign < P ? u1 * gem::kStrideAlign : P;
+  return GEM_OK;
+}
+
 int gem_commit(gem_t* h, int worker, const float* grad) {
   int rc = check_handle(h);
   if (rc) return rc;

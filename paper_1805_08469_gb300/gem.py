@@ -195,6 +195,14 @@ def gem_load_state(h: int, theta=None, m=None, s=None) -> None:
                                C.c_void_p(_any_ptr(s))), "gem_load_state")
 
 
+def gem_shard_range(P: int, world: int, rank: int) -> tuple[int, int]:
+    """[begin, end) of parameter shard `rank` of `world` (contiguous, 128-byte boundaries);
+    host-only."""
+    b, e = C.c_size_t(), C.c_size_t()
+    check(lib().gem_shard_range(P, world, rank, C.byref(b), C.byref(e)), "gem_shard_range")
+    return int(b.value), int(e.value)
+
+
 def gem_sync(h: int) -> None:
     check(lib().gem_sync(C.c_void_p(h)), "gem_sync")
 
