@@ -59,8 +59,11 @@ typedef struct gem_mlp gem_mlp_t;
 enum gem_mlp_precision {
   GEM_MLP_FP32 = 0, /* fp32 products and sums */
   GEM_MLP_TF32 = 1  /* TF32 operands (10 explicit mantissa bits, round to nearest, ties
-                       away from zero), products exact in fp32, fp32 sums: the numerics of
-                       a TF32 tensor-core product, evaluated on the CUDA cores */
+                       away from zero), products exact in fp32, fp32 sums: on the
+                       tcgen05 tensor cores where both operands are K-major (forward
+                       products; weight gradients through transposed minibatch panels),
+                       on warp-level mma.sync for the input gradients, and on the CUDA
+                       cores, with the same rounding, below 32 rows or a K of 32 */
 };
 
 /* Bind an MLP to a GEM handle (its P must equal the MLP's parameter count).  batch is the
@@ -102,7 +105,10 @@ int gem_mlp_run(gem_mlp_t* mlp, const int32_t* order, int T, const int32_t* batc
 int gem_mlp_run_pi(gem_mlp_t* mlp, const int32_t* order, int T, const int32_t* batch_rows,
                    float* losses, float* pi_lo, float* pi_hi);
 
-/* Wait for the MLP's work on the handle's stream; GEM_ECUDA if device work failed. */
+/* Wait for the MLP's work on the handle's stream (and its second stream); GEM_ECUDA if
+ * device work failed or a tensor-core product reported an error: a wait on the tensor cores
+ * that gave up after its time limit, or a read or write outside its buffers that it
+ * skipped.  The handle is then unusable (GEM_ESTATE). */
 int gem_mlp_status(gem_mlp_t* mlp);
 
 /* Number of kernels the MLP has launched (gather, forward, loss, backward; the commits are

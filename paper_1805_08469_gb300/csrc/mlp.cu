@@ -31,6 +31,7 @@
 #include "gem_internal.h"
 #include "mlp_internal.h"
 #include "pdl.h"
+#include "tc_gemm.h"
 
 namespace gem {
 namespace mlp {
@@ -82,6 +83,12 @@ struct GemmArgs {
   int kchunk;
   float* ws;            // null: no split
   long long ws_floats;  // capacity of ws
+  // tensor-core path: floats addressable from each operand's base (0: unknown, which keeps
+  // the product off that path) and the error word its kernels report to
+  long long a_extent, b_extent, c_extent, bias_extent, mask_extent;
+  unsigned* status;
+  // tensor-core path only: operands already TF32 (not rounded again), C stored rounded
+  int a_rounded, b_rounded, round_c;
   int workers[kMaxGroups];
 };
 
@@ -856,13 +863,36 @@ bool launch_small_n(const GemmArgs& a, int groups, cudaStream_t st, cudaError_t*
 
 // Minibatch gather: slot g's rows X[batch_rows[g][r]] -> Xs[g][r][:].
 __global__ void gather_rows_kernel(const float* X, int d0, const int32_t* batch_rows, int b,
-                                   float* Xs, long long slot_stride) {
+                                   float* Xs, long long slot_stride, int round) {
   gem::pdl_entry();
   const int g = blockIdx.y, r = blockIdx.x;
   const long long row = batch_rows[(long long)g * b + r];
   const float* src = X + row * d0;
   float* dst = Xs + g * slot_stride + (long long)r * d0;
-  for (int k = threadIdx.x; k < d0; k += blockDim.x) dst[k] = src[k];
+  // with TF32 products the gathered rows are only ever operands: stored rounded once
+  for (int k = threadIdx.x; k < d0; k += blockDim.x) dst[k] = round ? to_tf32(src[k]) : src[k];
+}
+
+// dst[g] = transpose(src[g]) rounded to TF32: src [rows][cols] row-major, dst [cols][rows],
+// both at slot stride slot_stride; 32 x 32 tiles through shared memory (the weight-gradient
+// products read the minibatch panels K-major, with the batch as K).
+__global__ void __launch_bounds__(256) transpose_round_kernel(const float* src, float* dst, int rows,
+                                                              int cols, long long slot_stride) {
+  gem::pdl_entry();
+  __shared__ float tile[32][33];
+  const int g = blockIdx.z, c0 = blockIdx.x * 32, r0 = blockIdx.y * 32;
+  const float* s = src + g * slot_stride;
+  float* d = dst + g * slot_stride;
+  const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
+  for (int i = ty; i < 32; i += 8) {
+    const int r = r0 + i, c = c0 + tx;
+    tile[i][tx] = (r < rows && c < cols) ? to_tf32(s[(long long)r * cols + c]) : 0.f;
+  }
+  __syncthreads();
+  for (int i = ty; i < 32; i += 8) {
+    const int c = c0 + i, r = r0 + tx;
+    if (r < rows && c < cols) d[(long long)c * rows + r] = tile[tx][i];
+  }
 }
 
 // Softmax cross-entropy over C classes for the b rows of each slot: the mean loss, and the
@@ -989,14 +1019,45 @@ void launch_mma(const GemmArgs& a, int groups, cudaStream_t st) {
 // split-K workspace is given and K is long, up to kMaxSplit splits of K whose partial sums a
 // second kernel adds in a fixed order.
 template <bool AK, bool BK_, int EPI>
-cudaError_t launch_gemm(const GemmArgs& a_in, int groups, bool tf32, cudaStream_t st) {
+cudaError_t launch_gemm(const GemmArgs& a_in, int groups, bool tf32, cudaStream_t st,
+                        bool* on_tc = nullptr) {
   GemmArgs a = a_in;
+  if (on_tc) *on_tc = false;
   a.ksplit = 1;
   a.kchunk = a.K;
   // Products with fewer than 32 rows or a K below 32 (the last layer's weight and input
   // gradients) would leave a 128-row tensor-core tile mostly empty or its pipeline idle:
   // they run on the CUDA cores, with the same TF32 operand rounding.
   const bool tc = tf32 && a.M >= 32 && a.K >= 32;
+  if (tc && a.a_extent > 0 && a.b_extent > 0 && a.c_extent > 0) {
+    // the 5th-generation tensor cores (tcgen05, accumulator in tensor memory), for products
+    // whose layout, epilogue and alignment its kernel takes; the others stay on mma.sync
+    gem::tc::Args t;
+    std::memset(&t, 0, sizeof(t));
+    t.M = a.M;
+    t.N = a.N;
+    t.K = a.K;
+    t.A = gem::tc::Operand{a.A.base, a.A.group_stride, a.A.ld, a.a_extent, a.A.by_worker, a.a_rounded};
+    t.B = gem::tc::Operand{a.B.base, a.B.group_stride, a.B.ld, a.b_extent, a.B.by_worker, a.b_rounded};
+    t.C = a.C;
+    t.c_group_stride = a.c_group_stride;
+    t.ldc = a.ldc;
+    t.c_extent = a.c_extent;
+    t.round_c = a.round_c;
+    t.bias = a.bias;
+    t.bias_group_stride = a.bias_group_stride;
+    t.bias_extent = a.bias_extent;
+    t.mask = a.mask;
+    t.mask_group_stride = a.mask_group_stride;
+    t.ldmask = a.ldmask;
+    t.mask_extent = a.mask_extent;
+    t.status = a.status;
+    for (int g = 0; g < groups && g < kMaxGroups; ++g) t.workers[g] = a.workers[g];
+    if (gem::tc::supported(t, AK, BK_, EPI)) {
+      if (on_tc) *on_tc = true;
+      return gem::tc::launch(t, groups, AK, BK_, EPI, st);
+    }
+  }
   const long long mt = (a.M + 127) / 128, nt64 = (a.N + 63) / 64, nt128 = (a.N + 127) / 128;
   const long long big = (tc ? nt128 : nt64) * mt * groups;
   if (big >= (tc ? GEM_TF32_BIG_TILE_BLOCKS : GEM_SIMT_BIG_TILE_BLOCKS) * kSmCountHint) {
@@ -1072,7 +1133,7 @@ int mlp_chunk(gem_mlp* M, const int32_t* workers, int G, const int32_t* batch_ro
   int rc = GEM_OK;
   if (!M->external_input) {
     gem::launch_pdl(gather_rows_kernel, dim3(b, G), 256, 0, st, M->X, M->dims[0], batch_rows, b,
-                                                   scr + M->off_x, S);
+                                                   scr + M->off_x, S, tf32 ? 1 : 0);
     if ((rc = cuda_rc(cudaGetLastError()))) return rc;
     M->launches++;
   }
@@ -1082,7 +1143,46 @@ int mlp_chunk(gem_mlp* M, const int32_t* workers, int G, const int32_t* batch_ro
   for (int g = 0; g < G; ++g) a.workers[g] = workers[g];
   a.ws = M->ws;
   a.ws_floats = M->ws_floats;
+  a.status = M->tc_status;
   const long long wstride = (long long)h->stride;
+  // floats addressable from p when it lies in the scratch or in the snapshots (0 otherwise)
+  const float* snap_end = h->s + (long long)h->n * wstride;
+  auto ext = [&](const float* p) -> long long {
+    if (!p) return 0;
+    if (M->scratch_end && p >= M->scratch && p < M->scratch_end) return M->scratch_end - p;
+    if (p >= h->s && p < snap_end) return snap_end - p;
+    return 0;
+  };
+  // the operands, bias and mask of a product in the scratch or the snapshots, its output
+  // in the scratch or in the gradient rows (the region the product writes)
+  auto set_extents = [&](GemmArgs& x, int groups) {
+    x.a_extent = ext(x.A.base);
+    x.b_extent = ext(x.B.base);
+    x.bias_extent = ext(x.bias);
+    x.mask_extent = ext(x.mask);
+    x.c_extent = ext(x.C);
+    if (x.c_extent == 0)
+      x.c_extent = (long long)(groups - 1) * x.c_group_stride + (long long)(x.M - 1) * x.ldc + x.N;
+  };
+
+  // Which activations hold TF32 values already (tensor-core products then read them without
+  // rounding again): the gathered rows (rounded by the gather) and activations stored
+  // rounded by a tensor-core forward product.
+  bool act_rnd[kMaxLayers + 1] = {};
+  act_rnd[0] = tf32 && !M->external_input;
+  // Weight gradients dW_l = D_{l+1}^T A_l that run on the tensor cores read the minibatch
+  // panels K-major (K = the batch): TF32-rounded transposes A_l^T and D_{l+1}^T, each
+  // written once by transpose_round_kernel right after the panel itself.
+  auto t_dw = [&](int l) {
+    return M->has_t && l + 1 < L && M->dims[l + 1] >= 32 && b >= 32 && b % 4 == 0;
+  };
+  auto transpose = [&](const float* src, float* dst, int rows, int cols) -> int {
+    gem::launch_pdl(transpose_round_kernel, dim3((cols + 31) / 32, (rows + 31) / 32, G), 256, 0, st,
+                    src, dst, rows, cols, S);
+    M->launches++;
+    return cuda_rc(cudaGetLastError());
+  };
+  if (t_dw(0) && (rc = transpose(scr + M->off_x, scr + M->off_actT[0], b, M->dims[0]))) return rc;
 
   // forward
   bool fused_loss = false;   // the logits kernel also produced the loss gradient
@@ -1111,11 +1211,20 @@ int mlp_chunk(gem_mlp* M, const int32_t* workers, int G, const int32_t* batch_ro
       // the loss with its gradient in the same kernel
       fused_loss = true;
     } else {
-      e = last ? launch_gemm<true, true, kBias>(a, G, tf32, st)
-               : launch_gemm<true, true, kBiasRelu>(a, G, tf32, st);
+      set_extents(a, G);
+      a.a_rounded = act_rnd[l] ? 1 : 0;
+      a.b_rounded = 0;
+      a.round_c = (!last && tf32) ? 1 : 0;   // hidden activations: only ever operands and masks
+      bool on_tc = false;
+      e = last ? launch_gemm<true, true, kBias>(a, G, tf32, st, &on_tc)
+               : launch_gemm<true, true, kBiasRelu>(a, G, tf32, st, &on_tc);
+      if (!last) act_rnd[l + 1] = on_tc && a.round_c;
+      a.round_c = 0;
     }
     if ((rc = cuda_rc(e))) return rc;
     M->launches++;
+    if (!last && t_dw(l + 1) && (rc = transpose(act(l + 1), scr + M->off_actT[l + 1], b, dout)))
+      return rc;
   }
   if (!fused_loss) {
     gem::launch_pdl(softmax_xent_kernel, G, 128, 0, st, scr + M->off_logits, scr + M->off_delta[L], S,
@@ -1135,16 +1244,34 @@ int mlp_chunk(gem_mlp* M, const int32_t* workers, int G, const int32_t* batch_ro
       if ((rc = cuda_rc(cudaEventRecord(M->ev_delta[l + 1], st)))) return rc;
       if ((rc = cuda_rc(cudaStreamWaitEvent(wst, M->ev_delta[l + 1], 0)))) return rc;
     }
-    // dW_l = D_{l+1}^T A_l: (m = o, k = r) from D [b x dout], (k = r, n = j) from A [b x din]
+    // dW_l = D_{l+1}^T A_l: (m = o, k = r) from D [b x dout], (k = r, n = j) from A [b x din],
+    // or from the transposes D^T [dout x b] and A^T [din x b], both K-major and TF32
     GemmArgs w = a;
     w.M = dout; w.N = din; w.K = b;
-    w.A = Operand{scr + M->off_delta[l + 1], S, dout, 0};
-    w.B = Operand{act(l), S, din, 0};
+    w.round_c = 0;
     w.C = grads + M->w_off[l];
     w.c_group_stride = grad_stride;
     w.ldc = din;
     if (two_streams) w.ws = nullptr;
-    if ((rc = cuda_rc(launch_gemm<false, false, kStore>(w, G, tf32, wst)))) return rc;
+    w.bias = nullptr;
+    w.mask = nullptr;
+    cudaError_t ew;
+    if (t_dw(l)) {
+      w.A = Operand{scr + M->off_deltaT[l + 1], S, b, 0};
+      w.B = Operand{scr + M->off_actT[l], S, b, 0};
+      w.a_rounded = 1;
+      w.b_rounded = 1;
+      set_extents(w, G);
+      ew = launch_gemm<true, true, kStore>(w, G, tf32, wst);
+    } else {
+      w.A = Operand{scr + M->off_delta[l + 1], S, dout, 0};
+      w.B = Operand{act(l), S, din, 0};
+      w.a_rounded = 0;
+      w.b_rounded = 0;
+      set_extents(w, G);
+      ew = launch_gemm<false, false, kStore>(w, G, tf32, wst);
+    }
+    if ((rc = cuda_rc(ew))) return rc;
     M->launches++;
     if (l == 0) {
       if (!M->input_grad) break;
@@ -1155,6 +1282,9 @@ int mlp_chunk(gem_mlp* M, const int32_t* workers, int G, const int32_t* batch_ro
       a.C = scr + M->off_delta[0];
       a.c_group_stride = S;
       a.ldc = din;
+      a.bias = nullptr;
+      a.mask = nullptr;
+      set_extents(a, G);
       if ((rc = cuda_rc(launch_gemm<true, false, kStore>(a, G, tf32, st)))) return rc;
       M->launches++;
       break;
@@ -1169,8 +1299,15 @@ int mlp_chunk(gem_mlp* M, const int32_t* workers, int G, const int32_t* batch_ro
     a.mask = act(l);
     a.mask_group_stride = S;
     a.ldmask = din;
+    a.bias = nullptr;
+    a.a_rounded = 0;
+    a.b_rounded = 0;
+    a.round_c = 0;
+    set_extents(a, G);
     if ((rc = cuda_rc(launch_gemm<true, false, kMask>(a, G, tf32, st)))) return rc;
     M->launches++;
+    // D_l^T for the tensor-core weight gradient dW_{l-1} (on the side stream after the event)
+    if (t_dw(l - 1) && (rc = transpose(scr + M->off_delta[l], scr + M->off_deltaT[l], b, din))) return rc;
   }
   BiasGradArgs ba;
   std::memset(&ba, 0, sizeof(ba));
@@ -1231,12 +1368,28 @@ int mlp_build(gem_t* g, int n_layers, const int32_t* dims, int batch, int precis
   }
   M->off_row_loss = off;
   off += round32(batch);
+  if (precision == GEM_MLP_TF32 && !external_input) {
+    M->has_t = true;
+    for (int l = 0; l + 1 < n_layers; ++l) {   // A_l^T for the weight gradients dW_l, l < L - 1
+      M->off_actT[l] = off;
+      off += round32((long long)batch * dims[l]);
+    }
+    for (int l = 1; l < n_layers; ++l) {       // D_l^T, l = 1 .. L - 1
+      M->off_deltaT[l] = off;
+      off += round32((long long)batch * dims[l]);
+    }
+  }
   M->slot_stride = off;
   M->slots = g->n < kMaxGroups ? g->n : kMaxGroups;
   int dev_prev = 0;
   cudaGetDevice(&dev_prev);
   cudaSetDevice(g->device);
   cudaError_t e = cudaMalloc(&M->scratch, sizeof(float) * size_t(M->slot_stride) * M->slots);
+  if (e == cudaSuccess) M->scratch_end = M->scratch + M->slot_stride * M->slots;
+  if (e == cudaSuccess && precision == GEM_MLP_TF32) {
+    e = cudaMalloc(&M->tc_status, sizeof(unsigned));
+    if (e == cudaSuccess) e = cudaMemset(M->tc_status, 0, sizeof(unsigned));
+  }
   if (e == cudaSuccess && own_grads) e = cudaMalloc(&M->grads, sizeof(float) * g->stride * size_t(g->n));
   if (e == cudaSuccess && batch <= 128) {
     // split-K workspace: kMaxSplit partial products of at most batch x widest layer per slot
@@ -1271,6 +1424,7 @@ void mlp_free(gem_mlp* M) {
   if (M->ev_side) cudaEventDestroy(M->ev_side);
   if (M->side) cudaStreamDestroy(M->side);
   cudaFree(M->scratch);
+  cudaFree(M->tc_status);
   cudaFree(M->grads);
   cudaFree(M->ws);
   cudaFree(M->pi_rows);
@@ -1342,9 +1496,13 @@ int gem_mlp_status(gem_mlp_t* M) {
   int dev_prev = 0;
   cudaGetDevice(&dev_prev);
   cudaSetDevice(h->device);
-  const cudaError_t e = cudaStreamSynchronize(h->stream);
+  cudaError_t e = cudaStreamSynchronize(h->stream);
+  if (e == cudaSuccess && M->side) e = cudaStreamSynchronize(M->side);
+  unsigned tc = 0;   // a tensor-core product that gave up a wait or skipped an access
+  if (e == cudaSuccess && M->tc_status)
+    e = cudaMemcpy(&tc, M->tc_status, sizeof(unsigned), cudaMemcpyDeviceToHost);
   cudaSetDevice(dev_prev);
-  if (e != cudaSuccess) {
+  if (e != cudaSuccess || tc != 0) {
     h->broken = true;
     return GEM_ECUDA;
   }

@@ -40,9 +40,17 @@ struct gem_mlp {
   // D_l [b x d_l] (l = 1..L, and l = 0 with input_grad)
   long long off_x = 0, off_act[gem::mlp::kMaxLayers + 1] = {}, off_logits = 0, off_delta[gem::mlp::kMaxLayers + 1] = {};
   long long off_row_loss = 0;   // per-row losses of the minibatch [b] (fused loss)
+  // TF32 engine: TF32-rounded transposes of the minibatch panels that the weight-gradient
+  // products dW_l = D_{l+1}^T A_l read K-major: A_l^T [d_l x b] (X^T for l = 0) and
+  // D_{l+1}^T [d_{l+1} x b] (has_t: the layout holds them)
+  bool has_t = false;
+  long long off_actT[gem::mlp::kMaxLayers + 1] = {};
+  long long off_deltaT[gem::mlp::kMaxLayers + 1] = {};
   long long slot_stride = 0;
   int slots = 0;
   float* scratch = nullptr;
+  float* scratch_end = nullptr;   // one past the scratch (bounds of the tensor-core reads)
+  unsigned* tc_status = nullptr;  // error word of the tensor-core products (TF32), 0 = none
   float* grads = nullptr;  // [n][gem stride]
   float* ws = nullptr;     // split-K partial sums
   float* pi_rows = nullptr;  // [n][gem stride] scaling factors of a segment's commits

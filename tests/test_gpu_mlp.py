@@ -65,11 +65,16 @@ def rel_l2(a, b):
 # (softmax - onehot) to TF32 breaks its exact cancellation over the classes, so a 1-ulp fp32
 # change in a pre-activation moves them by up to 1%.  The oracle's own TF32 mode and its
 # fp64 mode differ by 1-2% there.  Those blocks get 1e-2; the last layer, which sees no
-# rounded delta, keeps a tight bar.  The spec TF32 bar is on the theta trajectory.
+# rounded delta, keeps a tighter bar.  Its operands are still the previous layer's
+# activations rounded to TF32, and where an fp32 sum lies near a TF32 rounding boundary the
+# rounding can go either way: with K = 1000 sums the last layer's weight gradient moves by
+# 4-5e-5 between double sums and fp32 pairwise sums, and by 1.1e-4 with the tensor cores'
+# accumulation, so the 784-1000-1000-10 network's bar there is 3e-4.  The spec TF32
+# bar is on the theta trajectory.
 @pytest.mark.parametrize("dims,b,precision,tol,deep_tol", [
     ([784, 64, 10], 32, sim.GEM_MLP_FP32, 1e-5, 1e-5),
     ([784, 1000, 1000, 10], 128, sim.GEM_MLP_FP32, 1e-5, 1e-5),
-    ([784, 1000, 1000, 10], 128, sim.GEM_MLP_TF32, 1e-4, 1e-2),
+    ([784, 1000, 1000, 10], 128, sim.GEM_MLP_TF32, 3e-4, 1e-2),
     ([37, 19, 5, 3], 7, sim.GEM_MLP_FP32, 1e-5, 1e-5),    # ragged: nothing is a multiple of a tile
     ([37, 19, 5, 3], 7, sim.GEM_MLP_TF32, 1e-4, 1e-2),
 ])
@@ -113,6 +118,7 @@ def _gradient_parity(dims, b, precision, tol, deep_tol, n, workers):
             G.sync()
             got = [g.cpu().numpy() for g in grads]
             got_loss = losses.cpu().numpy()
+            sim.gem_mlp_status(M)   # no product reported an error
         finally:
             sim.gem_mlp_destroy(M)
     Xh, yh, local = host_rows(seed, batches, d0, C)
@@ -146,6 +152,7 @@ def test_mlp_rejects_invalid_rows_and_shapes():
                 sim.gem_mlp_run(M, [2], np.zeros((1, 32), np.int32))   # worker out of range
             sim.gem_mlp_run(M, [1], np.zeros((1, 32), np.int32))       # still usable
             G.sync()
+            sim.gem_mlp_status(M)   # no product reported an error
         finally:
             sim.gem_mlp_destroy(M)
 
@@ -176,6 +183,7 @@ def _e2e(dims, n, b, T, seed, schedule, precision, record_at):
             G.sync()
             final = G.theta().cpu().numpy().copy()
             lh = losses.cpu().numpy()
+            sim.gem_mlp_status(M)   # no product reported an error
         finally:
             sim.gem_mlp_destroy(M)
     return np.array(recs), lh, final, (order, batches, theta0)
@@ -260,6 +268,7 @@ def _windows(dims, n, b, seed, schedule, precision, starts, W, tol):
                         assert close.mean() > 0.999, (c, w, "m last layer", close.mean())
                     assert rel_l2(G.snapshot(w).cpu().numpy(), s[w]) < tol, (c, w, "s")
                 np.testing.assert_allclose(losses.cpu().numpy(), ref_losses, rtol=10 * tol)
+            sim.gem_mlp_status(M)   # no product reported an error
         finally:
             sim.gem_mlp_destroy(M)
     return worst
