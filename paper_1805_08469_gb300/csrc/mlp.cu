@@ -87,8 +87,11 @@ struct GemmArgs {
   // the product off that path) and the error word its kernels report to
   long long a_extent, b_extent, c_extent, bias_extent, mask_extent;
   unsigned* status;
-  // tensor-core path only: operands already TF32 (not rounded again), C stored rounded
+  // tensor-core path only: operands already TF32 (not rounded again), C stored rounded,
+  // and an optional TF32-rounded transposed copy of C (ct: [N x M] per group, ld ldct)
   int a_rounded, b_rounded, round_c;
+  float* ct;
+  long long ct_group_stride, ldct, ct_extent;
   int workers[kMaxGroups];
 };
 
@@ -873,16 +876,28 @@ __global__ void gather_rows_kernel(const float* X, int d0, const int32_t* batch_
   for (int k = threadIdx.x; k < d0; k += blockDim.x) dst[k] = round ? to_tf32(src[k]) : src[k];
 }
 
-// dst[g] = transpose(src[g]) rounded to TF32: src [rows][cols] row-major, dst [cols][rows],
-// both at slot stride slot_stride; 32 x 32 tiles through shared memory (the weight-gradient
-// products read the minibatch panels K-major, with the batch as K).
-__global__ void __launch_bounds__(256) transpose_round_kernel(const float* src, float* dst, int rows,
-                                                              int cols, long long slot_stride) {
+// dst[g] = transpose(src[g]) rounded to TF32: src [rows][cols] row-major, dst [cols][rows];
+// src[g] at src + (by_worker ? workers[g] : g) * src_stride, dst[g] at dst + g * dst_stride.
+// 32 x 32 tiles through shared memory.  The tensor-core products read their operands
+// K-major: the weight gradients read the minibatch panels transposed (the batch as K), the
+// input gradients the weights transposed.
+struct TransposeArgs {
+  const float* src;
+  long long src_stride;
+  float* dst;
+  long long dst_stride;
+  int rows, cols;
+  int by_worker;
+  int workers[kMaxGroups];
+};
+
+__global__ void __launch_bounds__(256) transpose_round_kernel(const __grid_constant__ TransposeArgs t) {
   gem::pdl_entry();
   __shared__ float tile[32][33];
   const int g = blockIdx.z, c0 = blockIdx.x * 32, r0 = blockIdx.y * 32;
-  const float* s = src + g * slot_stride;
-  float* d = dst + g * slot_stride;
+  const int rows = t.rows, cols = t.cols;
+  const float* s = t.src + (t.by_worker ? (long long)t.workers[g] : (long long)g) * t.src_stride;
+  float* d = t.dst + g * t.dst_stride;
   const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
   for (int i = ty; i < 32; i += 8) {
     const int r = r0 + i, c = c0 + tx;
@@ -1044,6 +1059,10 @@ cudaError_t launch_gemm(const GemmArgs& a_in, int groups, bool tf32, cudaStream_
     t.ldc = a.ldc;
     t.c_extent = a.c_extent;
     t.round_c = a.round_c;
+    t.ct = a.ct;
+    t.ct_group_stride = a.ct_group_stride;
+    t.ldct = a.ldct;
+    t.ct_extent = a.ct_extent;
     t.bias = a.bias;
     t.bias_group_stride = a.bias_group_stride;
     t.bias_extent = a.bias_extent;
@@ -1053,7 +1072,7 @@ cudaError_t launch_gemm(const GemmArgs& a_in, int groups, bool tf32, cudaStream_
     t.mask_extent = a.mask_extent;
     t.status = a.status;
     for (int g = 0; g < groups && g < kMaxGroups; ++g) t.workers[g] = a.workers[g];
-    if (gem::tc::supported(t, AK, BK_, EPI)) {
+    if (gem::tc::supported(t, AK, BK_, EPI, groups)) {
       if (on_tc) *on_tc = true;
       return gem::tc::launch(t, groups, AK, BK_, EPI, st);
     }
@@ -1171,18 +1190,38 @@ int mlp_chunk(gem_mlp* M, const int32_t* workers, int G, const int32_t* batch_ro
   bool act_rnd[kMaxLayers + 1] = {};
   act_rnd[0] = tf32 && !M->external_input;
   // Weight gradients dW_l = D_{l+1}^T A_l that run on the tensor cores read the minibatch
-  // panels K-major (K = the batch): TF32-rounded transposes A_l^T and D_{l+1}^T, each
-  // written once by transpose_round_kernel right after the panel itself.
+  // panels K-major (K = the batch): TF32-rounded transposes A_l^T and D_{l+1}^T.  A hidden
+  // activation's transpose comes from the epilogue of the tensor-core product that makes it;
+  // X^T and the deltas' transposes from transpose_round_kernel on the side stream, next to
+  // the main stream's chain.
   auto t_dw = [&](int l) {
     return M->has_t && l + 1 < L && M->dims[l + 1] >= 32 && b >= 32 && b % 4 == 0;
   };
-  auto transpose = [&](const float* src, float* dst, int rows, int cols) -> int {
-    gem::launch_pdl(transpose_round_kernel, dim3((cols + 31) / 32, (rows + 31) / 32, G), 256, 0, st,
-                    src, dst, rows, cols, S);
+  TransposeArgs ta;
+  std::memset(&ta, 0, sizeof(ta));
+  for (int g = 0; g < G; ++g) ta.workers[g] = workers[g];
+  auto transpose = [&](cudaStream_t s, const float* src, long long src_stride, bool by_worker,
+                       float* dst, int rows, int cols) -> int {
+    ta.src = src;
+    ta.src_stride = src_stride;
+    ta.by_worker = by_worker ? 1 : 0;
+    ta.dst = dst;
+    ta.dst_stride = S;
+    ta.rows = rows;
+    ta.cols = cols;
+    gem::launch_pdl(transpose_round_kernel, dim3((cols + 31) / 32, (rows + 31) / 32, G), 256, 0, s, ta);
     M->launches++;
     return cuda_rc(cudaGetLastError());
   };
-  if (t_dw(0) && (rc = transpose(scr + M->off_x, scr + M->off_actT[0], b, M->dims[0]))) return rc;
+  const bool two_streams = M->side != nullptr;
+  cudaStream_t wst = two_streams ? M->side : st;
+  if (t_dw(0)) {   // X^T on the side stream, after the gather
+    if (two_streams) {
+      if ((rc = cuda_rc(cudaEventRecord(M->ev_x, st)))) return rc;
+      if ((rc = cuda_rc(cudaStreamWaitEvent(wst, M->ev_x, 0)))) return rc;
+    }
+    if ((rc = transpose(wst, scr + M->off_x, S, false, scr + M->off_actT[0], b, M->dims[0]))) return rc;
+  }
 
   // forward
   bool fused_loss = false;   // the logits kernel also produced the loss gradient
@@ -1215,16 +1254,28 @@ int mlp_chunk(gem_mlp* M, const int32_t* workers, int G, const int32_t* batch_ro
       a.a_rounded = act_rnd[l] ? 1 : 0;
       a.b_rounded = 0;
       a.round_c = (!last && tf32) ? 1 : 0;   // hidden activations: only ever operands and masks
+      const bool want_t = !last && t_dw(l + 1);
+      if (want_t) {
+        a.ct = scr + M->off_actT[l + 1];
+        a.ct_group_stride = S;
+        a.ldct = b;
+        a.ct_extent = ext(a.ct);
+      }
       bool on_tc = false;
       e = last ? launch_gemm<true, true, kBias>(a, G, tf32, st, &on_tc)
                : launch_gemm<true, true, kBiasRelu>(a, G, tf32, st, &on_tc);
       if (!last) act_rnd[l + 1] = on_tc && a.round_c;
       a.round_c = 0;
+      a.ct = nullptr;
+      if ((rc = cuda_rc(e))) return rc;
+      M->launches++;
+      if (want_t && !on_tc &&
+          (rc = transpose(st, act(l + 1), S, false, scr + M->off_actT[l + 1], b, dout)))
+        return rc;
+      continue;
     }
     if ((rc = cuda_rc(e))) return rc;
     M->launches++;
-    if (!last && t_dw(l + 1) && (rc = transpose(act(l + 1), scr + M->off_actT[l + 1], b, dout)))
-      return rc;
   }
   if (!fused_loss) {
     gem::launch_pdl(softmax_xent_kernel, G, 128, 0, st, scr + M->off_logits, scr + M->off_delta[L], S,
@@ -1236,8 +1287,6 @@ int mlp_chunk(gem_mlp* M, const int32_t* workers, int G, const int32_t* batch_ro
   // backward.  The weight-gradient products go to the side stream when there is one: each
   // waits for its delta D_{l+1} (event recorded on the main stream) and runs next to the
   // input-gradient chain; they use no split-K workspace, which belongs to the main stream.
-  const bool two_streams = M->side != nullptr;
-  cudaStream_t wst = two_streams ? M->side : st;
   for (int l = L - 1; l >= 0; --l) {
     const int din = M->dims[l], dout = M->dims[l + 1];
     if (two_streams) {
@@ -1257,6 +1306,9 @@ int mlp_chunk(gem_mlp* M, const int32_t* workers, int G, const int32_t* batch_ro
     w.mask = nullptr;
     cudaError_t ew;
     if (t_dw(l)) {
+      // D_{l+1}^T, on the weight-gradient stream (the input-gradient chain goes on)
+      if ((rc = transpose(wst, scr + M->off_delta[l + 1], S, false, scr + M->off_deltaT[l + 1], b, dout)))
+        return rc;
       w.A = Operand{scr + M->off_deltaT[l + 1], S, b, 0};
       w.B = Operand{scr + M->off_actT[l], S, b, 0};
       w.a_rounded = 1;
@@ -1292,13 +1344,13 @@ int mlp_chunk(gem_mlp* M, const int32_t* workers, int G, const int32_t* batch_ro
     // D_l = (D_{l+1} W_l) * [A_l > 0]: (m = r, k = o) from D, (k = o, n = j) from W_l [dout x din]
     a.M = b; a.N = din; a.K = dout;
     a.A = Operand{scr + M->off_delta[l + 1], S, dout, 0};
-    a.B = Operand{h->s + M->w_off[l], wstride, din, 1};
     a.C = scr + M->off_delta[l];
     a.c_group_stride = S;
     a.ldc = din;
     a.mask = act(l);
     a.mask_group_stride = S;
     a.ldmask = din;
+    a.B = Operand{h->s + M->w_off[l], wstride, din, 1};
     a.bias = nullptr;
     a.a_rounded = 0;
     a.b_rounded = 0;
@@ -1306,8 +1358,6 @@ int mlp_chunk(gem_mlp* M, const int32_t* workers, int G, const int32_t* batch_ro
     set_extents(a, G);
     if ((rc = cuda_rc(launch_gemm<true, false, kMask>(a, G, tf32, st)))) return rc;
     M->launches++;
-    // D_l^T for the tensor-core weight gradient dW_{l-1} (on the side stream after the event)
-    if (t_dw(l - 1) && (rc = transpose(scr + M->off_delta[l], scr + M->off_deltaT[l], b, din))) return rc;
   }
   BiasGradArgs ba;
   std::memset(&ba, 0, sizeof(ba));
@@ -1402,6 +1452,7 @@ int mlp_build(gem_t* g, int n_layers, const int32_t* dims, int batch, int precis
   for (int l = 0; l <= n_layers && e == cudaSuccess; ++l)
     e = cudaEventCreateWithFlags(&M->ev_delta[l], cudaEventDisableTiming);
   if (e == cudaSuccess) e = cudaEventCreateWithFlags(&M->ev_side, cudaEventDisableTiming);
+  if (e == cudaSuccess) e = cudaEventCreateWithFlags(&M->ev_x, cudaEventDisableTiming);
   cudaSetDevice(dev_prev);
   if (e != cudaSuccess) {
     cudaGetLastError();
@@ -1422,6 +1473,7 @@ void mlp_free(gem_mlp* M) {
   for (int l = 0; l <= kMaxLayers; ++l)
     if (M->ev_delta[l]) cudaEventDestroy(M->ev_delta[l]);
   if (M->ev_side) cudaEventDestroy(M->ev_side);
+  if (M->ev_x) cudaEventDestroy(M->ev_x);
   if (M->side) cudaStreamDestroy(M->side);
   cudaFree(M->scratch);
   cudaFree(M->tc_status);

@@ -60,6 +60,8 @@ struct gem_mlp {
   cudaStream_t side = nullptr;
   cudaEvent_t ev_delta[gem::mlp::kMaxLayers + 1] = {};
   cudaEvent_t ev_side = nullptr;
+  // ev_x: the minibatch rows gathered (main stream), for X^T on the side stream
+  cudaEvent_t ev_x = nullptr;
   int32_t* rows_dev = nullptr;  // minibatch rows uploaded from the host
   size_t rows_cap = 0;
   uint64_t launches = 0;
