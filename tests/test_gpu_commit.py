@@ -72,7 +72,9 @@ def test_single_commits_bitwise(P):
         assert G.launches() == T
 
 
-@pytest.mark.parametrize("P,n,K", [(4099, 5, 450), (64, 2, 37), (1_048_579, 16, 64)])
+# (250_003, 40, 200): more repeats open at once than on-chip slots (every slot in use), and a
+# last warp whose lanes run past the coordinates
+@pytest.mark.parametrize("P,n,K", [(4099, 5, 450), (64, 2, 37), (1_048_579, 16, 64), (250_003, 40, 200)])
 def test_batch_equals_sequence_bitwise(P, n, K):
     rng = np.random.default_rng(K)
     theta0 = (0.05 * rng.standard_normal(P)).astype(np.float32)

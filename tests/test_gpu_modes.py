@@ -72,11 +72,13 @@ def _assert_bitwise(G, th, m, s, n, what):
 
 
 @pytest.mark.parametrize("mode,omode,kappa", RULES)
-@pytest.mark.parametrize("P", [5, 4099, 262_147])
-def test_rule_batches_bitwise(mode, omode, kappa, P):
+@pytest.mark.parametrize("P,n", [(5, 6), (4099, 6), (262_147, 6), (262_147, 40)])
+def test_rule_batches_bitwise(mode, omode, kappa, P, n):
     """450 commits (three launches of at most 200) with repeated workers, against the
-    oracle's run of the same rule."""
-    n, T = 6, 450
+    oracle's run of the same rule.  With 40 workers a launch has more repeats open at once
+    than it has on-chip slots, so every slot (shared memory and registers) is in use, next
+    to repeats that go through global memory."""
+    T = 450
     theta0, grads, order, tau = _inputs(P, n, T, 1000 + P)
     th, m, s = theta0.copy(), np.zeros((n, P), np.float32), np.tile(theta0, (n, 1))
     oracle.gem_run(th, m, s, grads, order, eta=ETA, mu=MU, eps=EPS, tau=tau, mode=omode, kappa=kappa)
