@@ -52,8 +52,8 @@ FALLBACK_HBM_GBS = 6800.0
 # on the device), scaled by P: the traffic per coordinate does not depend on P (captures at
 # P = 2,500,000 and 5,000,000 agree within 1%).  Valid only for the kernel source it was
 # taken on (NCU_TRAFFIC_SOURCE_SHA, a hash of the kernel's sources); null once that changes.
-NCU_TRAFFIC_BYTES_PER_LAUNCH = 5 * (8_138_659_840 + 7_833_025_792) // 2   # mean of two launches at P = 5M
-NCU_TRAFFIC_SOURCE_SHA = "368c534035347631"
+NCU_TRAFFIC_BYTES_PER_LAUNCH = 5 * (7_721_927_168 + 7_477_507_584) // 2   # mean of two launches at P = 5M
+NCU_TRAFFIC_SOURCE_SHA = "d154547f74268928"
 NCU_TRAFFIC_HOW = "two launches captured at P=5,000,000 (n=100, K=100), scaled by P to 25,000,000"
 
 
@@ -567,6 +567,9 @@ def run_gem(args, world, rank, local, pg):
                    "l2": "inputs larger than L2 (about 30 GB working set), no flush",
                    "parallelism": f"{world} independent replica(s)"},
         "commits_per_s": round(world * K_BATCH * args.steps / (total_ms * 1e-3), 1),
+        "value_basis": "algorithmic bytes (20 B per parameter and commit + 8 B per parameter and "
+                       "batch) over the CUDA-event launch time; a repeated worker's m_w, s_w kept "
+                       "on chip count as moved, so the DRAM-based rate is roofline.dram_gbs",
         "frac_of_hbm_peak": round(value / world / peak, 4),
         "frac_of_8tbs_nominal": round(value / world / 8000.0, 4),
         "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
@@ -576,6 +579,8 @@ def run_gem(args, world, rank, local, pg):
                      "launch_ms_min": round(min(per_step_ms), 4), "launch_ms_max": round(max(per_step_ms), 4),
                      # the DRAM rate the captured traffic implies, and the rate of the fewest
                      # bytes a batch with its repeated workers can move, both against the peak
+                     "dram_gbs": None if traffic is None else
+                     round(traffic / (avg_launch_ms * 1e-3) / 1e9, 1),
                      "dram_frac": None if traffic is None else
                      round(traffic / (avg_launch_ms * 1e-3) / 1e9 / peak, 4),
                      "traffic_how": NCU_TRAFFIC_HOW,

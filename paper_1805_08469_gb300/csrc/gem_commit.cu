@@ -90,6 +90,21 @@ __device__ __forceinline__ void store_state(float4* p, float4 v) {
 #endif
 }
 
+// A store of m_w or s_w with the launch's L2 policy for it: kept in L2 ahead of other lines
+// (evict-last, `keep` the access policy made by createpolicy) when a later commit of the
+// launch reads it back, streamed (evict-first) at the worker's last commit of the launch.
+__device__ __forceinline__ void store_state_hint(float4* p, float4 v, int hint, uint64_t keep) {
+  if (hint == kL2Keep) {
+    asm volatile("st.global.L2::cache_hint.v4.f32 [%0], {%1, %2, %3, %4}, %5;" ::"l"(p), "f"(v.x),
+                 "f"(v.y), "f"(v.z), "f"(v.w), "l"(keep)
+                 : "memory");
+  } else if (hint == kL2Stream) {
+    __stcs(p, v);
+  } else {
+    store_state(p, v);
+  }
+}
+
 // The momentum-SGD proxy committed as is (Eq. momentum_update): m <- mu m + dtheta,
 // theta <- theta + m, s <- theta.
 __device__ __forceinline__ void commit_coord_momentum(float& theta, float& m, float& s, float g,
@@ -169,6 +184,11 @@ commit_batch_kernel(const __grid_constant__ BatchArgsT<KCAP> a) {
   const size_t tid = size_t(blockIdx.x) * kThreads + threadIdx.x;
   float4* theta4 = reinterpret_cast<float4*>(a.theta);
   const unsigned lane = threadIdx.x & 31u;
+  // L2 hints on the stores of m_w and s_w: launches of more than kSmallBatch commits
+  constexpr bool kHints = KCAP > kSmallBatch && RULE != kRuleFixed;
+  uint64_t keep_policy = 0;
+  if constexpr (kHints)
+    asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(keep_policy));
   // factor counters of this block (recording launches with counts only)
   unsigned* cnt = nullptr;
   if constexpr (REC) {
@@ -292,6 +312,7 @@ commit_batch_kernel(const __grid_constant__ BatchArgsT<KCAP> a) {
             pi = make_float4(nan, nan, nan, nan);
             if constexpr (kR > 0) {
               if (sout >= 0) put(sout, l, m[l], nullptr);
+              else if constexpr (kHints) store_state_hint(m4 + i, m[l], a.l2[k], keep_policy);
               else store_state(m4 + i, m[l]);
             } else {
               if (sout >= 0) slot_m(sout, l) = m[l];
@@ -307,6 +328,9 @@ commit_batch_kernel(const __grid_constant__ BatchArgsT<KCAP> a) {
                 slot_m(sout, l) = m[l];
                 slot_s(sout, l) = s[l];
               }
+            } else if constexpr (kHints) {
+              store_state_hint(m4 + i, m[l], a.l2[k], keep_policy);
+              store_state_hint(s4 + i, s[l], a.l2[k], keep_policy);
             } else {
               store_state(m4 + i, m[l]);
               store_state(s4 + i, s[l]);
@@ -500,6 +524,7 @@ cudaError_t launch_rule(const BatchArgs& a, int sm_count, cudaStream_t stream) {
     b.slot_in[k] = in ? a.slot_in[k] : int8_t(-1);
     b.slot_out[k] = in ? a.slot_out[k] : int8_t(-1);
     b.keep_s[k] = in ? a.keep_s[k] : uint8_t(1);
+    b.l2[k] = kL2Normal;   // no hints below kSmallBatch + 1 commits
   }
   return launch_kernel<RULE, REC, kSmallBatch>(b, slots, sm_count, stream);
 }
@@ -531,6 +556,7 @@ void plan_slots(BatchArgs& a) {
     a.slot_in[k] = -1;
     a.slot_out[k] = -1;
     a.keep_s[k] = next[k] < 0 ? 1 : 0;
+    a.l2[k] = next[k] < 0 ? kL2Stream : kL2Keep;   // a slot below makes it irrelevant
   }
   const int total = a.K > kSmallBatch ? kTotalSlots : kCommitSlots;   // see the kernel
   if (a.rule == kRuleFixed || total == 0) return;

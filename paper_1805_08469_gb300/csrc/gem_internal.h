@@ -66,8 +66,14 @@ struct BatchArgsT {
   int8_t slot_in[KCAP];
   int8_t slot_out[KCAP];
   uint8_t keep_s[KCAP];
+  // L2 policy of commit k's stores of m_w and s_w to global memory (launches of more than
+  // kSmallBatch commits, energy rules): kL2Keep when a later commit of the launch reads
+  // them back from global memory (no slot), kL2Stream at the worker's last commit of the
+  // launch, kL2Normal otherwise.
+  uint8_t l2[KCAP];
 };
 using BatchArgs = BatchArgsT<kMaxBatchPerLaunch>;
+enum L2Hint : uint8_t { kL2Normal = 0, kL2Keep = 1, kL2Stream = 2 };
 constexpr int kSmallBatch = 32;
 
 // Shared-memory slots of the commit kernel (m_w and s_w lanes of one worker per slot), and
@@ -88,7 +94,7 @@ constexpr int kRegSlots = GEM_COMMIT_REG_SLOTS;
 constexpr int kTotalSlots = kCommitSlots + kRegSlots;
 constexpr int kSlotMinDistance = GEM_COMMIT_SLOT_MIN_DISTANCE;
 
-// Fill slot_in, slot_out and keep_s of a launch from its a.K workers.
+// Fill slot_in, slot_out, keep_s and l2 of a launch from its a.K workers.
 void plan_slots(BatchArgs& a);
 
 // Launch the fused commit kernel for a.K commits on `stream`.
