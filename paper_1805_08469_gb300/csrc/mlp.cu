@@ -717,7 +717,8 @@ __global__ void __launch_bounds__(256) splitk_reduce_kernel(const __grid_constan
 // copies the worker's B (N x K, TF32-rounded when asked) into shared memory; then each warp
 // takes whole rows m: lane l accumulates k = l, l + 32, ... (coalesced A reads, conflict-free
 // shared reads), a fixed butterfly adds the 32 lane sums, and lane 0 writes the N outputs
-// of the row.  Deterministic.  rows_per_block rows per block.
+// of the row.  Deterministic.  rows_per_block rows per block; NC >= N classes compiled in
+// (16 or 32), so that a network with few classes carries no idle class slots.
 // The last layer's softmax cross-entropy, fused into the logits kernel (XENT): the lane
 // that finishes a row's logits z goes on, with the operations and order of
 // softmax_xent_kernel, to the row's loss gradient (softmax(z) - onehot(y)) / b and its
@@ -731,7 +732,7 @@ struct XentArgs {
   int b;
 };
 
-template <bool TF32, bool XENT>
+template <bool TF32, bool XENT, int NC>
 __global__ void __launch_bounds__(256)
 gemm_small_n_kernel(const __grid_constant__ GemmArgs p, int rows_per_block,
                     const __grid_constant__ XentArgs x) {
@@ -774,18 +775,19 @@ gemm_small_n_kernel(const __grid_constant__ GemmArgs p, int rows_per_block,
   const int r1 = min(p.M, r0 + rows_per_block);
   for (int m = r0 + warp; m < r1; m += 8) {
     const float* a = A + (long long)m * p.A.ld;
-    float acc[kMaxClasses];
+    float acc[NC];
 #pragma unroll
-    for (int n = 0; n < kMaxClasses; ++n) acc[n] = 0.f;
-#pragma unroll 4
+    for (int n = 0; n < NC; ++n) acc[n] = 0.f;
+    constexpr int kUnroll = NC <= 16 ? 8 : 4;   // A loads in flight within the register budget
+#pragma unroll kUnroll
     for (int k = lane; k < K; k += 32) {
       const float av = TF32 ? to_tf32(a[k]) : a[k];
 #pragma unroll
-      for (int n = 0; n < kMaxClasses; ++n)
+      for (int n = 0; n < NC; ++n)
         if (n < N) acc[n] = fmaf(av, Bsm[n * K + k], acc[n]);
     }
 #pragma unroll
-    for (int n = 0; n < kMaxClasses; ++n) {
+    for (int n = 0; n < NC; ++n) {
       if (n < N) {
 #pragma unroll
         for (int off = 16; off > 0; off >>= 1) acc[n] += __shfl_xor_sync(0xffffffffu, acc[n], off);
@@ -794,7 +796,7 @@ gemm_small_n_kernel(const __grid_constant__ GemmArgs p, int rows_per_block,
     if (lane == 0) {
       float* c = p.C + (long long)g * p.c_group_stride + (long long)m * p.ldc;
 #pragma unroll
-      for (int n = 0; n < kMaxClasses; ++n)
+      for (int n = 0; n < NC; ++n)
         if (n < N) {
           acc[n] = acc[n] + bias[n];   // the logit z_n
           c[n] = acc[n];
@@ -805,12 +807,12 @@ gemm_small_n_kernel(const __grid_constant__ GemmArgs p, int rows_per_block,
         if (bad_label) y = 0;
         float zmax = acc[0];
 #pragma unroll
-        for (int n = 1; n < kMaxClasses; ++n)
+        for (int n = 1; n < NC; ++n)
           if (n < N) zmax = fmaxf(zmax, acc[n]);
-        float e[kMaxClasses];
+        float e[NC];
         float sum = 0.f;
 #pragma unroll
-        for (int n = 0; n < kMaxClasses; ++n)
+        for (int n = 0; n < NC; ++n)
           if (n < N) {
             e[n] = expf(acc[n] - zmax);
             sum += e[n];
@@ -820,7 +822,7 @@ gemm_small_n_kernel(const __grid_constant__ GemmArgs p, int rows_per_block,
         float* d = x.delta + (long long)g * x.group_stride + (long long)m * N;
         float zy = acc[0];
 #pragma unroll
-        for (int n = 0; n < kMaxClasses; ++n)
+        for (int n = 0; n < NC; ++n)
           if (n < N) {
             d[n] = (e[n] / sum - (n == y ? 1.f : 0.f)) * inv_b + poison;
             if (n == y) zy = acc[n];
@@ -843,10 +845,16 @@ bool launch_small_n(const GemmArgs& a, int groups, cudaStream_t st, cudaError_t*
   int dev = 0;
   cudaGetDevice(&dev);
   if (bytes > 48 * 1024 && (dev < 0 || dev >= 64 || !configured[dev])) {
-    *err = cudaFuncSetAttribute(gemm_small_n_kernel<TF32, false>,
+    *err = cudaFuncSetAttribute(gemm_small_n_kernel<TF32, false, 16>,
                                 cudaFuncAttributeMaxDynamicSharedMemorySize, int(kMaxBytes));
     if (*err == cudaSuccess)
-      *err = cudaFuncSetAttribute(gemm_small_n_kernel<TF32, true>,
+      *err = cudaFuncSetAttribute(gemm_small_n_kernel<TF32, true, 16>,
+                                  cudaFuncAttributeMaxDynamicSharedMemorySize, int(kMaxBytes));
+    if (*err == cudaSuccess)
+      *err = cudaFuncSetAttribute(gemm_small_n_kernel<TF32, false, kMaxClasses>,
+                                  cudaFuncAttributeMaxDynamicSharedMemorySize, int(kMaxBytes));
+    if (*err == cudaSuccess)
+      *err = cudaFuncSetAttribute(gemm_small_n_kernel<TF32, true, kMaxClasses>,
                                   cudaFuncAttributeMaxDynamicSharedMemorySize, int(kMaxBytes));
     if (*err != cudaSuccess) return true;
     if (dev >= 0 && dev < 64) configured[dev] = true;
@@ -856,10 +864,14 @@ bool launch_small_n(const GemmArgs& a, int groups, cudaStream_t st, cudaError_t*
   rows_per_block = rows_per_block < 8 ? 8 : (rows_per_block + 7) / 8 * 8;
   const int rpb = int(rows_per_block);
   dim3 grid(unsigned((a.M + rpb - 1) / rpb), unsigned(groups));
-  if (xent)
-    gem::launch_pdl(gemm_small_n_kernel<TF32, true>, grid, 256, bytes, st, a, rpb, *xent);
-  else
-    gem::launch_pdl(gemm_small_n_kernel<TF32, false>, grid, 256, bytes, st, a, rpb, XentArgs{});
+  const XentArgs xa = xent ? *xent : XentArgs{};
+  if (a.N <= 16) {
+    if (xent) gem::launch_pdl(gemm_small_n_kernel<TF32, true, 16>, grid, 256, bytes, st, a, rpb, xa);
+    else gem::launch_pdl(gemm_small_n_kernel<TF32, false, 16>, grid, 256, bytes, st, a, rpb, xa);
+  } else {
+    if (xent) gem::launch_pdl(gemm_small_n_kernel<TF32, true, kMaxClasses>, grid, 256, bytes, st, a, rpb, xa);
+    else gem::launch_pdl(gemm_small_n_kernel<TF32, false, kMaxClasses>, grid, 256, bytes, st, a, rpb, xa);
+  }
   *err = cudaGetLastError();
   return true;
 }
