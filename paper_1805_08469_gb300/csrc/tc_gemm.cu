@@ -61,15 +61,15 @@ constexpr int kThreads = kRounders + kEpilogue + 64;
 constexpr unsigned long long kWaitNs = 2000000000ull;   // 2 s
 
 // Per tile width: the stages of the ring (one CTA per SM: the ring takes 192 KB, the
-// epilogue's transpose blocks 16.5 KB).
+// epilogue's transpose blocks 33 KB).
 template <int BN>
 struct Cfg {
   static constexpr int kStages = BN == 64 ? 8 : 6;
   static constexpr int kATile = kBM * kBK * 4;         // bytes
   static constexpr int kBTile = BN * kBK * 4;
   static constexpr int kStage = kATile + kBTile;       // multiple of 1024
-  static constexpr int kEpiAt = kStages * kStage;      // 4 warps x 32 x 33 floats
-  static constexpr int kBarrierAt = kEpiAt + 4 * 32 * 33 * 4;
+  static constexpr int kEpiAt = kStages * kStage;      // 8 warps x 32 x 33 floats
+  static constexpr int kBarrierAt = kEpiAt + 8 * 32 * 33 * 4;
   static constexpr int kSmem = kBarrierAt + 512 + 1024;   // barriers, slots; alignment slack
   static constexpr int kTmemCols = 2 * BN;             // two accumulators
 };
@@ -303,7 +303,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
     }
     for (int a = 0; a < 2; ++a) {
       bar_init(&acc_full[a], 1);
-      bar_init(&acc_empty[a], kEpilogue);
+      bar_init(&acc_empty[a], rounding ? kEpilogue : kEpilogue + kRounders);
     }
     bar_init(done, 1);
     *abort_flag = 0;
@@ -321,104 +321,17 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
 
   bool bad = false;
 
-  if (warp == kTmaWarp) {
-    // ---- tensor copies (one lane): k-block q is k-block q % nkb of tile q / nkb
-    if (lane == 0) {
-      int za = 0, zb = 0, m0 = 0, n0 = 0;
-      long long q = 0;
-      for (; q < Q; ++q) {
-        if (aborted(abort_flag)) break;
-        const int s = int(q % S);
-        const long long use = q / S;
-        // the stage's previous k-block (q - kStages) must have been read by its MMAs
-        if (use > 0 && !bar_wait(&empty[s], uint32_t(use - 1) & 1u)) {
-          raise_abort(abort_flag, kWaitStage);
-          break;
-        }
-        const int kb = int(q % nkb);
-        if (kb == 0) {
-          int g;
-          tile_of(int(q / nkb), g, m0, n0);
-          za = p.A.by_worker ? p.workers[g] : g;
-          zb = p.B.by_worker ? p.workers[g] : g;
-        }
-        const uint32_t at = smem_addr(sm + s * C::kStage);
-        bar_arrive_expect(&loaded[s], uint32_t(C::kStage));
-        tma_load_3d(at, &kp.ta, kb * kBK, m0, za, &loaded[s]);
-        tma_load_3d(at + C::kATile, &kp.tb, kb * kBK, n0, zb, &loaded[s]);
-      }
-      *loads_slot = int(q);
-    }
-  } else if (warp < kRounders / 32) {
-    // ---- rounding of the operands that are not TF32 yet
-    if (rounding) {
-      for (long long q = 0; q < Q; ++q) {
-        const int s = int(q % S);
-        if (s % (kRounders / 32) != warp) continue;
-        if (aborted(abort_flag)) break;
-        if (!__all_sync(0xffffffffu, bar_wait(&loaded[s], uint32_t(q / S) & 1u))) {
-          raise_abort(abort_flag, kWaitStage);
-          break;
-        }
-        const uint32_t at = smem_addr(sm + s * C::kStage);
-        if (kp.round_a) round_tile<kBM * kBK>(at, lane);
-        if (kp.round_b) round_tile<BN * kBK>(at + C::kATile, lane);
-        fence_smem_to_async();
-        bar_arrive(&full[s]);
-      }
-    }
-  } else if (warp == kMmaWarp) {
-    // ---- MMA issue (one lane)
-    if (lane == 0) {
-      constexpr uint32_t idesc = idesc_tf32(kBM, BN);
-      uint64_t* ready = rounding ? full : loaded;
-      long long q = 0;
-      int issued = 0, tiles = 0;
-      for (int i = 0; i < my_tiles; ++i) {
-        if (aborted(abort_flag)) break;
-        const int a = i & 1, ua = i >> 1;
-        // the accumulator's previous tile (i - 2) has been read by the epilogue
-        if (ua > 0 && !bar_wait(&acc_empty[a], uint32_t(ua - 1) & 1u)) {
-          raise_abort(abort_flag, kWaitStage);
-          break;
-        }
-        fence_after_sync();
-        const uint32_t d = tmem + uint32_t(a * BN);
-        bool ok = true;
-        for (int kb = 0; kb < nkb; ++kb, ++q) {
-          const int s = int(q % S);
-          if (aborted(abort_flag) || !bar_wait(&ready[s], uint32_t(q / S) & 1u)) {
-            raise_abort(abort_flag, kWaitStage);
-            ok = false;
-            break;
-          }
-          fence_after_sync();
-          const uint32_t a_addr = smem_addr(sm + s * C::kStage);
-          const uint32_t b_addr = a_addr + C::kATile;
-#pragma unroll
-          for (int kk = 0; kk < kBK / 8; ++kk)
-            mma_tf32(d, slice_desc(a_addr, kk), slice_desc(b_addr, kk), idesc, (kb | kk) != 0 ? 1u : 0u);
-          commit_to(&empty[s]);
-          issued = int(q) + 1;
-        }
-        if (!ok) break;
-        commit_to(&acc_full[a]);
-        tiles = i + 1;
-      }
-      // every MMA issued so far has completed once `done` does (also after an abort)
-      commit_to(done);
-      *issued_slot = issued;
-      *tiles_slot = tiles;
-    }
-  } else {
-    // ---- epilogue: warp 4 + quad holds rows m0 + 32 quad + lane of the tile in tensor
-    // memory.  Per 32-column block the epilogue's arithmetic runs in registers (lane = row);
-    // C^T is stored straight from them (lanes hold consecutive rows: whole rows of C^T), and
-    // C goes through a 32 x 33 transpose in shared memory, so that lane l stores column
-    // nb + l of each row (whole row segments).  Shared memory is reached through explicit
-    // shared-space loads and stores, so that no access waits on a global store.
+  // ---- epilogue: the warp with quad = warp % 4 holds rows m0 + 32 quad + lane of the tile
+  // in tensor memory and takes the 32-column blocks c_first, c_first + c_step, ...  Per
+  // block the epilogue's arithmetic runs in registers (lane = row); C^T is stored straight
+  // from them (lanes hold consecutive rows: whole rows of C^T), and C goes through a 32 x 33
+  // transpose in shared memory, so that lane l stores column nb + l of each row (whole row
+  // segments).  Shared memory is reached through explicit shared-space loads and stores, so
+  // that no access waits on a global store.  Warps 4-7 take every block; when no operand
+  // needs rounding, warps 0-3 share the blocks with them (even and odd blocks).
+  auto epilogue = [&](int c_first, int c_step, int warp_slot) {
     const int quad = warp & 3;
-    const uint32_t stg = smem_addr(epi_stage + quad * (32 * 33));
+    const uint32_t stg = smem_addr(epi_stage + warp_slot * (32 * 33));
     for (int i = 0; i < my_tiles; ++i) {
       // warp-uniform decisions: tensor-memory loads are warp-wide
       if (__any_sync(0xffffffffu, aborted(abort_flag) != 0)) break;
@@ -437,7 +350,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
       const long long mask_row = EPI == kMask ? (long long)g * p.mask_group_stride + (long long)m_lane * p.ldmask : 0;
       const long long ct_goff = (long long)g * p.ct_group_stride;
 #pragma unroll 1
-      for (int c = 0; c < BN / 32; ++c) {
+      for (int c = c_first; c < BN / 32; c += c_step) {
         const int nb = n0 + c * 32;
         if (nb >= p.N) break;   // the same for the whole warp
         float v[32];
@@ -528,6 +441,101 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
       fence_before_sync();
       bar_arrive(&acc_empty[a]);
     }
+    };
+
+  if (warp == kTmaWarp) {
+    // ---- tensor copies (one lane): k-block q is k-block q % nkb of tile q / nkb
+    if (lane == 0) {
+      int za = 0, zb = 0, m0 = 0, n0 = 0;
+      long long q = 0;
+      for (; q < Q; ++q) {
+        if (aborted(abort_flag)) break;
+        const int s = int(q % S);
+        const long long use = q / S;
+        // the stage's previous k-block (q - kStages) must have been read by its MMAs
+        if (use > 0 && !bar_wait(&empty[s], uint32_t(use - 1) & 1u)) {
+          raise_abort(abort_flag, kWaitStage);
+          break;
+        }
+        const int kb = int(q % nkb);
+        if (kb == 0) {
+          int g;
+          tile_of(int(q / nkb), g, m0, n0);
+          za = p.A.by_worker ? p.workers[g] : g;
+          zb = p.B.by_worker ? p.workers[g] : g;
+        }
+        const uint32_t at = smem_addr(sm + s * C::kStage);
+        bar_arrive_expect(&loaded[s], uint32_t(C::kStage));
+        tma_load_3d(at, &kp.ta, kb * kBK, m0, za, &loaded[s]);
+        tma_load_3d(at + C::kATile, &kp.tb, kb * kBK, n0, zb, &loaded[s]);
+      }
+      *loads_slot = int(q);
+    }
+  } else if (warp < kRounders / 32) {
+    // ---- rounding of the operands that are not TF32 yet, else half of the epilogue
+    if (!rounding) {
+      epilogue(0, 2, warp);   // staging buffers 0-3 (the epilogue warps use 4-7)
+    } else {
+      for (long long q = 0; q < Q; ++q) {
+        const int s = int(q % S);
+        if (s % (kRounders / 32) != warp) continue;
+        if (aborted(abort_flag)) break;
+        if (!__all_sync(0xffffffffu, bar_wait(&loaded[s], uint32_t(q / S) & 1u))) {
+          raise_abort(abort_flag, kWaitStage);
+          break;
+        }
+        const uint32_t at = smem_addr(sm + s * C::kStage);
+        if (kp.round_a) round_tile<kBM * kBK>(at, lane);
+        if (kp.round_b) round_tile<BN * kBK>(at + C::kATile, lane);
+        fence_smem_to_async();
+        bar_arrive(&full[s]);
+      }
+    }
+  } else if (warp == kMmaWarp) {
+    // ---- MMA issue (one lane)
+    if (lane == 0) {
+      constexpr uint32_t idesc = idesc_tf32(kBM, BN);
+      uint64_t* ready = rounding ? full : loaded;
+      long long q = 0;
+      int issued = 0, tiles = 0;
+      for (int i = 0; i < my_tiles; ++i) {
+        if (aborted(abort_flag)) break;
+        const int a = i & 1, ua = i >> 1;
+        // the accumulator's previous tile (i - 2) has been read by the epilogue
+        if (ua > 0 && !bar_wait(&acc_empty[a], uint32_t(ua - 1) & 1u)) {
+          raise_abort(abort_flag, kWaitStage);
+          break;
+        }
+        fence_after_sync();
+        const uint32_t d = tmem + uint32_t(a * BN);
+        bool ok = true;
+        for (int kb = 0; kb < nkb; ++kb, ++q) {
+          const int s = int(q % S);
+          if (aborted(abort_flag) || !bar_wait(&ready[s], uint32_t(q / S) & 1u)) {
+            raise_abort(abort_flag, kWaitStage);
+            ok = false;
+            break;
+          }
+          fence_after_sync();
+          const uint32_t a_addr = smem_addr(sm + s * C::kStage);
+          const uint32_t b_addr = a_addr + C::kATile;
+#pragma unroll
+          for (int kk = 0; kk < kBK / 8; ++kk)
+            mma_tf32(d, slice_desc(a_addr, kk), slice_desc(b_addr, kk), idesc, (kb | kk) != 0 ? 1u : 0u);
+          commit_to(&empty[s]);
+          issued = int(q) + 1;
+        }
+        if (!ok) break;
+        commit_to(&acc_full[a]);
+        tiles = i + 1;
+      }
+      // every MMA issued so far has completed once `done` does (also after an abort)
+      commit_to(done);
+      *issued_slot = issued;
+      *tiles_slot = tiles;
+    }
+  } else {
+    epilogue(rounding ? 0 : 1, rounding ? 1 : 2, warp);
   }
 
   __syncthreads();
@@ -684,9 +692,11 @@ cudaError_t launch(const Args& a, int groups, bool a_kmajor, bool b_kmajor, int 
   if (groups < 1 || groups > kMaxGroups || a.M < 1 || a.N < 1 || a.K < 1 || !a.A.base ||
       !a.B.base || !a.C || !supported(a, a_kmajor, b_kmajor, epi, groups))
     return cudaErrorInvalidValue;
-  // 128-wide tiles when they still give every SM a tile (each k-block then feeds twice the
-  // MMA work per byte copied); otherwise 64-wide, which spreads a product with few tiles (a
-  // 128-row minibatch panel per worker) over more SMs
+  // 128-wide tiles when they still give every SM a tile (a k-block then feeds twice the MMA
+  // work for 4/3 of the bytes); otherwise 64-wide, which spreads a product with few tiles
+  // (a 128-row minibatch panel per worker) over more SMs: its weights come from DRAM, and
+  // more SMs pulling them finish sooner than fewer copying fewer bytes each (measured: the
+  // forward products of a 13-worker segment 29.7 us 64-wide, 36 us 128-wide)
   const long long tiles128 = (long long)((a.N + 127) / 128) * ((a.M + kBM - 1) / kBM) * groups;
   if (tiles128 >= 152) return launch_cfg<128>(a, groups, epi, stream);
   return launch_cfg<64>(a, groups, epi, stream);
