@@ -77,9 +77,20 @@ def rel_l2(a, b):
     ([784, 1000, 1000, 10], 128, sim.GEM_MLP_TF32, 3e-4, 1e-2),
     ([37, 19, 5, 3], 7, sim.GEM_MLP_FP32, 1e-5, 1e-5),    # ragged: nothing is a multiple of a tile
     ([37, 19, 5, 3], 7, sim.GEM_MLP_TF32, 1e-4, 1e-2),
+    # tensor-core products with partial tiles everywhere (72 and 40 outputs, K = 100 and 72);
+    # b = 48 reads the weight gradients' operands transposed, b = 50 does not
+    ([100, 72, 40, 10], 48, sim.GEM_MLP_TF32, 1e-4, 1e-2),
+    ([100, 72, 40, 10], 50, sim.GEM_MLP_TF32, 1e-4, 1e-2),
 ])
 def test_worker_gradients_match_oracle(dims, b, precision, tol, deep_tol):
     _gradient_parity(dims, b, precision, tol, deep_tol, 3, [0, 2, 1, 2])
+
+
+def test_tf32_gradients_of_a_wide_segment():
+    """Twenty workers in one call: the forward product 784 -> 1000 then has 160 tiles of 128
+    columns, enough for the tensor-core kernel's 128-wide tiles, whose 6-stage ring is
+    rounded to TF32 in shared memory (the weights), each stage by one warp."""
+    _gradient_parity([784, 1000, 10], 32, sim.GEM_MLP_TF32, 3e-4, 1e-2, 20, list(range(20)))
 
 
 @pytest.mark.parametrize("dims,b,precision,tol,deep_tol", [
