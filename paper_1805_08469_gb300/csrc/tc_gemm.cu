@@ -2,7 +2,7 @@
 //
 // A persistent kernel: one CTA per SM walks the 128 x BN output tiles t = blockIdx.x,
 // blockIdx.x + gridDim.x, ... of all groups (the workers of a segment), in k-blocks of 32
-// fp32 values (128 bytes per operand row).  Its warps have three roles that meet only at
+// fp32 values (128 bytes per operand row).  Its warps have four roles that meet only at
 // shared-memory barriers, so that the copies, the MMAs and the epilogue of consecutive
 // tiles overlap:
 //   - TMA (warp 9, one lane): each k-block of A (128 rows) and B (BN rows) is loaded with
@@ -18,26 +18,27 @@
 //     the A and/or B tile in place to TF32 (to nearest, ties away from zero: the operand
 //     values the rest of the library and the oracle use), makes its writes visible to the
 //     tensor cores' proxy and arrives on the stage's `full` barrier.  Without rounding the
-//     MMA lane waits on `loaded` itself.
+//     MMA lane waits on `loaded` itself, and these warps take half of the epilogue.
 //   - MMA (warp 8, one lane): per tile it takes accumulator buffer i % 2 (2 x BN columns of
 //     tensor memory, allocated by warp 8) once the epilogue has emptied it (`acc_empty`),
 //     issues four tcgen05.mma.cta_group::1.kind::tf32 per k-block (K = 8 each: the
 //     descriptors' start address advances 32 bytes; M = 128, N = BN, fp32 accumulation),
 //     frees each stage with tcgen05.commit on its `empty` barrier, and signals the tile's
 //     accumulator on `acc_full`.
-//   - epilogue (warps 4-7): warp 4 + q reads tensor-memory lanes 32 q .. 32 q + 31 (rows of
-//     the tile) with tcgen05.ld, 32 columns at a time; every block goes through a 32 x 33
-//     transpose in shared memory, so that a warp stores whole row segments (coalesced),
-//     after the epilogue's bias, ReLU or mask; stored rounded to TF32 where the caller asks
-//     (outputs that are only ever operands).  A transposed copy, rounded to TF32, goes back
-//     through the same shared-memory block, so that a warp stores whole columns of the tile
-//     as rows of C^T.  Then it releases the buffer on `acc_empty`.
+//   - epilogue (warps 4-7, and 0-3 when nothing is rounded): the warp with q = warp % 4
+//     reads tensor-memory lanes 32 q .. 32 q + 31 (rows of the tile) with tcgen05.ld, 32
+//     columns at a time, and applies the bias, ReLU or mask in registers (lane = row);
+//     C^T, rounded to TF32, is stored straight from the registers (lanes hold consecutive
+//     rows), C goes through a 32 x 33 transpose in shared memory so that a warp stores whole
+//     row segments, rounded to TF32 where the caller asks (outputs that are only ever
+//     operands).  Then it releases the buffer on `acc_empty`.
 // Before the CTA exits, every barrier has received the arrivals of the tensor cores' commits
-// (none is pending on shared memory that a later CTA may reuse) and warp 8 frees the tensor
-// memory.  Every wait gives up after a bounded time: it raises a shared abort flag that ends
-// every role's loop, the CTA still drains the MMAs it issued (bounded) and frees its tensor
-// memory, and the failure is reported in *status.  Every global access is checked against
-// the extent of its buffer.
+// and of the tensor copies (none is pending on shared memory that a later CTA may reuse) and
+// warp 8 frees the tensor memory.  Every wait gives up after a bounded time: it raises a
+// shared abort flag that ends every role's loop, the CTA still drains the MMAs it issued
+// (bounded) and frees its tensor memory, and the failure is reported in *status.  The tensor
+// copies' maps cover exactly what supported() checked against the operands' extents; every
+// other global access is checked against its buffer's extent.
 #include "tc_gemm.h"
 
 #include <cuda.h>
