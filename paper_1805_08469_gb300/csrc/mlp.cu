@@ -890,9 +890,9 @@ __global__ void gather_rows_kernel(const float* X, int d0, const int32_t* batch_
 
 // dst[g] = transpose(src[g]) rounded to TF32: src [rows][cols] row-major, dst [cols][rows];
 // src[g] at src + (by_worker ? workers[g] : g) * src_stride, dst[g] at dst + g * dst_stride.
-// 32 x 32 tiles through shared memory.  The tensor-core products read their operands
-// K-major: the weight gradients read the minibatch panels transposed (the batch as K), the
-// input gradients the weights transposed.
+// 32 x 32 tiles through shared memory.  The tensor-core products read both operands
+// K-major, so the weight gradients read the minibatch panels X and D transposed (the batch
+// as K); the hidden activations' transposes come from the forward products' epilogue.
 struct TransposeArgs {
   const float* src;
   long long src_stride;
