@@ -332,6 +332,10 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
   // needs rounding, warps 0-3 share the blocks with them (even and odd blocks).
   auto epilogue = [&](int c_first, int c_step, int warp_slot) {
     const int quad = warp & 3;
+    // plain stores (the weight gradients, which the commit reads next) are kept in L2 ahead
+    // of other lines (evict-last), the rest written through normally
+    uint64_t keep = 0;
+    if (EPI == kStore) asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(keep));
     const uint32_t stg = smem_addr(epi_stage + warp_slot * (32 * 33));
     for (int i = 0; i < my_tiles; ++i) {
       // warp-uniform decisions: tensor-memory loads are warp-wide
@@ -424,7 +428,14 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
         if (__all_sync(0xffffffffu, whole && c0 >= 0 && c0 + 31 * p.ldc + 31 < p.c_extent)) {
           float* dst = p.C + c0 + lane;
 #pragma unroll
-          for (int r = 0; r < 32; ++r) __stcg(dst + (long long)r * p.ldc, col[r]);
+          for (int r = 0; r < 32; ++r) {
+            if (EPI == kStore)
+              asm volatile("st.global.L2::cache_hint.f32 [%0], %1, %2;" ::"l"(dst + (long long)r * p.ldc),
+                           "f"(col[r]), "l"(keep)
+                           : "memory");
+            else
+              __stcg(dst + (long long)r * p.ldc, col[r]);
+          }
         } else if (n < p.N) {
 #pragma unroll
           for (int r = 0; r < 32; ++r) {
