@@ -68,7 +68,8 @@ enum gem_mlp_precision {
 
 /* Bind an MLP to a GEM handle (its P must equal the MLP's parameter count).  batch is the
  * per-worker minibatch b (1..1024); dims[L] <= 32 classes.  Allocates per-worker scratch
- * (activations and deltas) and one gradient buffer per worker on the handle's device. */
+ * (activations and deltas, and for GEM_MLP_TF32 their TF32 transposes) and one gradient
+ * buffer per worker on the handle's device. */
 int gem_mlp_create(gem_t* gem, int n_layers, const int32_t* dims, int batch, int precision,
                    gem_mlp_t** out);
 
